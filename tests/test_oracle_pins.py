@@ -1,0 +1,388 @@
+"""Pins of the CPU oracle against facts fixed outside the oracle itself.
+
+Each test checks one oracle function against a hand-derived value (golden
+files), a closed form from the paper, brute force on tiny inputs written as
+plain loops, or a special case that reduces to a library routine.  A plausible
+mistake in the oracle (dropped codebook, swapped index, transposed operand,
+wrong rounding, wrong tap order) fails at least one of them.
+"""
+
+import math
+import os
+import struct
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+from aq_synth import CONFIGS, ConvSpec, LinearSpec, make_conv, make_linear
+from oracle import aq_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _h(hexstr):
+    return np.frombuffer(struct.pack("<H", int(hexstr, 16)), dtype=np.float16)[0]
+
+
+def _read_golden(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            rows.append([p.strip() for p in line.split(";", 2)])
+    return rows
+
+
+# ----------------------------------------------------------------------------- decode
+def test_decode_rule_golden_values():
+    """Hand-derived fp32-sum-then-fp16 outcomes (Eq. 4 with the decode rule)."""
+    for entries, expected, why in _read_golden("decode_rule_fp16.txt"):
+        vals = [_h(e) for e in entries.split()]
+        M = len(vals)
+        cb = np.zeros((M, 256, 8), dtype=np.float16)
+        for m, v in enumerate(vals):
+            cb[m, 7, 3] = v                      # entry e=3 of codeword 7 in codebook m
+        codes = np.full((1, 1, M), 7, dtype=np.uint8)
+        W = O.decode_rule_f16(codes, cb)
+        got = int(W.view(np.uint16)[0, 3])
+        assert got == int(expected, 16), f"{entries}: got {got:04X}, want {expected} ({why})"
+        # the other 7 entries of the group are sums of zeros
+        assert np.all(W.view(np.uint16)[0, [0, 1, 2, 4, 5, 6, 7]] == 0)
+
+
+def test_decode_identity_bruteforce():
+    """Eq. 4: W-hat group i of row n = sum over m of codeword C^(m)[b[n,i,m]]."""
+    rng = np.random.default_rng(123)
+    N, G, M, g, B = 3, 4, 3, 8, 8
+    cb = rng.normal(0, 0.1, size=(M, 1 << B, g)).astype(np.float16)
+    codes = rng.integers(0, 1 << B, size=(N, G, M), dtype=np.uint8)
+    W = O.decode_f64(codes, cb)
+    assert W.shape == (N, G * g)
+    for n in range(N):
+        for i in range(G):
+            for e in range(g):
+                s = 0.0
+                for m in range(M):
+                    s += float(cb[m][int(codes[n][i][m])][e])
+                assert W[n][i * g + e] == pytest.approx(s, rel=0, abs=1e-15)
+
+
+def test_decode_codebook_order_and_element_index():
+    """Exactly representable books: W[n, 8i+e] = (b0 + e)/64 - (b1 + 2e)/128."""
+    cb = np.zeros((2, 256, 8), dtype=np.float16)
+    for c in range(256):
+        for e in range(8):
+            cb[0, c, e] = (c + e) / 64.0
+            cb[1, c, e] = -(c + 2 * e) / 128.0
+    rng = np.random.default_rng(5)
+    codes = rng.integers(0, 256, size=(5, 6, 2), dtype=np.uint8)
+    Wr = O.decode_rule_f16(codes, cb).astype(np.float64)
+    W64 = O.decode_f64(codes, cb)
+    for n in range(5):
+        for i in range(6):
+            b0, b1 = int(codes[n, i, 0]), int(codes[n, i, 1])
+            for e in range(8):
+                want = Fraction(b0 + e, 64) - Fraction(b1 + 2 * e, 128)
+                assert Fraction(W64[n, i * 8 + e]) == want
+                assert Fraction(float(Wr[n, i * 8 + e])) == want
+
+
+def test_decode_rule_matches_exact_sum_when_representable():
+    """If the exact sum is an fp16 value, the rule returns it bit for bit."""
+    cb = np.zeros((4, 256, 8), dtype=np.float16)
+    for m in range(4):
+        for c in range(256):
+            cb[m, c, :] = np.float16((c - 128) * (1 << m))   # integers <= 1024 in magnitude
+    rng = np.random.default_rng(9)
+    codes = rng.integers(0, 256, size=(4, 3, 4), dtype=np.uint8)
+    Wr = O.decode_rule_f16(codes, cb)
+    for n in range(4):
+        for i in range(3):
+            s = sum((int(codes[n, i, m]) - 128) * (1 << m) for m in range(4))
+            assert abs(s) <= 2048                          # exact in fp16
+            assert np.all(Wr[n, i * 8:(i + 1) * 8] == np.float16(s))
+
+
+def test_decode_kaq_grouping():
+    """Sec. 3.1.2: one group = the 9 taps of one (cout, cin) filter."""
+    rng = np.random.default_rng(3)
+    Cout, Cin, M = 2, 3, 2
+    cb = rng.normal(0, 0.1, size=(M, 16, 9)).astype(np.float16)
+    codes = rng.integers(0, 16, size=(Cout, Cin, M), dtype=np.uint8)
+    F = O.decode_kaq_f64(codes, cb)
+    for o in range(Cout):
+        for c in range(Cin):
+            for t in range(9):
+                s = float(cb[0, codes[o, c, 0], t]) + float(cb[1, codes[o, c, 1], t])
+                assert F[o, c, t] == pytest.approx(s, abs=1e-15)
+
+
+# ----------------------------------------------------------------------------- packing
+def test_pack_layout_positions():
+    """Packed byte index of code b[n, i, m]: ((kb*N + n)*8 + i%8)*M + m (8-bit codes)."""
+    rng = np.random.default_rng(1)
+    N, K, M = 5, 200, 3          # K/8 = 25 groups -> 4 blocks, last one has 1 group
+    codes = rng.integers(0, 256, size=(N, K // 8, M), dtype=np.uint8)
+    p = O.pack_codes(codes, 8)
+    assert p.size == O.packed_nbytes(N, K, 8, M, 8) == 4 * N * 8 * M
+    for n in range(N):
+        for i in range(K // 8):
+            for m in range(M):
+                kb, ii = divmod(i, 8)
+                assert p[((kb * N + n) * 8 + ii) * M + m] == codes[n, i, m]
+    # padding groups of the last block are zero
+    for n in range(N):
+        for ii in range(1, 8):
+            for m in range(M):
+                assert p[((3 * N + n) * 8 + ii) * M + m] == 0
+
+
+def test_pack_16bit_little_endian():
+    codes = np.array([[[0x1234], [0xABCD]]], dtype=np.uint16)       # N=1, G=2, M=1
+    p = O.pack_codes(codes, 8)
+    assert p.size == O.packed_nbytes(1, 16, 8, 1, 16) == 16
+    assert list(p[:4]) == [0x34, 0x12, 0xCD, 0xAB]
+    assert np.all(p[4:] == 0)
+
+
+# ----------------------------------------------------------------------------- activations
+def test_quant_act_golden():
+    for args, expected, why in _read_golden("quant_act.txt"):
+        xs, ss = args.split()
+        x = np.array([float(xs)], dtype=np.float16)
+        got = int(O.quant_act(x, float(ss))[0])
+        assert got == int(expected), f"{args}: got {got}, want {expected} ({why})"
+
+
+def test_quant_act_random_bounds_and_monotone():
+    x = np.sort(np.random.default_rng(0).normal(0, 3, 5000).astype(np.float16))
+    q = O.quant_act(x, 0.02)
+    assert q.dtype == np.int8
+    assert q.min() >= -127 and q.max() <= 127
+    assert np.all(np.diff(q.astype(np.int32)) >= 0)       # monotone in x
+    # away from clipping, |x/s - q| <= 1/2
+    inside = np.abs(x.astype(np.float64) / 0.02) < 126
+    err = np.abs(x.astype(np.float64)[inside] / np.float64(np.float32(0.02)) - q[inside])
+    assert err.max() <= 0.5 + 1e-5          # fp32 division can move a near-tie by 2^-24 relative
+
+
+# ----------------------------------------------------------------------------- linear
+def test_linear_worked_example():
+    rows = {}
+    with open(os.path.join(GOLDEN, "linear_worked_example.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, *v = line.split()
+                rows[k] = [float(t) for t in v]
+    cb = np.zeros((2, 256, 8), dtype=np.float16)
+    cb[0, int(rows["code1"][0])] = rows["cb1_row3"]
+    cb[1, int(rows["code2"][0])] = rows["cb2_row5"]
+    codes = np.array([[[int(rows["code1"][0]), int(rows["code2"][0])]]], dtype=np.uint8)
+    xq = np.array([rows["xq"]], dtype=np.int8)
+    W = O.decode_f64(codes, cb)
+    assert np.array_equal(W[0], np.array(rows["W"]))
+    assert np.array_equal(O.decode_rule_f16(codes, cb)[0].astype(np.float64), np.array(rows["W"]))
+    y = O.linear_f64(xq, rows["s_x"][0], W, np.array(rows["scale"], np.float16),
+                     np.array(rows["bias"], np.float16))
+    assert y.shape == (1, 1) and y[0, 0] == rows["y"][0]
+    y2 = O.lut_linear_f64(xq, rows["s_x"][0], codes, cb, np.array(rows["scale"], np.float16),
+                          np.array(rows["bias"], np.float16))
+    assert y2[0, 0] == rows["y"][0]
+
+
+def _bruteforce_linear(xq, s_x, codes, cb, scale, bias):
+    """Per-codeword direct sum, never materialising W-hat (plain loops)."""
+    T, K = xq.shape
+    N, G, M = codes.shape
+    g = cb.shape[2]
+    y = np.zeros((T, N))
+    for t in range(T):
+        for n in range(N):
+            s = 0.0
+            for i in range(G):
+                for m in range(M):
+                    row = cb[m][int(codes[n][i][m])]
+                    for e in range(g):
+                        s += float(xq[t][i * g + e]) * s_x * float(row[e])
+            y[t][n] = s * float(scale[n]) + (float(bias[n]) if bias is not None else 0.0)
+    return y
+
+
+@pytest.mark.parametrize("M,B", [(1, 8), (2, 8), (3, 8), (1, 16)])
+def test_linear_bruteforce_tiny(M, B):
+    inp = make_linear(LinearSpec(T=3, K=32, N=5, M=M, B=B), seed=11 + M)
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    y = O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"])
+    yb = _bruteforce_linear(inp["xq"], inp["s_x"], inp["codes"], inp["codebooks"],
+                            inp["scale"], inp["bias"])
+    np.testing.assert_allclose(y, yb, rtol=1e-12, atol=1e-12)
+    yl = O.lut_linear_f64(inp["xq"], inp["s_x"], inp["codes"], inp["codebooks"],
+                          inp["scale"], inp["bias"])
+    np.testing.assert_allclose(yl, yb, rtol=1e-12, atol=1e-12)
+    # no bias
+    y0 = O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], None)
+    np.testing.assert_allclose(y0, yb - inp["bias"].astype(np.float64)[None, :], atol=1e-12)
+
+
+def test_one_hot_codebooks_reproduce_dense_int_layer():
+    """M = g = 8, C^(m)[c] = (c - 128) e_m: W-hat is any integer matrix in [-128, 127],
+    i.e. a plain W8 scalar-quantized layer (Eq. 3 with z = 0).  The oracle must equal
+    an int64 matmul exactly."""
+    g = M = 8
+    cb = np.zeros((M, 256, g), dtype=np.float16)
+    for m in range(M):
+        for c in range(256):
+            cb[m, c, m] = c - 128
+    rng = np.random.default_rng(77)
+    N, K, T = 12, 64, 9
+    Wint = rng.integers(-128, 128, size=(N, K))
+    codes = np.zeros((N, K // g, M), dtype=np.uint8)
+    for n in range(N):
+        for i in range(K // g):
+            for m in range(M):
+                codes[n, i, m] = Wint[n, i * g + m] + 128
+    W = O.decode_f64(codes, cb)
+    assert np.array_equal(W, Wint.astype(np.float64))
+    assert np.array_equal(O.decode_rule_f16(codes, cb).astype(np.int64), Wint)
+    xq = rng.integers(-127, 128, size=(T, K)).astype(np.int8)
+    ones = np.ones(N, dtype=np.float16)
+    y = O.linear_f64(xq, 1.0, W, ones, None)
+    assert np.array_equal(y, (xq.astype(np.int64) @ Wint.T).astype(np.float64))
+
+
+def test_bits_per_weight_closed_form():
+    for cfg in (0, 1):
+        spec = CONFIGS[cfg]
+        inp = make_linear(spec, seed=cfg) if cfg == 0 else None
+        if inp is None:
+            continue
+        got = O.bits_per_weight(inp["codes"], inp["codebooks"], inp["scale"], spec.N, spec.K)
+        want = O.bits_per_weight_closed_form(spec.N, spec.K, spec.g, spec.M, spec.B)
+        assert got == pytest.approx(want, rel=1e-15)
+    # exact rational check of the closed form on the qkv projection shape
+    N, K = 2880, 960
+    bits = Fraction(N * K * 2 * 8, 8) + 2 * 256 * 8 * 16 + N * 16  # codes + books + scales
+    assert float(bits / (N * K)) == pytest.approx(O.bits_per_weight_closed_form(N, K, 8, 2, 8), rel=1e-15)
+    assert O.bits_per_weight_closed_form(N, K, 8, 2, 8) == pytest.approx(2.04037, abs=1e-5)
+    # a 2x8 layer is about 2 bits per weight (Sec. 2.4), a 1x16 layer too
+    assert 2.0 < O.bits_per_weight_closed_form(4096, 4096, 8, 2, 8) < 2.01
+    big = make_conv(ConvSpec(Nb=1, H=2, W=2, Cin=16, Cout=16, M=1, B=16), seed=0)
+    got = O.bits_per_weight(big["codes"], big["codebooks"], big["scale"], 16, 144)
+    assert got == pytest.approx(O.bits_per_weight_closed_form(16, 144, 8, 1, 16), rel=1e-15)
+
+
+# ----------------------------------------------------------------------------- conv
+def _bruteforce_conv(xq, s_x, W, scale, bias, kh, kw, stride, pad):
+    Nb, H, Wd, Cin = xq.shape
+    Cout = W.shape[0]
+    Ho = (H + 2 * pad - kh) // stride + 1
+    Wo = (Wd + 2 * pad - kw) // stride + 1
+    y = np.zeros((Nb, Ho, Wo, Cout))
+    for b in range(Nb):
+        for ho in range(Ho):
+            for wo in range(Wo):
+                for n in range(Cout):
+                    s = 0.0
+                    for i in range(kh):
+                        for j in range(kw):
+                            hi, wi = ho * stride + i - pad, wo * stride + j - pad
+                            if 0 <= hi < H and 0 <= wi < Wd:
+                                for c in range(Cin):
+                                    s += s_x * float(xq[b, hi, wi, c]) * W[n, (i * kw + j) * Cin + c]
+                    y[b, ho, wo, n] = s * float(scale[n]) + float(bias[n])
+    return y
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_conv_bruteforce_tiny(stride):
+    spec = ConvSpec(Nb=2, H=5, W=4, Cin=8, Cout=3, stride=stride, M=2)
+    inp = make_conv(spec, seed=21 + stride)
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    y = O.layer_f64(inp)
+    assert y.shape == (2, spec.Ho, spec.Wo, 3)
+    yb = _bruteforce_conv(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"], 3, 3, stride, 1)
+    np.testing.assert_allclose(y, yb, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_conv_matches_torch_conv2d_f64(stride):
+    torch = pytest.importorskip("torch")
+    spec = ConvSpec(Nb=3, H=9, W=7, Cin=16, Cout=24, stride=stride, M=2)
+    inp = make_conv(spec, seed=31)
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    y = O.layer_f64(inp)
+    x = torch.from_numpy(inp["xq"].astype(np.float64) * inp["s_x"]).permute(0, 3, 1, 2)
+    w = torch.from_numpy(W.reshape(24, 3, 3, 16)).permute(0, 3, 1, 2)      # OHWI -> OIHW
+    ref = torch.nn.functional.conv2d(x, w, stride=stride, padding=1).permute(0, 2, 3, 1).numpy()
+    ref = ref * inp["scale"].astype(np.float64) + inp["bias"].astype(np.float64)
+    np.testing.assert_allclose(y, ref, rtol=1e-11, atol=1e-11)
+
+
+def test_conv_centre_tap_equals_linear():
+    """Only the centre tap non-zero (one-hot books) -> the conv is the linear layer on pixels."""
+    Cin, Cout = 8, 4
+    spec = ConvSpec(Nb=1, H=3, W=3, Cin=Cin, Cout=Cout, M=1)
+    inp = make_conv(spec, seed=2)
+    # rebuild codes so every non-centre tap selects an all-zero codeword (row 0)
+    cb = inp["codebooks"].copy()
+    cb[0, 0, :] = 0
+    codes = inp["codes"].copy()
+    centre = 4 * Cin // 8
+    for j in range(codes.shape[1]):
+        if j != centre:
+            codes[:, j, 0] = 0
+        else:
+            codes[:, j, 0] = np.maximum(codes[:, j, 0], 1)
+    W = O.decode_f64(codes, cb)
+    y = O.conv2d_nhwc_f64(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"])
+    Wc = W[:, 4 * Cin:5 * Cin]
+    yl = O.linear_f64(inp["xq"].reshape(-1, Cin), inp["s_x"], Wc, inp["scale"], inp["bias"])
+    np.testing.assert_allclose(y.reshape(-1, Cout), yl, rtol=1e-13, atol=1e-13)
+
+
+def test_conv_1x1_equals_linear():
+    spec = ConvSpec(Nb=2, H=3, W=5, Cin=16, Cout=8, kh=1, kw=1, pad=0, M=2)
+    inp = make_conv(spec, seed=4)
+    y = O.layer_f64(inp)
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    yl = O.linear_f64(inp["xq"].reshape(-1, 16), inp["s_x"], W, inp["scale"], inp["bias"])
+    np.testing.assert_allclose(y.reshape(-1, 8), yl, rtol=1e-13, atol=1e-13)
+
+
+# ----------------------------------------------------------------------------- op counts
+@pytest.mark.parametrize("M,k,Cin,Cout,h,w", [(1, 2, 2, 3, 4, 4), (2, 2, 1, 2, 3, 5)])
+def test_eq_a7_op_count_and_lut_result(M, k, Cin, Cout, h, w):
+    """App. A.1: the LUT kernel's counted ops equal Eq. A7, its output the dense conv."""
+    rng = np.random.default_rng(M * 100 + k)
+    H = rng.normal(size=(Cin, h, w))
+    cb = rng.normal(size=(M, 2 ** k, 9)).astype(np.float16)
+    codes = rng.integers(0, 2 ** k, size=(Cout, Cin, M), dtype=np.uint8)
+    G, mults, adds = O.lut_conv_kaq_counted(H, codes, cb)
+    assert (mults, adds) == O.eq_a7_flops(M, k, Cin, Cout, h, w)
+    F = O.decode_kaq_f64(codes, cb).reshape(Cout, Cin, 3, 3)
+    Gd, flops = O.direct_conv_counted(H, F)
+    assert flops == O.eq_a2_flops(Cin, Cout, h, w)
+    np.testing.assert_allclose(G, Gd, rtol=1e-12, atol=1e-12)
+    # and the torch library conv agrees on the dense result
+    torch = pytest.importorskip("torch")
+    ref = torch.nn.functional.conv2d(torch.from_numpy(H)[None], torch.from_numpy(F), padding=1)[0]
+    np.testing.assert_allclose(Gd, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_breakeven_from_eq_a7():
+    """Where Eq. A7 falls below Eq. A2; the appendix's printed threshold differs."""
+    for M in (1, 2, 3, 4):
+        k = 8
+        be = O.eq_a7_breakeven(M, k)
+        c_lo, c_hi = math.floor(be), math.ceil(be)
+        if c_lo == c_hi:
+            c_lo -= 1
+        lut = lambda co: sum(O.eq_a7_flops(M, k, 16, co, 8, 8))
+        dense = lambda co: O.eq_a2_flops(16, co, 8, 8)
+        assert lut(c_hi) <= dense(c_hi)
+        assert lut(c_lo) > dense(c_lo)
+    assert O.eq_a7_breakeven(2, 8) == 544.0
+    assert O.paper_lut_breakeven(2, 8) == pytest.approx(286.875)
