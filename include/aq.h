@@ -1,0 +1,174 @@
+/*
+ * aq.h -- C ABI of the GB300 (sm_103a) additive-quantized (AQ) weight x
+ * 8-bit activation (A8) layer library.
+ *
+ * The method (AQUATIC-Diff, arXiv 2506.05960) stores every linear and
+ * convolution weight of a diffusion UNet in the additive-quantization format
+ * of Sec. 2.4, Eq. 4: the weight matrix is cut row-major into groups of g
+ * consecutive weights, and each group is the sum of M codewords, one from each
+ * codebook C^(m) (2^B rows of g entries), selected by the M codes b[i, m] of
+ * the group.  Activations are quantized to 8 bits with one scale per call
+ * (one per denoising timestep, Sec. 4.2.3).  A convolution is the same
+ * contraction over the im2col matrix (Sec. 3.1.1), computed here as an
+ * implicit GEMM without materialising im2col.
+ *
+ * Conventions shared by every entry point
+ *   - All array pointers are DEVICE pointers owned by the caller.  The library
+ *     allocates no device memory and never synchronises the device; each call
+ *     only enqueues kernels on `stream` (a cudaStream_t, NULL = legacy default
+ *     stream).  Inputs are not modified.
+ *   - Sizes are element counts.  Arrays are dense, row-major, C-contiguous.
+ *   - Every pointer must be 16-byte aligned (AQ_ERR_ALIGN otherwise).
+ *   - Supported formats: g = 8; B = 8 with M in 1..8, or B = 16 with M in 1..2.
+ *     Codes of B = 8 are uint8, codes of B = 16 are uint16 (little endian).
+ *     Codebooks are fp16 [M][2^B][g].  Per-output-channel scale and bias are
+ *     fp16 [N] (bias may be NULL).  The activation scale s_x is fp32.
+ *   - Return value: AQ_OK (0) or a negative AQ_ERR_* code.  On error nothing
+ *     is enqueued, and aq_last_error_string() describes the failure (text is
+ *     per host thread, valid until the next call on that thread).
+ *   - Device-side waits are bounded: a pipeline stage that does not complete
+ *     in about two seconds sets a device error word and the kernel returns;
+ *     aq_device_error() reads (and clears) that word.
+ */
+#ifndef AQ_H_
+#define AQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AQ_ABI_VERSION 1
+
+#if defined(__GNUC__)
+#define AQ_API __attribute__((visibility("default")))
+#else
+#define AQ_API
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define AQ_OK                    0
+#define AQ_ERR_NULL             -1  /* a required pointer is NULL                      */
+#define AQ_ERR_SHAPE            -2  /* a size is negative/zero where it must not be, or
+                                       not a multiple of what the format needs           */
+#define AQ_ERR_UNSUPPORTED      -3  /* (g, M, B), conv geometry or path not supported   */
+#define AQ_ERR_ALIGN            -4  /* a pointer is not 16-byte aligned                 */
+#define AQ_ERR_WORKSPACE        -5  /* workspace NULL or smaller than required          */
+#define AQ_ERR_CUDA             -6  /* a CUDA runtime/driver call or launch failed      */
+#define AQ_ERR_DEVICE_TIMEOUT   -7  /* a kernel gave up on a bounded wait               */
+
+/* ---- enums --------------------------------------------------------------- */
+typedef enum aq_dtype {
+  AQ_DTYPE_F16 = 0,   /* output fp16, round to nearest even */
+  AQ_DTYPE_F32 = 1    /* output fp32                        */
+} aq_dtype;
+
+typedef enum aq_path {
+  AQ_PATH_AUTO  = 0,  /* library picks from (T, N, K, M, B)                               */
+  AQ_PATH_DENSE = 1,  /* decode W-hat once into the workspace (Sec. 4.4: decompress, then
+                         the ordinary layer op), then a TMA-fed tcgen05 tensor-core GEMM   */
+  AQ_PATH_FUSED = 2,  /* decode inside the GEMM into shared memory (codebooks in shared
+                         memory, or in L2 for 2^16-entry books); W-hat never touches HBM  */
+  AQ_PATH_LUT   = 3   /* lookup-table order of App. A.1 (Eq. A5-A6): per token and group,
+                         the dot product with every codeword, then a gather-sum by code;
+                         for small token counts and B = 8                                  */
+} aq_path;
+
+/* ---- library information -------------------------------------------------- */
+
+/* ABI version of the loaded library (AQ_ABI_VERSION). */
+AQ_API int aq_abi_version(void);
+
+/* Text of the last error on the calling host thread ("" if none). */
+AQ_API const char* aq_last_error_string(void);
+
+/* Reads and clears the device error word of the current device (kernels set it
+ * when a bounded wait gives up).  Synchronises the device.  *code_out = 0 if no
+ * kernel reported an error.  Returns AQ_OK or AQ_ERR_CUDA. */
+AQ_API int aq_device_error(int* code_out);
+
+/* ---- kernel timing (diagnostics) -------------------------------------------
+ * When enabled, every entry point records a CUDA event pair on the caller's
+ * stream around each kernel it launches; aq_profile_read() waits for the
+ * recorded events and returns, per kernel kind, the summed device time in
+ * milliseconds and the number of launches since the last aq_profile_enable().
+ * Kinds: 0 quantizer, 1 pack, 2 decode, 3 tensor-core GEMM, 4 split-K reduce,
+ * 5 LUT build, 6 LUT gather, 7 fused-decode GEMM.  Uses host-side CUDA events
+ * only (no device memory).  Not for use inside CUDA graph capture.          */
+#define AQ_PROFILE_KINDS 8
+AQ_API int aq_profile_enable(int on);
+AQ_API int aq_profile_read(double* ms_out, int64_t* launches_out, int n_kinds);
+
+/* ---- code packing (Eq. 4 codes b[i, m]) -------------------------------------
+ * Canonical code layout: [N][K/g][M] (uint8 for B = 8, uint16 for B = 16), the
+ * groups of each output row in order along K, the M codes of a group
+ * contiguous.  Packed layout (storage format of every other entry point):
+ * [ceil(K/64)][N][64/g][M], i.e. for each 64-wide block of K the codes that one
+ * output row needs are contiguous (16 bytes for M = 2, B = 8) and consecutive
+ * rows follow each other, so a warp reads a block of rows with 128-bit loads.
+ * Codes of a zero-padded K tail are 0.                                        */
+
+/* Bytes of the packed buffer for an N x K layer. */
+AQ_API int aq_packed_size(int N, int K, int g, int M, int B, size_t* bytes);
+
+/* Canonical codes -> packed codes (device to device; run once per layer). */
+AQ_API int aq_pack(const void* codes_canon, void* codes_packed,
+            int N, int K, int g, int M, int B, void* stream);
+
+/* ---- decode (Sec. 2.4 Eq. 4; Sec. 4.4 "decompress prior to the layer op") --
+ * W_out[n][k] = fp16( sum_{m=0..M-1} fp32(C^(m)[b[n, k/g, m]][k mod g]) ), the
+ * fp32 sum taken in ascending m and rounded once to fp16 (round to nearest
+ * even, overflow to +-inf, subnormals kept).  Bit-exact against that rule.
+ * The per-channel scale is NOT folded in.  W_out is fp16 [N][K].             */
+AQ_API int aq_decode(const void* codes_packed, const void* codebooks, void* W_out,
+              int N, int K, int g, int M, int B, void* stream);
+
+/* ---- 8-bit activation quantizer (Sec. 4.2.3; symmetric form of Eq. 3) ------
+ * xq[i] = clip(round_half_even(x[i] / s_x), -127, 127), x fp16, division in
+ * IEEE fp32, NaN -> 0.  s_x must be finite and > 0 (AQ_ERR_SHAPE otherwise).
+ * numel == 0 is a no-op.                                                     */
+AQ_API int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stream);
+
+/* ---- AQ x A8 linear layer --------------------------------------------------
+ * y[t][n] = (s_x * scale[n]) * sum_k xq[t][k] * W[n][k] + bias[n]
+ * with W = the decoded AQ weight (fp16 under the decode rule above),
+ * products accumulated in fp32, the scale/bias epilogue in fp32, y fp16 (round
+ * to nearest even) or fp32.
+ *   xq      int8 [T][K]
+ *   y       [T][N] of out_dtype
+ *   T >= 0 (T == 0 is a no-op), K % 16 == 0, N % 8 == 0, N, K > 0.
+ *   workspace: device scratch of at least aq_linear_workspace_size() bytes
+ *   (may be NULL when that size is 0); contents on entry are ignored.
+ *   path: AQ_PATH_* (AUTO recommended).                                       */
+AQ_API int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
+                             size_t* bytes);
+AQ_API int aq_linear(const int8_t* xq, float s_x, const void* codes_packed,
+              const void* codebooks, const void* scale, const void* bias,
+              void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
+              void* workspace, size_t workspace_bytes, int path, void* stream);
+
+/* ---- AQ x A8 3x3 convolution, NHWC, implicit GEMM (Sec. 3.1.1) -------------
+ * y[b][ho][wo][n] = (s_x*scale[n]) * sum_{i,j,c} xq[b][ho*s+i-pad][wo*s+j-pad][c]
+ *                   * W[n][(i*kw + j)*Cin + c] + bias[n],
+ * out-of-image taps read as 0.  The weight is the decoded AQ matrix [Cout][K]
+ * with K = kh*kw*Cin in OHWI order, groups of g along Cin inside one tap.
+ *   xq int8 [Nb][H][W][Cin];  y [Nb][Ho][Wo][Cout] of out_dtype,
+ *   Ho = (H + 2*pad - kh)/stride + 1, Wo likewise.
+ *   Supported: kh = kw = 3, pad = 1, stride 1 or 2, Cin % 64 == 0,
+ *   Cout % 8 == 0.  A 1x1 convolution is aq_linear over the NHWC rows.       */
+AQ_API int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
+                             int stride, int pad, int g, int M, int B, int path,
+                             size_t* bytes);
+AQ_API int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed,
+                   const void* codebooks, const void* scale, const void* bias,
+                   void* y, int out_dtype, int Nb, int H, int W, int Cin, int Cout,
+                   int kh, int kw, int stride, int pad, int g, int M, int B,
+                   void* workspace, size_t workspace_bytes, int path, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AQ_H_ */

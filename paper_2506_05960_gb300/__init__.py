@@ -1,0 +1,17 @@
+"""GB300-native AQ x A8 layer library (AQUATIC-Diff inference hot path).
+
+The compute lives in the sm_103a shared library ``lib/libaq_gb300.so`` (C ABI
+in ``include/aq.h``).  This package is a thin ctypes binding with the same
+function names: it converts tensors to device pointers and sizes, passes the
+current CUDA stream, and raises :class:`AQError` on a non-zero status.  There
+is no Python or CPU fallback: if the library is missing, importing the binding
+raises.
+"""
+
+from ._binding import (  # noqa: F401
+    AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_PATH_AUTO, AQ_PATH_DENSE, AQ_PATH_FUSED, AQ_PATH_LUT,
+    AQError, aq_abi_version, aq_conv2d_nhwc, aq_conv2d_workspace_size, aq_decode,
+    aq_device_error, aq_last_error_string, aq_linear, aq_linear_workspace_size, aq_pack,
+    aq_packed_size, aq_profile_enable, aq_profile_read, aq_quant_act, library_path,
+    load_library, PROFILE_KINDS,
+)

@@ -1,0 +1,555 @@
+// aq_api.cu -- the C ABI declared in include/aq.h: argument validation, path
+// and tile planning, TMA descriptor encoding, and kernel launches.  Nothing
+// here allocates device memory or synchronises (except aq_device_error).
+#include <algorithm>
+#include <atomic>
+#include <vector>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "aq.h"
+#include "aq_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int set_error(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+int ok() {
+  g_last_error.clear();
+  return AQ_OK;
+}
+
+int cuda_status(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return ok();
+  return set_error(AQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ---- format checks (g, M, B)
+int check_format(int g, int M, int B) {
+  if (g != 8) return set_error(AQ_ERR_UNSUPPORTED, "group size g=%d unsupported (g=8 only)", g);
+  if (B == 8) {
+    if (M < 1 || M > 8) return set_error(AQ_ERR_UNSUPPORTED, "M=%d unsupported for B=8 (1..8)", M);
+  } else if (B == 16) {
+    if (M < 1 || M > 2) return set_error(AQ_ERR_UNSUPPORTED, "M=%d unsupported for B=16 (1..2)", M);
+  } else {
+    return set_error(AQ_ERR_UNSUPPORTED, "B=%d unsupported (8 or 16)", B);
+  }
+  return AQ_OK;
+}
+
+// ---- cuTensorMapEncodeTiled through the runtime's driver entry point
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = []() -> EncodeTiledFn {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+
+int encode(CUtensorMap* map, CUtensorMapDataType dt, int rank, const void* base,
+           const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box,
+           CUtensorMapSwizzle sw) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return set_error(AQ_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  cuuint32_t es[5] = {1, 1, 1, 1, 1};
+  CUresult r = fn(map, dt, static_cast<cuuint32_t>(rank), const_cast<void*>(base), dims, strides,
+                  box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return set_error(AQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return AQ_OK;
+}
+
+// ---- GEMM planning
+struct Plan {
+  int BN, n_tiles, m_tiles, splits, kb_per_split, num_kb;
+};
+
+Plan plan_gemm(int N, int K, int m_tiles) {
+  Plan pl{};
+  const int nt0 = (N + aq::kMaxBN - 1) / aq::kMaxBN;
+  int best_nt = -1, best_bn = 0;
+  long best_cols = 0;
+  for (int nt = nt0; nt <= nt0 + 3; ++nt) {
+    const int bn = ((N + nt - 1) / nt + 15) / 16 * 16;
+    if (bn > aq::kMaxBN || bn < 16) continue;
+    const long cols = static_cast<long>(nt) * bn;
+    if (best_nt < 0 || cols < best_cols) {
+      best_nt = nt;
+      best_bn = bn;
+      best_cols = cols;
+    }
+  }
+  pl.BN = best_bn;
+  pl.n_tiles = (N + best_bn - 1) / best_bn;
+  pl.m_tiles = m_tiles;
+  pl.num_kb = (K + aq::kBK - 1) / aq::kBK;
+  const long tiles = static_cast<long>(pl.n_tiles) * m_tiles;
+  int splits = 1;
+  if (tiles < 76 && pl.num_kb >= 8) {
+    splits = static_cast<int>(std::min<long>(pl.num_kb / 4, (152 + tiles - 1) / tiles));
+    splits = std::max(splits, 1);
+  }
+  pl.kb_per_split = (pl.num_kb + splits - 1) / splits;
+  pl.splits = (pl.num_kb + pl.kb_per_split - 1) / pl.kb_per_split;
+  return pl;
+}
+
+size_t dense_ws_bytes(int T, int N, int K, const Plan& pl) {
+  size_t b = align_up(static_cast<size_t>(N) * K * 2, 1024);
+  if (pl.splits > 1) b += align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024);
+  return b;
+}
+
+int resolve_path(int path) {
+  if (path == AQ_PATH_AUTO) return AQ_PATH_DENSE;
+  if (path == AQ_PATH_DENSE) return AQ_PATH_DENSE;
+  return -1;
+}
+
+// Conv tile geometry: 128 output pixels per tile as one 4-D box.
+struct ConvGeom {
+  int Ho, Wo, tiles_per_img, rows_per_tile, imgs_per_tile, m_tiles, bw, bh, bn;
+};
+
+int conv_geometry(int Nb, int H, int W, int kh, int kw, int stride, int pad, ConvGeom* g) {
+  g->Ho = (H + 2 * pad - kh) / stride + 1;
+  g->Wo = (W + 2 * pad - kw) / stride + 1;
+  if (stride != 1) return set_error(AQ_ERR_UNSUPPORTED, "conv stride %d not supported yet", stride);
+  const int Wo = g->Wo, Ho = g->Ho;
+  if (Wo > aq::kBM || aq::kBM % Wo != 0)
+    return set_error(AQ_ERR_UNSUPPORTED, "conv output width %d must divide 128", Wo);
+  const int rpt = aq::kBM / Wo;
+  if (rpt <= Ho) {
+    if (Ho % rpt != 0)
+      return set_error(AQ_ERR_UNSUPPORTED, "conv output height %d not a multiple of %d", Ho, rpt);
+    g->rows_per_tile = rpt;
+    g->tiles_per_img = Ho / rpt;
+    g->imgs_per_tile = 0;
+    g->m_tiles = Nb * g->tiles_per_img;
+    g->bw = Wo;
+    g->bh = rpt;
+    g->bn = 1;
+  } else {
+    if (rpt % Ho != 0)
+      return set_error(AQ_ERR_UNSUPPORTED, "conv image %dx%d does not tile 128 pixels", Ho, Wo);
+    g->imgs_per_tile = rpt / Ho;
+    g->rows_per_tile = Ho;
+    g->tiles_per_img = 1;
+    g->m_tiles = (Nb + g->imgs_per_tile - 1) / g->imgs_per_tile;
+    g->bw = Wo;
+    g->bh = Ho;
+    g->bn = g->imgs_per_tile;
+  }
+  return AQ_OK;
+}
+
+int check_conv_args(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
+                    int pad) {
+  if (Nb < 0 || H <= 0 || W <= 0 || Cin <= 0 || Cout <= 0)
+    return set_error(AQ_ERR_SHAPE, "conv sizes must be positive (Nb >= 0)");
+  if (kh != 3 || kw != 3 || pad != 1)
+    return set_error(AQ_ERR_UNSUPPORTED, "only 3x3 convolutions with pad 1 are supported");
+  if (stride != 1 && stride != 2) return set_error(AQ_ERR_UNSUPPORTED, "stride must be 1 or 2");
+  if (Cin % 64 != 0) return set_error(AQ_ERR_UNSUPPORTED, "Cin=%d must be a multiple of 64", Cin);
+  if (Cout % 8 != 0) return set_error(AQ_ERR_SHAPE, "Cout=%d must be a multiple of 8", Cout);
+  return AQ_OK;
+}
+
+
+// ---- kernel timing (aq_profile_*): CUDA event pairs around each launch
+namespace prof {
+std::mutex mu;
+std::atomic<bool> enabled{false};
+struct Rec {
+  cudaEvent_t a, b;
+  int kind;
+};
+std::vector<Rec> pending;
+std::vector<cudaEvent_t> pool;
+double ms[AQ_PROFILE_KINDS] = {};
+int64_t launches[AQ_PROFILE_KINDS] = {};
+
+cudaEvent_t take_locked() {
+  if (!pool.empty()) {
+    cudaEvent_t e = pool.back();
+    pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+void fold_locked(bool accumulate) {
+  for (const Rec& r : pending) {
+    float t = 0.0f;
+    if (cudaEventSynchronize(r.b) == cudaSuccess && cudaEventElapsedTime(&t, r.a, r.b) == cudaSuccess &&
+        accumulate) {
+      ms[r.kind] += t;
+      launches[r.kind] += 1;
+    }
+    pool.push_back(r.a);
+    pool.push_back(r.b);
+  }
+  pending.clear();
+}
+}  // namespace prof
+
+// Records an event pair around the launches made while it is alive.
+struct ProfScope {
+  cudaStream_t st;
+  int kind;
+  cudaEvent_t a = nullptr;
+  ProfScope(int k, cudaStream_t s) : st(s), kind(k) {
+    if (!prof::enabled.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> g(prof::mu);
+    a = prof::take_locked();
+    if (a && cudaEventRecord(a, st) != cudaSuccess) {
+      prof::pool.push_back(a);
+      a = nullptr;
+    }
+  }
+  ~ProfScope() {
+    if (!a) return;
+    std::lock_guard<std::mutex> g(prof::mu);
+    cudaEvent_t b = prof::take_locked();
+    if (!b || cudaEventRecord(b, st) != cudaSuccess) {
+      prof::pool.push_back(a);
+      if (b) prof::pool.push_back(b);
+      return;
+    }
+    prof::pending.push_back({a, b, kind});
+    if (prof::pending.size() > 16384) prof::fold_locked(true);
+  }
+};
+
+enum ProfKind { kProfQuant = 0, kProfPack = 1, kProfDecode = 2, kProfGemm = 3, kProfSplitK = 4,
+                kProfLutBuild = 5, kProfLutGather = 6, kProfFused = 7 };
+
+}  // namespace
+
+extern "C" {
+
+int aq_abi_version(void) { return AQ_ABI_VERSION; }
+
+int aq_profile_enable(int on) {
+  std::lock_guard<std::mutex> g(prof::mu);
+  prof::fold_locked(false);
+  for (int i = 0; i < AQ_PROFILE_KINDS; ++i) {
+    prof::ms[i] = 0.0;
+    prof::launches[i] = 0;
+  }
+  prof::enabled.store(on != 0);
+  return ok();
+}
+
+int aq_profile_read(double* ms_out, int64_t* launches_out, int n_kinds) {
+  if (!ms_out || !launches_out) return set_error(AQ_ERR_NULL, "NULL output");
+  std::lock_guard<std::mutex> g(prof::mu);
+  prof::fold_locked(true);
+  for (int i = 0; i < n_kinds; ++i) {
+    ms_out[i] = i < AQ_PROFILE_KINDS ? prof::ms[i] : 0.0;
+    launches_out[i] = i < AQ_PROFILE_KINDS ? prof::launches[i] : 0;
+  }
+  return ok();
+}
+
+const char* aq_last_error_string(void) { return g_last_error.c_str(); }
+
+int aq_device_error(int* code_out) {
+  if (!code_out) return set_error(AQ_ERR_NULL, "code_out is NULL");
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_status(e, "cudaDeviceSynchronize");
+  unsigned v = 0;
+  e = aq::read_clear_gemm_error(&v);
+  if (e != cudaSuccess) return cuda_status(e, "reading device error word");
+  *code_out = static_cast<int>(v);
+  return ok();
+}
+
+int aq_packed_size(int N, int K, int g, int M, int B, size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
+  *bytes = static_cast<size_t>((K + 63) / 64) * N * (64 / g) * M * (B / 8);
+  return ok();
+}
+
+int aq_pack(const void* codes_canon, void* codes_packed, int N, int K, int g, int M, int B,
+            void* stream) {
+  if (!codes_canon || !codes_packed) return set_error(AQ_ERR_NULL, "NULL code buffer");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
+  if (!aligned16(codes_canon) || !aligned16(codes_packed))
+    return set_error(AQ_ERR_ALIGN, "code buffers must be 16-byte aligned");
+  ProfScope ps(kProfPack, static_cast<cudaStream_t>(stream));
+  return cuda_status(aq::launch_pack(codes_canon, codes_packed, N, K, M, B,
+                                     static_cast<cudaStream_t>(stream)),
+                     "aq_pack launch");
+}
+
+int aq_decode(const void* codes_packed, const void* codebooks, void* W_out, int N, int K, int g,
+              int M, int B, void* stream) {
+  if (!codes_packed || !codebooks || !W_out) return set_error(AQ_ERR_NULL, "NULL argument");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
+  if (!aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(W_out))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  ProfScope ps(kProfDecode, static_cast<cudaStream_t>(stream));
+  return cuda_status(aq::launch_decode(codes_packed, codebooks, W_out, N, K, M, B,
+                                       static_cast<cudaStream_t>(stream)),
+                     "aq_decode launch");
+}
+
+int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stream) {
+  if (numel < 0) return set_error(AQ_ERR_SHAPE, "numel < 0");
+  if (!(s_x > 0.0f) || s_x == __builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite and > 0");
+  if (numel == 0) return ok();
+  if (!x || !xq) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(x) || !aligned16(xq)) return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  ProfScope ps(kProfQuant, static_cast<cudaStream_t>(stream));
+  return cuda_status(aq::launch_quant_act(x, xq, numel, s_x, static_cast<cudaStream_t>(stream)),
+                     "aq_quant_act launch");
+}
+
+int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path, size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
+  const int rp = resolve_path(path);
+  if (rp < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
+  const Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
+  *bytes = dense_ws_bytes(T, N, K, pl);
+  return ok();
+}
+
+int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+              const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
+              int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
+              void* stream) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite");
+  const int rp = resolve_path(path);
+  if (rp < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
+  if (T == 0) return ok();
+  if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+      !aligned16(y) || (bias && !aligned16(bias)))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  const Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
+  const size_t need = dense_ws_bytes(T, N, K, pl);
+  if (!workspace || workspace_bytes < need || !aligned16(workspace))
+    return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  void* Wdec = workspace;
+  float* partial = nullptr;
+  if (pl.splits > 1)
+    partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
+                                       align_up(static_cast<size_t>(N) * K * 2, 1024));
+
+  CUtensorMap mapA, mapB;
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
+    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (r) return r;
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
+    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+    if (r) return r;
+  }
+  cudaError_t e;
+  {
+    ProfScope ps(kProfDecode, st);
+    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "decode launch");
+
+  aq::GemmParams p{};
+  p.T = T;
+  p.N = N;
+  p.K = K;
+  p.BN = pl.BN;
+  p.num_kb = pl.num_kb;
+  p.kb_per_split = pl.kb_per_split;
+  p.conv = 0;
+  p.s_x = s_x;
+  p.scale = static_cast<const __half*>(scale);
+  p.bias = static_cast<const __half*>(bias);
+  p.y = y;
+  p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  p.partial = partial;
+  {
+    ProfScope ps(kProfGemm, st);
+    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, pl.splits, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
+  if (pl.splits > 1) {
+    ProfScope ps(kProfSplitK, st);
+    e = aq::launch_splitk_reduce(p, pl.splits, st);
+    if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
+  }
+  return ok();
+}
+
+int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
+                             int pad, int g, int M, int B, int path, size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
+  if (r) return r;
+  if (resolve_path(path) < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
+  ConvGeom cg;
+  r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
+  if (r) return r;
+  const int K = kh * kw * Cin;
+  const int T = Nb * cg.Ho * cg.Wo;
+  const Plan pl = plan_gemm(Cout, K, cg.m_tiles);
+  *bytes = dense_ws_bytes(T, Cout, K, pl);
+  return ok();
+}
+
+int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+                   const void* scale, const void* bias, void* y, int out_dtype, int Nb, int H,
+                   int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
+                   int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
+  if (r) return r;
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite");
+  if (resolve_path(path) < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
+  ConvGeom cg;
+  r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
+  if (r) return r;
+  if (Nb == 0) return ok();
+  if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+      !aligned16(y) || (bias && !aligned16(bias)))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  const int K = kh * kw * Cin;
+  const int T = Nb * cg.Ho * cg.Wo;
+  const Plan pl = plan_gemm(Cout, K, cg.m_tiles);
+  const size_t need = dense_ws_bytes(T, Cout, K, pl);
+  if (!workspace || workspace_bytes < need || !aligned16(workspace))
+    return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* Wdec = workspace;
+  float* partial = nullptr;
+  if (pl.splits > 1)
+    partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
+                                       align_up(static_cast<size_t>(Cout) * K * 2, 1024));
+
+  CUtensorMap mapA, mapB;
+  {
+    cuuint64_t dims[4] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W),
+                          static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(Nb)};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W) * Cin,
+                             static_cast<cuuint64_t>(H) * W * Cin};
+    cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(cg.bw),
+                         static_cast<cuuint32_t>(cg.bh), static_cast<cuuint32_t>(cg.bn)};
+    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (r) return r;
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(Cout)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
+    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+    if (r) return r;
+  }
+  cudaError_t e;
+  {
+    ProfScope ps(kProfDecode, st);
+    e = aq::launch_decode(codes_packed, codebooks, Wdec, Cout, K, M, B, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "decode launch");
+
+  aq::GemmParams p{};
+  p.T = T;
+  p.N = Cout;
+  p.K = K;
+  p.BN = pl.BN;
+  p.num_kb = pl.num_kb;
+  p.kb_per_split = pl.kb_per_split;
+  p.conv = 1;
+  p.cin_blocks = Cin / aq::kBK;
+  p.pad = pad;
+  p.tiles_per_img = cg.tiles_per_img;
+  p.rows_per_tile = cg.rows_per_tile;
+  p.imgs_per_tile = cg.imgs_per_tile;
+  p.s_x = s_x;
+  p.scale = static_cast<const __half*>(scale);
+  p.bias = static_cast<const __half*>(bias);
+  p.y = y;
+  p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  p.partial = partial;
+  {
+    ProfScope ps(kProfGemm, st);
+    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, pl.splits, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
+  if (pl.splits > 1) {
+    ProfScope ps(kProfSplitK, st);
+    e = aq::launch_splitk_reduce(p, pl.splits, st);
+    if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
+  }
+  return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,188 @@
+// aq_codec.cu -- memory-bound kernels of the AQ x A8 layer:
+//   * 8-bit activation quantizer (Sec. 4.2.3, symmetric form of Eq. 3)
+//   * code packing into the 64-wide-K-block layout
+//   * AQ decode (Sec. 2.4 Eq. 4): W-hat = sum of the selected codewords, fp32
+//     sum in ascending codebook order, one round to fp16.
+#include <cstdint>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "aq_internal.h"
+
+namespace aq {
+
+// ============================================================== quantizer
+// x / s in IEEE fp32, round half to even, NaN -> 0, clip to [-127, 127].
+__device__ __forceinline__ int8_t quant_one(__half h, float s) {
+  float q = rintf(__fdiv_rn(__half2float(h), s));
+  if (q != q) q = 0.0f;
+  q = fminf(fmaxf(q, -127.0f), 127.0f);
+  return static_cast<int8_t>(static_cast<int>(q));
+}
+
+// Each thread: 16 elements (32 B in, 16 B out) per grid-stride step.
+__global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
+                                                        int8_t* __restrict__ xq,
+                                                        int64_t nvec, int64_t numel, float s) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec;
+       v += stride) {
+    const uint4* src = reinterpret_cast<const uint4*>(x) + 2 * v;
+    uint4 a = __ldcs(src);
+    uint4 b = __ldcs(src + 1);
+    const __half* ha = reinterpret_cast<const __half*>(&a);
+    const __half* hb = reinterpret_cast<const __half*>(&b);
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __half* h = (i < 2) ? ha + 4 * i : hb + 4 * (i - 2);
+      uint32_t b0 = static_cast<uint8_t>(quant_one(h[0], s));
+      uint32_t b1 = static_cast<uint8_t>(quant_one(h[1], s));
+      uint32_t b2 = static_cast<uint8_t>(quant_one(h[2], s));
+      uint32_t b3 = static_cast<uint8_t>(quant_one(h[3], s));
+      w[i] = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
+    }
+    __stcs(reinterpret_cast<uint4*>(xq) + v, make_uint4(w[0], w[1], w[2], w[3]));
+  }
+  // scalar tail (numel % 16 elements), handled by the first threads of block 0
+  if (blockIdx.x == 0) {
+    for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x) xq[i] = quant_one(x[i], s);
+  }
+}
+
+cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s,
+                             cudaStream_t st) {
+  const int64_t nvec = numel / 16;
+  int64_t blocks = (nvec + 255) / 256;
+  const int64_t cap = 152 * 16;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  quant_act_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(
+      static_cast<const __half*>(x), xq, nvec, numel, s);
+  return cudaGetLastError();
+}
+
+// ============================================================== packing
+// canonical [N][G][M] (elem bytes eb) -> packed [KB][N][8][M]; one thread per (kb, n).
+__global__ void pack_kernel(const uint8_t* __restrict__ canon, uint8_t* __restrict__ packed,
+                            int N, int G, int M, int eb, int KB) {
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= static_cast<int64_t>(KB) * N) return;
+  const int kb = static_cast<int>(idx / N);
+  const int n = static_cast<int>(idx % N);
+  const int row_bytes = 8 * M * eb;                    // packed bytes of one (kb, n)
+  const int g0 = kb * 8;
+  const int ng = min(8, G - g0);
+  const uint8_t* src = canon + (static_cast<int64_t>(n) * G + g0) * M * eb;
+  uint8_t* dst = packed + idx * row_bytes;
+  const int valid = ng * M * eb;
+  for (int i = 0; i < row_bytes; ++i) dst[i] = (i < valid) ? src[i] : 0;
+}
+
+cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, int B,
+                        cudaStream_t st) {
+  const int G = K / 8;
+  const int KB = (K + 63) / 64;
+  const int64_t total = static_cast<int64_t>(KB) * N;
+  const int threads = 256;
+  const int64_t blocks = (total + threads - 1) / threads;
+  pack_kernel<<<static_cast<unsigned>(blocks), threads, 0, st>>>(
+      static_cast<const uint8_t*>(canon), static_cast<uint8_t*>(packed), N, G, M, B / 8, KB);
+  return cudaGetLastError();
+}
+
+// ============================================================== decode
+// Sum of M codewords of one group in fp32, ascending m, one RNE to fp16.
+// cw(m) returns the 16-byte codeword of codebook m.
+struct F8 {
+  float v[8];
+};
+
+__device__ __forceinline__ void widen_add(F8& acc, const uint4& cw, bool first) {
+  const __half2* h = reinterpret_cast<const __half2*>(&cw);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __half22float2(h[i]);
+    if (first) {
+      acc.v[2 * i] = f.x;
+      acc.v[2 * i + 1] = f.y;
+    } else {
+      acc.v[2 * i] = __fadd_rn(acc.v[2 * i], f.x);
+      acc.v[2 * i + 1] = __fadd_rn(acc.v[2 * i + 1], f.y);
+    }
+  }
+}
+
+__device__ __forceinline__ uint4 narrow(const F8& acc) {
+  uint4 r;
+  uint32_t* p = reinterpret_cast<uint32_t*>(&r);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __half2 h = __floats2half2_rn(acc.v[2 * i], acc.v[2 * i + 1]);
+    p[i] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  return r;
+}
+
+// 8-bit codes: all M codebooks (M x 256 x 16 B <= 32 KB) staged in shared memory.
+// One thread decodes the 8 groups of one (kb, n) into 128 contiguous bytes of W.
+__global__ void __launch_bounds__(256) decode_b8_kernel(const uint8_t* __restrict__ packed,
+                                                        const uint4* __restrict__ books,
+                                                        __half* __restrict__ W, int N, int K,
+                                                        int M, int KB) {
+  extern __shared__ uint4 sbook[];                       // [M][256]
+  for (int i = threadIdx.x; i < M * 256; i += blockDim.x) sbook[i] = books[i];
+  __syncthreads();
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= static_cast<int64_t>(KB) * N) return;
+  const int kb = static_cast<int>(idx / N);
+  const int n = static_cast<int>(idx % N);
+  const uint8_t* codes = packed + idx * (8 * M);
+  const int gvalid = min(8, (K - kb * 64) / 8);
+  uint4* out = reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + kb * 64);
+  for (int j = 0; j < gvalid; ++j) {
+    F8 acc;
+    for (int m = 0; m < M; ++m) widen_add(acc, sbook[m * 256 + codes[j * M + m]], m == 0);
+    out[j] = narrow(acc);
+  }
+}
+
+// 16-bit codes: codebooks (M x 65536 x 16 B) stay in global memory / L2.
+__global__ void __launch_bounds__(256) decode_b16_kernel(const uint16_t* __restrict__ packed,
+                                                         const uint4* __restrict__ books,
+                                                         __half* __restrict__ W, int N, int K,
+                                                         int M, int KB) {
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= static_cast<int64_t>(KB) * N) return;
+  const int kb = static_cast<int>(idx / N);
+  const int n = static_cast<int>(idx % N);
+  const uint16_t* codes = packed + idx * (8 * M);
+  const int gvalid = min(8, (K - kb * 64) / 8);
+  uint4* out = reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + kb * 64);
+  for (int j = 0; j < gvalid; ++j) {
+    F8 acc;
+    for (int m = 0; m < M; ++m)
+      widen_add(acc, __ldg(books + (static_cast<int64_t>(m) << 16) + codes[j * M + m]), m == 0);
+    out[j] = narrow(acc);
+  }
+}
+
+cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
+                          int B, cudaStream_t st) {
+  const int KB = (K + 63) / 64;
+  const int64_t total = static_cast<int64_t>(KB) * N;
+  const int threads = 256;
+  const int64_t blocks = (total + threads - 1) / threads;
+  if (B == 8) {
+    decode_b8_kernel<<<static_cast<unsigned>(blocks), threads, M * 256 * 16, st>>>(
+        static_cast<const uint8_t*>(packed), static_cast<const uint4*>(books),
+        static_cast<__half*>(W), N, K, M, KB);
+  } else {
+    decode_b16_kernel<<<static_cast<unsigned>(blocks), threads, 0, st>>>(
+        static_cast<const uint16_t*>(packed), static_cast<const uint4*>(books),
+        static_cast<__half*>(W), N, K, M, KB);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace aq

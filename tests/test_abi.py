@@ -1,0 +1,103 @@
+"""The C-ABI library builds, loads and exports every symbol of include/aq.h,
+and its host-side validation rejects bad arguments without touching a GPU."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2506_05960_gb300 import _binding
+    if not os.path.exists(_binding.library_path()):
+        from paper_2506_05960_gb300.build import build
+        build()
+    return _binding.load_library()
+
+
+def _declared_functions():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            names += re.findall(r"^AQ_API\s+[\w\s\*]+?\b(aq_\w+)\s*\(", text, flags=re.M)
+    return names
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared_functions()
+    assert len(names) >= 11
+    for n in names:
+        assert hasattr(lib, n), n
+    assert lib.aq_abi_version() == 1
+
+
+def test_binding_covers_header():
+    from paper_2506_05960_gb300 import _binding
+    assert set(_declared_functions()) == set(_binding._SIGNATURES)
+
+
+def _size(fn, *args):
+    out = ctypes.c_size_t(0)
+    return fn(*args, ctypes.byref(out)), out.value
+
+
+def test_packed_size(lib):
+    r, v = _size(lib.aq_packed_size, 2880, 960, 8, 2, 8)
+    assert r == 0 and v == 15 * 2880 * 16
+    r, v = _size(lib.aq_packed_size, 960, 8640, 8, 1, 16)
+    assert r == 0 and v == 135 * 960 * 16
+    r, v = _size(lib.aq_packed_size, 8, 200, 8, 3, 8)          # ragged K: 4 blocks
+    assert r == 0 and v == 4 * 8 * 8 * 3
+
+
+@pytest.mark.parametrize("g,M,B,code", [(9, 2, 8, -3), (8, 0, 8, -3), (8, 9, 8, -3),
+                                        (8, 3, 16, -3), (8, 2, 4, -3)])
+def test_unsupported_formats(lib, g, M, B, code):
+    r, _ = _size(lib.aq_packed_size, 64, 64, g, M, B)
+    assert r == code
+    assert b"unsupported" in lib.aq_last_error_string()
+
+
+def test_shape_errors(lib):
+    assert _size(lib.aq_packed_size, 64, 60, 8, 2, 8)[0] == -2          # K % g
+    assert _size(lib.aq_linear_workspace_size, 4, 24, 64, 8, 2, 8, 0)[0] == -2   # K % 16
+    assert _size(lib.aq_linear_workspace_size, 4, 64, 60, 8, 2, 8, 0)[0] == -2   # N % 8
+    assert _size(lib.aq_linear_workspace_size, -1, 64, 64, 8, 2, 8, 0)[0] == -2
+    # conv: Cin % 64, kernel size, stride
+    assert _size(lib.aq_conv2d_workspace_size, 1, 8, 8, 48, 64, 3, 3, 1, 1, 8, 2, 8, 0)[0] == -3
+    assert _size(lib.aq_conv2d_workspace_size, 1, 8, 8, 64, 64, 5, 5, 1, 2, 8, 2, 8, 0)[0] == -3
+    assert _size(lib.aq_conv2d_workspace_size, 1, 8, 8, 64, 64, 3, 3, 3, 1, 8, 2, 8, 0)[0] == -3
+
+
+def test_null_and_alignment_errors_do_not_launch(lib):
+    # T > 0 with NULL pointers -> AQ_ERR_NULL before any CUDA call
+    r = lib.aq_linear(None, 0.02, None, None, None, None, None, 0, 4, 64, 64, 8, 2, 8, None,
+                      0, 0, None)
+    assert r == -1
+    # misaligned pointers (never dereferenced: validation fails first)
+    r = lib.aq_linear(8 + 1, 0.02, 16, 16, 16, None, 16, 0, 4, 64, 64, 8, 2, 8, 16, 1 << 20,
+                      0, None)
+    assert r == -4
+    # workspace too small
+    r = lib.aq_linear(16, 0.02, 16, 16, 16, None, 16, 0, 4, 64, 64, 8, 2, 8, 16, 8, 0, None)
+    assert r == -5
+    # T == 0 is a no-op even with NULL buffers
+    assert lib.aq_linear(None, 0.02, None, None, None, None, None, 0, 0, 64, 64, 8, 2, 8, None,
+                         0, 0, None) == 0
+    # quantizer: numel 0 no-op; bad scale
+    assert lib.aq_quant_act(None, None, 0, 0.5, None) == 0
+    assert lib.aq_quant_act(16, 16, 16, 0.0, None) == -2
+    assert lib.aq_quant_act(16, 16, 16, float("nan"), None) == -2
+    assert lib.aq_quant_act(16, 16, 16, float("inf"), None) == -2
+
+
+def test_workspace_sizes(lib):
+    r, v = _size(lib.aq_linear_workspace_size, 4096, 960, 2880, 8, 2, 8, 0)
+    assert r == 0 and v >= 2880 * 960 * 2
+    r, v = _size(lib.aq_conv2d_workspace_size, 16, 64, 64, 192, 192, 3, 3, 1, 1, 8, 4, 8, 0)
+    assert r == 0 and v >= 192 * 1728 * 2
