@@ -41,7 +41,7 @@ _SIGNATURES = {
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
-    "aq_conv2d_nhwc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 15
+    "aq_conv2d_nhwc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
 }
 

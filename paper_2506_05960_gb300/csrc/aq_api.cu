@@ -213,10 +213,13 @@ cudaEvent_t take_locked() {
 void fold_locked(bool accumulate) {
   for (const Rec& r : pending) {
     float t = 0.0f;
-    if (cudaEventSynchronize(r.b) == cudaSuccess && cudaEventElapsedTime(&t, r.a, r.b) == cudaSuccess &&
-        accumulate) {
-      ms[r.kind] += t;
-      launches[r.kind] += 1;
+    if (cudaEventSynchronize(r.b) == cudaSuccess && cudaEventElapsedTime(&t, r.a, r.b) == cudaSuccess) {
+      if (accumulate) {
+        ms[r.kind] += t;
+        launches[r.kind] += 1;
+      }
+    } else {
+      (void)cudaGetLastError();  // do not leave the failure for the next launch check
     }
     pool.push_back(r.a);
     pool.push_back(r.b);

@@ -41,6 +41,26 @@ def test_binding_covers_header():
     assert set(_declared_functions()) == set(_binding._SIGNATURES)
 
 
+def _declared_arity():
+    """{name: parameter count} parsed from the AQ_API declarations."""
+    out = {}
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            for m in re.finditer(r"^AQ_API\s+[\w\s\*]+?\b(aq_\w+)\s*\(([^)]*)\)", text,
+                                 flags=re.M):
+                params = m.group(2).strip()
+                out[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_arity_matches_header():
+    from paper_2506_05960_gb300 import _binding
+    arity = _declared_arity()
+    for name, (_, args) in _binding._SIGNATURES.items():
+        assert len(args) == arity[name], (name, len(args), arity[name])
+
+
 def _size(fn, *args):
     out = ctypes.c_size_t(0)
     return fn(*args, ctypes.byref(out)), out.value
