@@ -149,6 +149,33 @@ AQ_API int aq_linear(const int8_t* xq, float s_x, const void* codes_packed,
               void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
               void* workspace, size_t workspace_bytes, int path, void* stream);
 
+/* ---- linear layer without any device allocation --------------------------
+ * The paper has no counterpart: this is a deployment convenience.  Some callers
+ * cannot call cudaMalloc at all (code running under a fixed memory budget that
+ * is reserved up front, a host allocator that must not be re-entered from a
+ * callback, or an engine that forbids allocation once it is serving), so they
+ * cannot provide the workspace that aq_linear needs for the decoded weights.
+ * aq_linear_noalloc computes exactly what aq_linear computes (same kernels,
+ * dense path, no K splitting), but decodes the weights into a fixed scratch
+ * array that the library holds in device memory: AQ_NOALLOC_SCRATCH_BYTES
+ * (16 MiB) per GPU that loads the library, kept until the process exits.
+ *   - Limit: N * K * 2 <= AQ_NOALLOC_SCRATCH_BYTES (N * K <= 8,388,608
+ *     weights); larger layers return AQ_ERR_WORKSPACE before any CUDA call.
+ *   - The first call on each device looks up the array's device address
+ *     (with that device current); make that first call before any stream
+ *     capture.  Later calls make no CUDA runtime call other than launches.
+ *   - Every call shares the one array and overwrites what it uses (nothing
+ *     in it needs to start at zero).  Calls that can overlap on the GPU (on
+ *     different streams without ordering) race on the array and give wrong
+ *     results: order them on one stream or with events.
+ *   - Never calls cudaMalloc, cudaFree or any allocating library routine.
+ * Arguments, layouts and other errors as for aq_linear.                     */
+#define AQ_NOALLOC_SCRATCH_BYTES (16u << 20)
+AQ_API int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_packed,
+                             const void* codebooks, const void* scale, const void* bias,
+                             void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
+                             void* stream);
+
 /* ---- AQ x A8 3x3 convolution, NHWC, implicit GEMM (Sec. 3.1.1) -------------
  * y[b][ho][wo][n] = (s_x*scale[n]) * sum_{i,j,c} xq[b][ho*s+i-pad][wo*s+j-pad][c]
  *                   * W[n][(i*kw + j)*Cin + c] + bias[n],

@@ -40,6 +40,8 @@ _SIGNATURES = {
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_linear_noalloc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
+                          + [_c_void_p]),
     "aq_conv2d_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
     "aq_conv2d_nhwc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
@@ -168,6 +170,14 @@ def aq_linear(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K,
         _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
         _ptr(y), out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
         _stream(stream)), "aq_linear")
+
+
+def aq_linear_noalloc(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N,
+                      g=8, M=2, B=8, stream=None) -> None:
+    """aq_linear with the library's fixed device scratch instead of a caller workspace."""
+    _check(load_library().aq_linear_noalloc(
+        _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(y), out_dtype, T, K, N, g, M, B, _stream(stream)), "aq_linear_noalloc")
 
 
 def aq_conv2d_workspace_size(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8,

@@ -16,6 +16,10 @@
 #include "aq.h"
 #include "aq_internal.h"
 
+// Scratch of aq_linear_noalloc: the decoded weights of one call.  Lives for the
+// life of the process on every device that loads this module.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[AQ_NOALLOC_SCRATCH_BYTES];
+
 namespace {
 
 thread_local std::string g_last_error;
@@ -556,3 +560,104 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
 }
 
 }  // extern "C"
+
+// Device address of g_noalloc_scratch on the current device, looked up once per
+// device (the host-side symbol is only a stand-in, never a device address).
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_dev_ptr[kMaxDevices] = {};
+
+int noalloc_scratch_ptr(void** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_status(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return set_error(AQ_ERR_CUDA, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> g(g_noalloc_mu);
+  if (g_noalloc_dev_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress(no-alloc scratch)");
+    if (p == nullptr || !aligned16(p)) return set_error(AQ_ERR_CUDA, "no-alloc scratch address invalid");
+    g_noalloc_dev_ptr[dev] = p;
+  }
+  *out = g_noalloc_dev_ptr[dev];
+  return AQ_OK;
+}
+}  // namespace
+
+extern "C" int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_packed,
+                                 const void* codebooks, const void* scale, const void* bias,
+                                 void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
+                                 void* stream) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
+  const size_t need = static_cast<size_t>(N) * static_cast<size_t>(K) * 2;
+  if (need > AQ_NOALLOC_SCRATCH_BYTES)
+    return set_error(AQ_ERR_WORKSPACE,
+                     "aq_linear_noalloc: N*K*2 = %zu bytes exceeds the fixed scratch of %u bytes",
+                     need, (unsigned)AQ_NOALLOC_SCRATCH_BYTES);
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite");
+  if (T == 0) return ok();
+  if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+      !aligned16(y) || (bias && !aligned16(bias)))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  void* Wdec = nullptr;
+  r = noalloc_scratch_ptr(&Wdec);
+  if (r) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
+  pl.splits = 1;                      // no split-K: the scratch holds only the weights
+  pl.kb_per_split = pl.num_kb;
+
+  CUtensorMap mapA, mapB;
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
+    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (r) return r;
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
+    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+    if (r) return r;
+  }
+  cudaError_t e;
+  {
+    ProfScope ps(kProfDecode, st);
+    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "decode launch");
+  aq::GemmParams p{};
+  p.T = T;
+  p.N = N;
+  p.K = K;
+  p.BN = pl.BN;
+  p.num_kb = pl.num_kb;
+  p.kb_per_split = pl.kb_per_split;
+  p.conv = 0;
+  p.s_x = s_x;
+  p.scale = static_cast<const __half*>(scale);
+  p.bias = static_cast<const __half*>(bias);
+  p.y = y;
+  p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  p.partial = nullptr;
+  {
+    ProfScope ps(kProfGemm, st);
+    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, 1, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
+  return ok();
+}
