@@ -93,39 +93,68 @@ int encode(CUtensorMap* map, CUtensorMapDataType dt, int rank, const void* base,
   return AQ_OK;
 }
 
-// ---- GEMM planning
+// ---- GEMM planning (no device queries: the plan, and so the workspace size,
+// depends only on the shapes)
+constexpr int kPlanSMs = 152;            // GB300 SM count assumed by the cost model
+constexpr size_t kSmemOptin = 232448;    // max dynamic shared memory per CTA on sm_103
+
 struct Plan {
   int BN, n_tiles, m_tiles, splits, kb_per_split, num_kb;
+  int stages, a_stages, acc_stride, a_col, total_tiles;
 };
 
-Plan plan_gemm(int N, int K, int m_tiles) {
-  Plan pl{};
-  const int nt0 = (N + aq::kMaxBN - 1) / aq::kMaxBN;
-  int best_nt = -1, best_bn = 0;
-  long best_cols = 0;
-  for (int nt = nt0; nt <= nt0 + 3; ++nt) {
-    const int bn = ((N + nt - 1) / nt + 15) / 16 * 16;
-    if (bn > aq::kMaxBN || bn < 16) continue;
-    const long cols = static_cast<long>(nt) * bn;
-    if (best_nt < 0 || cols < best_cols) {
-      best_nt = nt;
-      best_bn = bn;
-      best_cols = cols;
+// Cycles of one pipeline stage (eight 128 x BN x 16 MMAs issued by one thread),
+// measured on GB300: an MMA takes BN/2 cycles (at least 48; N = 160 runs at 88),
+// and the stage's barrier wait + commits hide under the MMAs only from BN = 192.
+double stage_cycles(int BN) {
+  double mma = BN == 160 ? 88.0 : (BN / 2.0 < 48.0 ? 48.0 : BN / 2.0);
+  double exposed = BN >= 192 ? 0.0 : (BN >= 160 ? 60.0 : 115.0);
+  return 8.0 * mma + exposed;
+}
+
+void finish_plan(Plan& pl, bool f32_out) {
+  pl.acc_stride = pl.BN;
+  pl.a_col = 2 * pl.acc_stride;
+  pl.a_stages = aq::gemm_a_stages(pl.BN);
+  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1);
+  pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
+}
+
+// Picks the N tile and the K split that minimise a model of the busiest SM's time:
+// waves x (stage cycles x stages per tile + a fixed tile overhead), plus the traffic
+// and launch of the split-K reduction when K is split.  Depends only on the shapes.
+Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out) {
+  const int num_kb = (K + aq::kBK - 1) / aq::kBK;
+  double best = 1e30;
+  Plan bp{};
+  for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
+    if (BN == 224) continue;
+    if (aq::gemm_a_stages(BN) < 2) continue;
+    const int n_tiles = (N + BN - 1) / BN;
+    const int max_split = allow_split ? std::min(num_kb, 64) : 1;
+    for (int sp = 1; sp <= max_split; ++sp) {
+      const int kbps = (num_kb + sp - 1) / sp;
+      const int s_eff = (num_kb + kbps - 1) / kbps;
+      if (s_eff != sp) continue;
+      const long tiles = static_cast<long>(m_tiles) * n_tiles * s_eff;
+      const long waves = (tiles + kPlanSMs - 1) / kPlanSMs;
+      const double tile_cycles = (kbps / 2) * stage_cycles(BN) + (kbps & 1) * 0.5 * stage_cycles(BN) + 800.0;
+      double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
+      if (s_eff > 1) t += (s_eff * 8.0 + 2.0) * T * static_cast<double>(N) / 6.0e12 + 2.0e-6;
+      if (t < best * 0.999) {
+        best = t;
+        bp = Plan{};
+        bp.BN = BN;
+        bp.n_tiles = n_tiles;
+        bp.m_tiles = m_tiles;
+        bp.splits = s_eff;
+        bp.kb_per_split = kbps;
+        bp.num_kb = num_kb;
+      }
     }
   }
-  pl.BN = best_bn;
-  pl.n_tiles = (N + best_bn - 1) / best_bn;
-  pl.m_tiles = m_tiles;
-  pl.num_kb = (K + aq::kBK - 1) / aq::kBK;
-  const long tiles = static_cast<long>(pl.n_tiles) * m_tiles;
-  int splits = 1;
-  if (tiles < 76 && pl.num_kb >= 8) {
-    splits = static_cast<int>(std::min<long>(pl.num_kb / 4, (152 + tiles - 1) / tiles));
-    splits = std::max(splits, 1);
-  }
-  pl.kb_per_split = (pl.num_kb + splits - 1) / splits;
-  pl.splits = (pl.num_kb + pl.kb_per_split - 1) / pl.kb_per_split;
-  return pl;
+  finish_plan(bp, f32_out);
+  return bp;
 }
 
 size_t dense_ws_bytes(int T, int N, int K, const Plan& pl) {
@@ -263,6 +292,99 @@ struct ProfScope {
 enum ProfKind { kProfQuant = 0, kProfPack = 1, kProfDecode = 2, kProfGemm = 3, kProfSplitK = 4,
                 kProfLutBuild = 5, kProfLutGather = 6, kProfFused = 7 };
 
+int sm_count() {
+  static int counts[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    (void)cudaGetLastError();
+    return kPlanSMs;
+  }
+  if (counts[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+      (void)cudaGetLastError();
+      n = kPlanSMs;
+    }
+    counts[dev] = n;
+  }
+  return counts[dev];
+}
+
+// Dense path after the activation map is built: decode W-hat into the workspace,
+// then the tensor-core GEMM with the fused epilogue (or split-K partials + reduce).
+int run_dense(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
+              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st) {
+  p.BN = pl.BN;
+  p.num_kb = pl.num_kb;
+  p.kb_per_split = pl.kb_per_split;
+  p.m_tiles = pl.m_tiles;
+  p.n_tiles = pl.n_tiles;
+  p.splits = pl.splits;
+  p.total_tiles = pl.total_tiles;
+  p.stages = pl.stages;
+  p.a_stages = pl.a_stages;
+  p.acc_stride = pl.acc_stride;
+  p.a_col = pl.a_col;
+  p.partial = pl.splits > 1 ? partial : nullptr;
+  const int T = p.T, N = p.N, K = p.K;
+  int r;
+  CUtensorMap mapB, mapY;
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
+    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+    if (r) return r;
+  }
+  if (p.partial) {
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T),
+                          static_cast<cuuint64_t>(pl.splits)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(N) * 4, static_cast<cuuint64_t>(T) * N * 4};
+    cuuint32_t box[3] = {32, 32, 1};
+    r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, p.partial, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+  } else if (p.out_f32) {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(N) * 4};
+    cuuint32_t box[2] = {32, 32};
+    r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, p.y, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_128B);
+  } else {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(N) * 2};
+    cuuint32_t box[2] = {32, 32};
+    r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.y, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_64B);
+  }
+  if (r) return r;
+  cudaError_t e;
+  {
+    ProfScope ps(kProfDecode, st);
+    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "decode launch");
+  {
+    ProfScope ps(kProfGemm, st);
+    e = aq::launch_gemm(mapA, mapB, mapY, p, std::min(pl.total_tiles, sm_count()), st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
+  if (pl.splits > 1) {
+    ProfScope ps(kProfSplitK, st);
+    e = aq::launch_splitk_reduce(p, pl.splits, st);
+    if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
+  }
+  return ok();
+}
+
+int encode_linear_a(CUtensorMap* mapA, const int8_t* xq, int T, int K) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
+  return encode(mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
+                CU_TENSOR_MAP_SWIZZLE_64B);
+}
+
 }  // namespace
 
 extern "C" {
@@ -361,7 +483,7 @@ int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
   const int rp = resolve_path(path);
   if (rp < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
-  const Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
+  const Plan pl = plan_gemm(T, N, K, (T + aq::kBM - 1) / aq::kBM, true, false);
   *bytes = dense_ws_bytes(T, N, K, pl);
   return ok();
 }
@@ -385,67 +507,28 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
   if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
-  const Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
+  const Plan pl = plan_gemm(T, N, K, (T + aq::kBM - 1) / aq::kBM, true, out_dtype == AQ_DTYPE_F32);
   const size_t need = dense_ws_bytes(T, N, K, pl);
   if (!workspace || workspace_bytes < need || !aligned16(workspace))
     return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-
   void* Wdec = workspace;
-  float* partial = nullptr;
-  if (pl.splits > 1)
-    partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
-                                       align_up(static_cast<size_t>(N) * K * 2, 1024));
-
-  CUtensorMap mapA, mapB;
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
-    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_NONE);
-    if (r) return r;
-  }
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
-    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_128B);
-    if (r) return r;
-  }
-  cudaError_t e;
-  {
-    ProfScope ps(kProfDecode, st);
-    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "decode launch");
-
+  float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
+                                            align_up(static_cast<size_t>(N) * K * 2, 1024));
+  CUtensorMap mapA;
+  r = encode_linear_a(&mapA, xq, T, K);
+  if (r) return r;
   aq::GemmParams p{};
   p.T = T;
   p.N = N;
   p.K = K;
-  p.BN = pl.BN;
-  p.num_kb = pl.num_kb;
-  p.kb_per_split = pl.kb_per_split;
   p.conv = 0;
   p.s_x = s_x;
   p.scale = static_cast<const __half*>(scale);
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  p.partial = partial;
-  {
-    ProfScope ps(kProfGemm, st);
-    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, pl.splits, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
-  if (pl.splits > 1) {
-    ProfScope ps(kProfSplitK, st);
-    e = aq::launch_splitk_reduce(p, pl.splits, st);
-    if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
-  }
-  return ok();
+  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, partial, st);
 }
 
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
@@ -461,7 +544,7 @@ int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, in
   if (r) return r;
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  const Plan pl = plan_gemm(Cout, K, cg.m_tiles);
+  const Plan pl = plan_gemm(T, Cout, K, cg.m_tiles, true, false);
   *bytes = dense_ws_bytes(T, Cout, K, pl);
   return ok();
 }
@@ -489,18 +572,15 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  const Plan pl = plan_gemm(Cout, K, cg.m_tiles);
+  const Plan pl = plan_gemm(T, Cout, K, cg.m_tiles, true, out_dtype == AQ_DTYPE_F32);
   const size_t need = dense_ws_bytes(T, Cout, K, pl);
   if (!workspace || workspace_bytes < need || !aligned16(workspace))
     return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   void* Wdec = workspace;
-  float* partial = nullptr;
-  if (pl.splits > 1)
-    partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
-                                       align_up(static_cast<size_t>(Cout) * K * 2, 1024));
-
-  CUtensorMap mapA, mapB;
+  float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
+                                            align_up(static_cast<size_t>(Cout) * K * 2, 1024));
+  CUtensorMap mapA;
   {
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W),
                           static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(Nb)};
@@ -509,31 +589,13 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
     cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(cg.bw),
                          static_cast<cuuint32_t>(cg.bh), static_cast<cuuint32_t>(cg.bn)};
     r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_NONE);
+               CU_TENSOR_MAP_SWIZZLE_64B);
     if (r) return r;
   }
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(Cout)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
-    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_128B);
-    if (r) return r;
-  }
-  cudaError_t e;
-  {
-    ProfScope ps(kProfDecode, st);
-    e = aq::launch_decode(codes_packed, codebooks, Wdec, Cout, K, M, B, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "decode launch");
-
   aq::GemmParams p{};
   p.T = T;
   p.N = Cout;
   p.K = K;
-  p.BN = pl.BN;
-  p.num_kb = pl.num_kb;
-  p.kb_per_split = pl.kb_per_split;
   p.conv = 1;
   p.cin_blocks = Cin / aq::kBK;
   p.pad = pad;
@@ -545,18 +607,7 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  p.partial = partial;
-  {
-    ProfScope ps(kProfGemm, st);
-    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, pl.splits, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
-  if (pl.splits > 1) {
-    ProfScope ps(kProfSplitK, st);
-    e = aq::launch_splitk_reduce(p, pl.splits, st);
-    if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
-  }
-  return ok();
+  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, partial, st);
 }
 
 }  // extern "C"
@@ -613,51 +664,20 @@ extern "C" int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_
   if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
 
-  Plan pl = plan_gemm(N, K, (T + aq::kBM - 1) / aq::kBM);
-  pl.splits = 1;                      // no split-K: the scratch holds only the weights
-  pl.kb_per_split = pl.num_kb;
-
-  CUtensorMap mapA, mapB;
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
-    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_NONE);
-    if (r) return r;
-  }
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
-    r = encode(&mapB, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Wdec, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_128B);
-    if (r) return r;
-  }
-  cudaError_t e;
-  {
-    ProfScope ps(kProfDecode, st);
-    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "decode launch");
+  // no K split: the scratch holds only the decoded weights
+  const Plan pl = plan_gemm(T, N, K, (T + aq::kBM - 1) / aq::kBM, false, out_dtype == AQ_DTYPE_F32);
+  CUtensorMap mapA;
+  r = encode_linear_a(&mapA, xq, T, K);
+  if (r) return r;
   aq::GemmParams p{};
   p.T = T;
   p.N = N;
   p.K = K;
-  p.BN = pl.BN;
-  p.num_kb = pl.num_kb;
-  p.kb_per_split = pl.kb_per_split;
   p.conv = 0;
   p.s_x = s_x;
   p.scale = static_cast<const __half*>(scale);
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  p.partial = nullptr;
-  {
-    ProfScope ps(kProfGemm, st);
-    e = aq::launch_gemm(mapA, mapB, p, pl.n_tiles, pl.m_tiles, 1, st);
-  }
-  if (e != cudaSuccess) return cuda_status(e, "gemm launch");
-  return ok();
+  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, nullptr, st);
 }

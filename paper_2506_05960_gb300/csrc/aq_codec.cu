@@ -13,8 +13,16 @@ namespace aq {
 
 // ============================================================== quantizer
 // x / s in IEEE fp32, round half to even, NaN -> 0, clip to [-127, 127].
-__device__ __forceinline__ int8_t quant_one(__half h, float s) {
-  float q = rintf(__fdiv_rn(__half2float(h), s));
+// Fast path: q = x * fl(1/s) lies within 3 * 2^-24 * |x/s| of fl(x/s); for
+// |x/s| < 128 that is < 2.3e-5, so unless q is within 1e-4 of a half-integer
+// both round to the same integer (and for |x/s| >= 128 both clip to the same
+// end).  Near a tie, and for NaN/inf, the exact IEEE quotient decides.
+__device__ __forceinline__ int8_t quant_one(__half h, float s, float rs) {
+  const float x = __half2float(h);
+  float q = x * rs;
+  const float fr = q - floorf(q);
+  if (!(fabsf(fr - 0.5f) > 1e-4f)) q = __fdiv_rn(x, s);
+  q = rintf(q);
   if (q != q) q = 0.0f;
   q = fminf(fmaxf(q, -127.0f), 127.0f);
   return static_cast<int8_t>(static_cast<int>(q));
@@ -28,6 +36,7 @@ __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec;
        v += stride) {
     const uint4* src = reinterpret_cast<const uint4*>(x) + 2 * v;
+    const float rs = __frcp_rn(s);
     uint4 a = __ldcs(src);
     uint4 b = __ldcs(src + 1);
     const __half* ha = reinterpret_cast<const __half*>(&a);
@@ -36,17 +45,18 @@ __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const __half* h = (i < 2) ? ha + 4 * i : hb + 4 * (i - 2);
-      uint32_t b0 = static_cast<uint8_t>(quant_one(h[0], s));
-      uint32_t b1 = static_cast<uint8_t>(quant_one(h[1], s));
-      uint32_t b2 = static_cast<uint8_t>(quant_one(h[2], s));
-      uint32_t b3 = static_cast<uint8_t>(quant_one(h[3], s));
+      uint32_t b0 = static_cast<uint8_t>(quant_one(h[0], s, rs));
+      uint32_t b1 = static_cast<uint8_t>(quant_one(h[1], s, rs));
+      uint32_t b2 = static_cast<uint8_t>(quant_one(h[2], s, rs));
+      uint32_t b3 = static_cast<uint8_t>(quant_one(h[3], s, rs));
       w[i] = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
     }
     __stcs(reinterpret_cast<uint4*>(xq) + v, make_uint4(w[0], w[1], w[2], w[3]));
   }
   // scalar tail (numel % 16 elements), handled by the first threads of block 0
   if (blockIdx.x == 0) {
-    for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x) xq[i] = quant_one(x[i], s);
+    for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x)
+      xq[i] = quant_one(x[i], s, __frcp_rn(s));
   }
 }
 
@@ -125,54 +135,64 @@ __device__ __forceinline__ uint4 narrow(const F8& acc) {
 }
 
 // 8-bit codes: all M codebooks (M x 256 x 16 B <= 32 KB) staged in shared memory.
-// One thread decodes the 8 groups of one (kb, n) into 128 contiguous bytes of W.
-__global__ void __launch_bounds__(256) decode_b8_kernel(const uint8_t* __restrict__ packed,
+// One thread per group: packed index idx = (kb*N + n)*8 + j is also the thread's
+// linear index, so code loads are contiguous across the warp and each group of 8
+// threads writes 128 contiguous bytes of W.
+__global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restrict__ packed,
                                                         const uint4* __restrict__ books,
                                                         __half* __restrict__ W, int N, int K,
                                                         int M, int KB) {
   extern __shared__ uint4 sbook[];                       // [M][256]
   for (int i = threadIdx.x; i < M * 256; i += blockDim.x) sbook[i] = books[i];
   __syncthreads();
-  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (idx >= static_cast<int64_t>(KB) * N) return;
-  const int kb = static_cast<int>(idx / N);
-  const int n = static_cast<int>(idx % N);
-  const uint8_t* codes = packed + idx * (8 * M);
-  const int gvalid = min(8, (K - kb * 64) / 8);
-  uint4* out = reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + kb * 64);
-  for (int j = 0; j < gvalid; ++j) {
+  const int G = K / 8;
+  const int64_t total = static_cast<int64_t>(KB) * N * 8;
+  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(idx & 7);
+    const int64_t rem = idx >> 3;
+    const int kb = static_cast<int>(rem / N);
+    const int n = static_cast<int>(rem - static_cast<int64_t>(kb) * N);
+    const int grp = kb * 8 + j;
+    if (grp >= G) continue;
+    const uint8_t* c = packed + idx * M;
     F8 acc;
-    for (int m = 0; m < M; ++m) widen_add(acc, sbook[m * 256 + codes[j * M + m]], m == 0);
-    out[j] = narrow(acc);
+    for (int m = 0; m < M; ++m) widen_add(acc, sbook[m * 256 + c[m]], m == 0);
+    *reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + grp * 8) = narrow(acc);
   }
 }
 
 // 16-bit codes: codebooks (M x 65536 x 16 B) stay in global memory / L2.
-__global__ void __launch_bounds__(256) decode_b16_kernel(const uint16_t* __restrict__ packed,
+__global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restrict__ packed,
                                                          const uint4* __restrict__ books,
                                                          __half* __restrict__ W, int N, int K,
                                                          int M, int KB) {
-  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (idx >= static_cast<int64_t>(KB) * N) return;
-  const int kb = static_cast<int>(idx / N);
-  const int n = static_cast<int>(idx % N);
-  const uint16_t* codes = packed + idx * (8 * M);
-  const int gvalid = min(8, (K - kb * 64) / 8);
-  uint4* out = reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + kb * 64);
-  for (int j = 0; j < gvalid; ++j) {
+  const int G = K / 8;
+  const int64_t total = static_cast<int64_t>(KB) * N * 8;
+  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(idx & 7);
+    const int64_t rem = idx >> 3;
+    const int kb = static_cast<int>(rem / N);
+    const int n = static_cast<int>(rem - static_cast<int64_t>(kb) * N);
+    const int grp = kb * 8 + j;
+    if (grp >= G) continue;
+    const uint16_t* c = packed + idx * M;
     F8 acc;
     for (int m = 0; m < M; ++m)
-      widen_add(acc, __ldg(books + (static_cast<int64_t>(m) << 16) + codes[j * M + m]), m == 0);
-    out[j] = narrow(acc);
+      widen_add(acc, __ldg(books + (static_cast<int64_t>(m) << 16) + c[m]), m == 0);
+    *reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + grp * 8) = narrow(acc);
   }
 }
 
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st) {
   const int KB = (K + 63) / 64;
-  const int64_t total = static_cast<int64_t>(KB) * N;
-  const int threads = 256;
-  const int64_t blocks = (total + threads - 1) / threads;
+  const int64_t total = static_cast<int64_t>(KB) * N * 8;
+  const int threads = 512;
+  int64_t blocks = (total + threads - 1) / threads;
+  if (blocks > 152 * 4) blocks = 152 * 4;
+  if (blocks < 1) blocks = 1;
   if (B == 8) {
     decode_b8_kernel<<<static_cast<unsigned>(blocks), threads, M * 256 * 16, st>>>(
         static_cast<const uint8_t*>(packed), static_cast<const uint4*>(books),

@@ -1,17 +1,29 @@
 // aq_gemm.cu -- tcgen05 tensor-core contraction of the AQ x A8 layer.
 //
-// acc[t][n] = sum_k fp16(xq[t][k]) * W[n][k]   (fp32 in TMEM), then the fused
-// epilogue y = acc * (s_x * scale[n]) + bias[n] (Sec. 3.1.1: the layer is the
-// product Y = W X; for a convolution X is the im2col matrix, built here tap by
-// tap from 4-D TMA boxes instead of being materialised).
+// acc[t][n] = sum_k fp16(xq[t][k]) * W[n][k]   (fp32 in tensor memory), then the
+// fused epilogue y = acc * (s_x * scale[n]) + bias[n] (Sec. 3.1.1: the layer is
+// the product Y = W X; for a convolution X is the im2col matrix, assembled here
+// from 4-D TMA boxes per (tap, 64-channel block) instead of being materialised).
 //
-// One CTA computes a 128 x BN output tile (optionally one K split of it):
-//   warp 0      TMA producer: int8 activation box + fp16 weight box per stage
-//   warp 1      TMEM allocator and single-thread tcgen05.mma issuer
-//   warps 2..5  int8 -> fp16 converters (into the 128B-swizzled K-major A
-//               tile), then the epilogue (TMEM -> registers -> global)
-// Stages are handed over with mbarriers; every wait is bounded (about 2 s),
-// after which the CTA records an error, drains its own copies and exits.
+// Persistent kernel, one CTA per SM, static round-robin over 128 x BN output
+// tiles (and K splits).  A pipeline stage covers 128 of K (two 64-wide TMA
+// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps:
+//   warp 0      TMA producer: int8 activation boxes (64-byte swizzle) and fp16
+//               weight boxes (128-byte swizzle) into an S-deep smem ring
+//   warp 1      TMEM owner (all 512 columns) and the single MMA-issuing thread:
+//               tcgen05.mma.kind::f16 with A read from TMEM and B from shared
+//               memory.  Its loop is kept minimal (one barrier wait per eight
+//               MMAs, descriptors advanced by addition, no divisions): with
+//               BN = 192 the wait, fence and commits hide under the MMAs.
+//   warps 2..5  converters: int8 rows -> fp16 exactly -> tcgen05.st into a
+//               TMEM A ring (no shared-memory round trip for the fp16 operand)
+//   warps 6..9  epilogue: TMEM accumulator -> scale/bias -> 32 x 32 boxes in
+//               shared memory -> TMA stores (ragged edges clipped by TMA)
+// The fp32 accumulator is double-buffered in TMEM so the epilogue of one tile
+// runs under the mainloop of the next.  The issue loop carries no divisions:
+// ring index and phase advance by counters.  Every wait is bounded (about 2 s);
+// on time-out the CTA records an error word, drains its in-flight work, frees
+// TMEM and exits.
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_fp16.h>
@@ -24,249 +36,396 @@ namespace aq {
 
 __device__ unsigned g_gemm_err = 0;
 
-constexpr int kStages = 3;
-constexpr int kA16Bytes = kBM * 128;       // 16 KB fp16 A stage (128 rows x 64 fp16)
-constexpr int kB16Bytes = kMaxBN * 128;    // 32 KB fp16 B stage (<= 256 rows x 64 fp16)
-constexpr int kA8Bytes = kBM * 64;         // 8 KB int8 A stage
-constexpr int kTmemCols = 256;
+constexpr int kThreads = 320;
+constexpr int kA8Half = kBM * 64;               // one 64-wide int8 box: 128 rows x 64 B
+constexpr int kA8Stage = kStageBlocks * kA8Half;
+constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A slot
+constexpr int kEpiBuf32 = 4096;                 // one 32 x 32 fp32 output box (128-byte rows)
+constexpr int kEpiBuf16 = 2048;                 // one 32 x 32 fp16 output box (64-byte rows)
+constexpr int kScaleBytes = 4 * 2 * kMaxBN * 4; // per epilogue warp: scale and bias of a tile
+constexpr int kTmemCols = 512;
 
-struct alignas(8) GemmSmemTail {
-  uint64_t full[kStages];    // TMA bytes landed (A int8 + B fp16)
-  uint64_t conv[kStages];    // A converted to fp16 (4 converter warps arrive)
-  uint64_t empty[kStages];   // MMA finished reading the stage (tcgen05.commit)
-  uint64_t accum;            // all MMAs of the tile done
+struct alignas(8) GemmBarriers {
+  uint64_t full[kMaxStages];     // TMA bytes of a smem stage landed
+  uint64_t empty[kMaxStages];    // smem stage consumed: 4 converter warps + 1 MMA commit
+  uint32_t a_ready[kMaxStages];  // fp16 A slot written: +1 per converter warp (4 per use)
+  uint64_t a_empty[kMaxStages];  // MMAs reading the TMEM slot done (commit)
+  uint64_t acc_full[2];          // accumulator buffer complete (commit)
+  uint64_t acc_empty[2];         // accumulator buffer drained (4 epilogue warps)
+  uint64_t drain;                // all MMAs of this CTA complete (teardown)
   uint32_t tmem_base;
   int abort_flag;
-  float scale[kMaxBN];       // s_x * scale[n]
-  float bias[kMaxBN];
 };
 
-constexpr size_t kGemmSmemBytes =
-    1024 /*alignment slack*/ + static_cast<size_t>(kStages) * (kA16Bytes + kB16Bytes + kA8Bytes) +
-    sizeof(GemmSmemTail);
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out) {
+  return 1024 + static_cast<size_t>(stages) * (kStageBlocks * BN * 128 + kA8Stage) +
+         4 * 2 * (f32_out ? kEpiBuf32 : kEpiBuf16) + kScaleBytes + sizeof(GemmBarriers);
+}
 
-__device__ __forceinline__ void record_failure(GemmSmemTail* tl, unsigned code) {
-  *reinterpret_cast<volatile int*>(&tl->abort_flag) = 1;
+int gemm_max_stages(int BN, bool f32_out) {
+  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out);
+  const size_t per = static_cast<size_t>(kStageBlocks) * BN * 128 + kA8Stage;
+  const int s = static_cast<int>((232448 - fixed) / per);
+  return s < kMaxStages ? s : kMaxStages;
+}
+
+int gemm_a_stages(int BN) {
+  const int s = (kTmemCols - 2 * BN) / kASlotCols;
+  return s < kMaxStages ? s : kMaxStages;
+}
+
+__device__ __forceinline__ void record_failure(GemmBarriers* b, unsigned code) {
+  *reinterpret_cast<volatile int*>(&b->abort_flag) = 1;
   atomicOr(&g_gemm_err, code);
 }
 
-__global__ void __launch_bounds__(192, 1)
+struct TileCoord {
+  int m_tile, n_tile, split, kb_begin, kb_end;
+};
+
+__device__ __forceinline__ TileCoord tile_coord(const GemmParams& p, int t) {
+  TileCoord c;
+  const int tiles_mn = p.m_tiles * p.n_tiles;
+  c.split = t / tiles_mn;
+  const int r = t - c.split * tiles_mn;
+  c.n_tile = r / p.m_tiles;
+  c.m_tile = r - c.n_tile * p.m_tiles;
+  c.kb_begin = c.split * p.kb_per_split;
+  c.kb_end = min(p.num_kb, c.kb_begin + p.kb_per_split);
+  return c;
+}
+
+// Ring position: slot index and the parity of the slot's current lap.
+struct Ring {
+  int s = 0;
+  uint32_t ph = 0;
+  uint32_t lap0 = 1;  // 1 while still in the first lap over the slots
+  __device__ __forceinline__ void next(int S) {
+    if (++s == S) {
+      s = 0;
+      ph ^= 1u;
+      lap0 = 0;
+    }
+  }
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
     aq_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
-                   const __grid_constant__ CUtensorMap mapB, const GemmParams p) {
+                   const __grid_constant__ CUtensorMap mapB,
+                   const __grid_constant__ CUtensorMap mapY, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* a16 = smem;
-  uint8_t* b16 = a16 + kStages * kA16Bytes;
-  uint8_t* a8 = b16 + kStages * kB16Bytes;
-  GemmSmemTail* tl = reinterpret_cast<GemmSmemTail*>(a8 + kStages * kA8Bytes);
-  const volatile int* abort_flag = &tl->abort_flag;
+  const int S = p.stages;
+  const int SA = p.a_stages;
+  const int BN = p.BN;
+  const int b_half = BN * 128;                 // one 64-wide fp16 B box
+  const int b_stage = kStageBlocks * b_half;
+  const bool raw = p.partial != nullptr;
+  const bool f32 = raw || p.out_f32;
+  const int epi_buf = f32 ? kEpiBuf32 : kEpiBuf16;
+  uint8_t* bring = smem;
+  uint8_t* aring = bring + S * b_stage;
+  uint8_t* epi = aring + S * kA8Stage;
+  float* sscale = reinterpret_cast<float*>(epi + 4 * 2 * epi_buf);
+  GemmBarriers* bar =
+      reinterpret_cast<GemmBarriers*>(reinterpret_cast<uint8_t*>(sscale) + kScaleBytes);
+  const volatile int* abort_flag = &bar->abort_flag;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int BN = p.BN;
-  const int n0 = blockIdx.x * BN;
-  const int mt = blockIdx.y;
-  const int m0 = mt * kBM;
-  const int split = blockIdx.z;
-  const int kb_begin = split * p.kb_per_split;
-  const int kb_end = min(p.num_kb, kb_begin + p.kb_per_split);
-  const int nk = kb_end - kb_begin;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&tl->full[s], 1);
-      mbar_init(&tl->conv[s], 4);
-      mbar_init(&tl->empty[s], 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&bar->full[s], 1);
+      mbar_init(&bar->empty[s], 5);
     }
-    mbar_init(&tl->accum, 1);
-    tl->abort_flag = 0;
+    for (int s = 0; s < SA; ++s) {
+      bar->a_ready[s] = 0;
+      mbar_init(&bar->a_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar->acc_full[b], 1);
+      mbar_init(&bar->acc_empty[b], 4);
+    }
+    mbar_init(&bar->drain, 1);
+    bar->abort_flag = 0;
     mbar_fence_init();
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapB);
+    tma_prefetch_desc(&mapY);
   }
   if (warp == 1) {
-    tmem_alloc(&tl->tmem_base, kTmemCols);
+    tmem_alloc(&bar->tmem_base, kTmemCols);
     tmem_relinquish();
-  }
-  for (int i = threadIdx.x; i < BN; i += blockDim.x) {
-    const int n = n0 + i;
-    tl->scale[i] = (n < p.N) ? p.s_x * __half2float(p.scale[n]) : 0.0f;
-    tl->bias[i] = (n < p.N && p.bias != nullptr) ? __half2float(p.bias[n]) : 0.0f;
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem_base = tl->tmem_base;
+  const uint32_t tmem_base = bar->tmem_base;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    if (lane == 0 && nk > 0) {
-      int b0 = 0, ho0 = 0;
-      if (p.conv) {
-        if (p.imgs_per_tile > 0) {
-          b0 = mt * p.imgs_per_tile;
-        } else {
-          b0 = mt / p.tiles_per_img;
-          ho0 = (mt % p.tiles_per_img) * p.rows_per_tile;
+    // ================================================================ TMA producer
+    if (lane == 0) {
+      Ring rg;
+      uint32_t issued = 0;
+      bool failed = false;
+      for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
+        const TileCoord tc = tile_coord(p, t);
+        const int m0 = tc.m_tile * kBM;
+        const int n0 = tc.n_tile * BN;
+        int b0 = 0, ho0 = 0, tap = 0, cb = 0;
+        if (p.conv) {
+          if (p.imgs_per_tile > 0) {
+            b0 = tc.m_tile * p.imgs_per_tile;
+          } else {
+            b0 = tc.m_tile / p.tiles_per_img;
+            ho0 = (tc.m_tile - b0 * p.tiles_per_img) * p.rows_per_tile;
+          }
+          tap = tc.kb_begin / p.cin_blocks;
+          cb = tc.kb_begin - tap * p.cin_blocks;
         }
-      }
-      const uint32_t stage_bytes = kA8Bytes + static_cast<uint32_t>(BN) * 128u;
-      int issued = 0;
-      for (int i = 0; i < nk; ++i) {
-        const int s = i % kStages;
-        const uint32_t ph = (i / kStages) & 1u;
-        if (i >= kStages && !mbar_wait(&tl->empty[s], ph ^ 1u, abort_flag)) {
-          record_failure(tl, kDevErrTimeoutEmpty);
-          break;
+        for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
+          const int nb = min(kStageBlocks, tc.kb_end - kb);
+          if (!rg.lap0 && !mbar_wait(&bar->empty[rg.s], rg.ph ^ 1u, abort_flag)) {
+            if (!*abort_flag) record_failure(bar, kDevErrTimeoutEmpty);
+            failed = true;
+            break;
+          }
+          uint64_t* fb = &bar->full[rg.s];
+          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (kA8Half + b_half)));
+          uint8_t* a_dst = aring + rg.s * kA8Stage;
+          uint8_t* b_dst = bring + rg.s * b_stage;
+          for (int h = 0; h < nb; ++h) {
+            const int k = kb + h;
+            if (!p.conv) {
+              tma_load_2d(a_dst + h * kA8Half, &mapA, fb, k * kBK, m0);
+            } else {
+              const int kh = tap / 3, kw = tap - 3 * (tap / 3);
+              tma_load_4d(a_dst + h * kA8Half, &mapA, fb, cb * kBK, kw - p.pad, ho0 + kh - p.pad, b0);
+              if (++cb == p.cin_blocks) {
+                cb = 0;
+                ++tap;
+              }
+            }
+            tma_load_2d(b_dst + h * b_half, &mapB, fb, k * kBK, n0);
+          }
+          ++issued;
+          rg.next(S);
         }
-        if (*abort_flag) break;
-        const int kb = kb_begin + i;
-        mbar_arrive_expect_tx(&tl->full[s], stage_bytes);
-        if (!p.conv) {
-          tma_load_2d(a8 + s * kA8Bytes, &mapA, &tl->full[s], kb * kBK, m0);
-        } else {
-          const int tap = kb / p.cin_blocks;
-          const int c0 = (kb - tap * p.cin_blocks) * kBK;
-          const int kh = tap / 3, kw = tap - 3 * (tap / 3);
-          tma_load_4d(a8 + s * kA8Bytes, &mapA, &tl->full[s], c0, kw - p.pad, ho0 + kh - p.pad,
-                      b0);
-        }
-        tma_load_2d(b16 + s * kB16Bytes, &mapB, &tl->full[s], kb * kBK, n0);
-        ++issued;
       }
       if (*abort_flag) {
-        // drain: the last (up to kStages) issued stages may still be in flight
+        // drain: the stages issued in the last lap may still be in flight
         const int zero = 0;
-        for (int i = max(0, issued - kStages); i < issued; ++i) {
-          if (!mbar_wait(&tl->full[i % kStages], (i / kStages) & 1u, &zero)) {
+        Ring d;
+        const uint32_t first = issued > static_cast<uint32_t>(S) ? issued - S : 0u;
+        for (uint32_t i = 0; i < issued; ++i) {
+          if (i >= first && !mbar_wait(&bar->full[d.s], d.ph, &zero)) {
             atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
             break;
           }
+          d.next(S);
         }
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && nk > 0) {
+    // ================================================================ MMA issuer
+    if (lane == 0) {
       const uint32_t idesc = idesc_f16_f32(kBM, BN);
-      for (int i = 0; i < nk; ++i) {
-        const int s = i % kStages;
-        const uint32_t ph = (i / kStages) & 1u;
-        if (!mbar_wait(&tl->full[s], ph, abort_flag) || !mbar_wait(&tl->conv[s], ph, abort_flag)) {
-          record_failure(tl, kDevErrTimeoutConv);
+      const uint64_t bdesc0 = sw128_kmajor_desc(smem_u32(bring));
+      const uint64_t bstep = static_cast<uint64_t>(b_stage >> 4);  // descriptor units: 16 B
+      const uint64_t bhalf = static_cast<uint64_t>(b_half >> 4);
+      const uint32_t a_slot0 = tmem_base + static_cast<uint32_t>(p.a_col);
+      int s = 0, sa = 0;
+      uint32_t a_target = 4;     // a_ready value that marks the current lap of the A ring
+      uint32_t lt = 0;
+      bool failed = false;
+      for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
+        int nblk = p.num_kb;
+        if (p.splits > 1) {
+          const TileCoord tc = tile_coord(p, t);
+          nblk = tc.kb_end - tc.kb_begin;
+        }
+        const int nst = (nblk + 1) >> 1;
+        const bool half_tail = (nblk & 1) != 0;
+        const int buf = static_cast<int>(lt & 1u);
+        if (lt >= 2 && !mbar_wait(&bar->acc_empty[buf], ((lt >> 1) & 1u) ^ 1u, abort_flag)) {
+          if (!*abort_flag) record_failure(bar, kDevErrTimeoutAccum);
           break;
         }
         tc_fence_after();
-        const uint32_t a_base = smem_u32(a16 + s * kA16Bytes);
-        const uint32_t b_base = smem_u32(b16 + s * kB16Bytes);
-#pragma unroll
-        for (int k = 0; k < kBK / 16; ++k) {
-          mma_f16_ss(tmem_base, sw128_kmajor_desc(a_base + 32u * k),
-                     sw128_kmajor_desc(b_base + 32u * k), idesc, (i | k) != 0 ? 1u : 0u);
+        const uint32_t d = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
+        for (int st = 0; st < nst; ++st) {
+          if (!ctr_wait(&bar->a_ready[sa], a_target, abort_flag)) {
+            if (!*abort_flag) record_failure(bar, kDevErrTimeoutConv);
+            failed = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = a_slot0 + static_cast<uint32_t>(kASlotCols * sa);
+          const uint64_t b0 = bdesc0 + static_cast<uint64_t>(s) * bstep;
+          const uint64_t b1 = b0 + bhalf;
+          mma_f16_ts(d, a, b0, idesc, st > 0 ? 1u : 0u);
+          mma_f16_ts(d, a + 8u, b0 + 2u, idesc, 1u);
+          mma_f16_ts(d, a + 16u, b0 + 4u, idesc, 1u);
+          mma_f16_ts(d, a + 24u, b0 + 6u, idesc, 1u);
+          if (!(half_tail && st == nst - 1)) {
+            mma_f16_ts(d, a + 32u, b1, idesc, 1u);
+            mma_f16_ts(d, a + 40u, b1 + 2u, idesc, 1u);
+            mma_f16_ts(d, a + 48u, b1 + 4u, idesc, 1u);
+            mma_f16_ts(d, a + 56u, b1 + 6u, idesc, 1u);
+          }
+          mma_commit(&bar->empty[s]);
+          mma_commit(&bar->a_empty[sa]);
+          if (++s == S) s = 0;
+          if (++sa == SA) {
+            sa = 0;
+            a_target += 4;
+          }
         }
-        mma_commit(&tl->empty[s]);
+        if (!failed) mma_commit(&bar->acc_full[buf]);
       }
-      mma_commit(&tl->accum);
-      if (*abort_flag) {
-        const int zero = 0;
-        if (!mbar_wait(&tl->accum, 0, &zero)) atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
+      // every MMA of this CTA completes before teardown frees tensor memory
+      mma_commit(&bar->drain);
+      const int zero = 0;
+      if (!mbar_wait(&bar->drain, 0, &zero)) atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
+    }
+  } else if (warp < 6) {
+    // ================================================================ converters
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const int swz = (row >> 1) & 3;            // 64-byte swizzle of the int8 box
+    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    Ring rg;   // smem ring
+    Ring ra;   // TMEM A ring
+    bool failed = false;
+    for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
+      const TileCoord tc = tile_coord(p, t);
+      for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
+        const int nb = min(kStageBlocks, tc.kb_end - kb);
+        bool okw = mbar_wait(&bar->full[rg.s], rg.ph, abort_flag);
+        if (okw && !ra.lap0) okw = mbar_wait(&bar->a_empty[ra.s], ra.ph ^ 1u, abort_flag);
+        if (!okw) {
+          if (!*abort_flag) record_failure(bar, kDevErrTimeoutFull);
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const uint8_t* src = aring + rg.s * kA8Stage + row * 64;
+        const uint32_t slot = t_row + static_cast<uint32_t>(p.a_col + kASlotCols * ra.s);
+        for (int h = 0; h < nb; ++h) {
+          uint32_t v[32];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const uint4 w = *reinterpret_cast<const uint4*>(src + h * kA8Half + ((c ^ swz) << 4));
+            i8x4_to_f16x4(w.x, v[8 * c + 0], v[8 * c + 1]);
+            i8x4_to_f16x4(w.y, v[8 * c + 2], v[8 * c + 3]);
+            i8x4_to_f16x4(w.z, v[8 * c + 4], v[8 * c + 5]);
+            i8x4_to_f16x4(w.w, v[8 * c + 6], v[8 * c + 7]);
+          }
+          tmem_st_32x32b_x32(slot + 32u * h, v);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          smem_release_add(&bar->a_ready[ra.s], 1u);
+          mbar_arrive(&bar->empty[rg.s]);
+        }
+        rg.next(S);
+        ra.next(SA);
       }
     }
   } else {
-    // ------------------------------------------------------------ converters
-    const int ct = threadIdx.x - 64;  // 0..127
-    for (int i = 0; i < nk; ++i) {
-      const int s = i % kStages;
-      const uint32_t ph = (i / kStages) & 1u;
-      if (!mbar_wait(&tl->full[s], ph, abort_flag)) {
-        record_failure(tl, kDevErrTimeoutFull);
-        break;
-      }
-      const uint8_t* src = a8 + s * kA8Bytes;
-      uint8_t* dst = a16 + s * kA16Bytes;
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int q = ct + 128 * j;
-        const int row = q >> 2;
-        const int c = q & 3;
-        const uint4 v = *reinterpret_cast<const uint4*>(src + row * 64 + c * 16);
-        uint32_t o[8];
-        i8x4_to_f16x4(v.x, o[0], o[1]);
-        i8x4_to_f16x4(v.y, o[2], o[3]);
-        i8x4_to_f16x4(v.z, o[4], o[5]);
-        i8x4_to_f16x4(v.w, o[6], o[7]);
-        const int sw = row & 7;
-        *reinterpret_cast<uint4*>(dst + row * 128 + (((2 * c) ^ sw) << 4)) =
-            make_uint4(o[0], o[1], o[2], o[3]);
-        *reinterpret_cast<uint4*>(dst + row * 128 + (((2 * c + 1) ^ sw) << 4)) =
-            make_uint4(o[4], o[5], o[6], o[7]);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tl->conv[s]);
-    }
-
-    // ------------------------------------------------------------ epilogue
-    bool ok = nk > 0 && mbar_wait(&tl->accum, 0, abort_flag);
-    if (nk > 0 && !ok && !*abort_flag) record_failure(tl, kDevErrTimeoutAccum);
-    ok = __all_sync(0xffffffffu, ok ? 1 : 0) != 0;
-    if (ok) {
-      tc_fence_after();
-      const int qd = warp & 3;                 // TMEM lane quadrant of this warp
-      const int row = qd * 32 + lane;
-      const int t = m0 + row;
-      const uint32_t tq = tmem_base + (static_cast<uint32_t>(qd * 32) << 16);
-      const int cols = min(BN, p.N - n0);      // valid columns of this tile
-      for (int c0 = 0; c0 < BN; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tq + static_cast<uint32_t>(c0), r);
-        tmem_wait_ld();
-        if (t < p.T) {
-          if (p.partial != nullptr) {
-            float* dst = p.partial + (static_cast<int64_t>(split) * p.T + t) * p.N + n0;
-#pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              if (c0 + j < cols)
-                *reinterpret_cast<float4*>(dst + c0 + j) =
-                    make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
-                                __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
-            }
-          } else if (p.out_f32) {
-            float* dst = static_cast<float*>(p.y) + static_cast<int64_t>(t) * p.N + n0;
-#pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              if (c0 + j < cols) {
-                float4 v;
-                v.x = fmaf(__uint_as_float(r[j]), tl->scale[c0 + j], tl->bias[c0 + j]);
-                v.y = fmaf(__uint_as_float(r[j + 1]), tl->scale[c0 + j + 1], tl->bias[c0 + j + 1]);
-                v.z = fmaf(__uint_as_float(r[j + 2]), tl->scale[c0 + j + 2], tl->bias[c0 + j + 2]);
-                v.w = fmaf(__uint_as_float(r[j + 3]), tl->scale[c0 + j + 3], tl->bias[c0 + j + 3]);
-                *reinterpret_cast<float4*>(dst + c0 + j) = v;
-              }
-            }
-          } else {
-            __half* dst = static_cast<__half*>(p.y) + static_cast<int64_t>(t) * p.N + n0;
-#pragma unroll
-            for (int j = 0; j < 32; j += 8) {
-              if (c0 + j < cols) {
-                uint32_t w[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  const int cc = c0 + j + 2 * e;
-                  const float lo = fmaf(__uint_as_float(r[j + 2 * e]), tl->scale[cc], tl->bias[cc]);
-                  const float hi =
-                      fmaf(__uint_as_float(r[j + 2 * e + 1]), tl->scale[cc + 1], tl->bias[cc + 1]);
-                  __half2 h = __floats2half2_rn(lo, hi);
-                  w[e] = *reinterpret_cast<uint32_t*>(&h);
-                }
-                *reinterpret_cast<uint4*>(dst + c0 + j) = make_uint4(w[0], w[1], w[2], w[3]);
-              }
-            }
-          }
+    // ================================================================ epilogue
+    const int q = warp & 3;
+    const int ew = warp - 6;
+    float* wscale = sscale + ew * 2 * kMaxBN;
+    float* wbias = wscale + kMaxBN;
+    uint8_t* wbuf = epi + ew * 2 * epi_buf;
+    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    uint32_t lt = 0, chunk = 0;
+    for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
+      const TileCoord tc = tile_coord(p, t);
+      const int buf = static_cast<int>(lt & 1u);
+      const int m0 = tc.m_tile * kBM;
+      const int n0 = tc.n_tile * BN;
+      if (!raw) {
+        // this tile's scale/bias, loaded while the accumulator is still being computed
+        for (int i = lane; i < BN; i += 32) {
+          const int n = n0 + i;
+          wscale[i] = (n < p.N) ? p.s_x * __half2float(p.scale[n]) : 0.0f;
+          wbias[i] = (n < p.N && p.bias != nullptr) ? __half2float(p.bias[n]) : 0.0f;
         }
       }
+      if (!mbar_wait(&bar->acc_full[buf], (lt >> 1) & 1u, abort_flag)) {
+        if (!*abort_flag) record_failure(bar, kDevErrTimeoutAccum);
+        break;
+      }
+      tc_fence_after();
+      __syncwarp();
+      const uint32_t tacc = t_row + static_cast<uint32_t>(buf * p.acc_stride);
+      for (int c0 = 0; c0 < BN; c0 += 32, ++chunk) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tacc + static_cast<uint32_t>(c0), r);
+        tmem_wait_ld();
+        if (c0 + 32 >= BN) {
+          // last read of this accumulator buffer: hand it back to the MMA warp
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar->acc_empty[buf]);
+        }
+        uint8_t* dst = wbuf + (chunk & 1u) * epi_buf;
+        if (lane == 0) bulk_wait_group_read<1>();   // the store issued from dst two chunks ago
+        __syncwarp();
+        if (f32) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 o;
+            o.x = __uint_as_float(r[4 * j + 0]);
+            o.y = __uint_as_float(r[4 * j + 1]);
+            o.z = __uint_as_float(r[4 * j + 2]);
+            o.w = __uint_as_float(r[4 * j + 3]);
+            if (!raw) {
+              const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
+              const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
+              o.x = fmaf(o.x, sc.x, bi.x);
+              o.y = fmaf(o.y, sc.y, bi.y);
+              o.z = fmaf(o.z, sc.z, bi.z);
+              o.w = fmaf(o.w, sc.w, bi.w);
+            }
+            *reinterpret_cast<float4*>(dst + lane * 128 + ((j ^ (lane & 7)) << 4)) = o;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const float4 sc0 = *reinterpret_cast<const float4*>(wscale + c0 + 8 * j);
+            const float4 sc1 = *reinterpret_cast<const float4*>(wscale + c0 + 8 * j + 4);
+            const float4 bi0 = *reinterpret_cast<const float4*>(wbias + c0 + 8 * j);
+            const float4 bi1 = *reinterpret_cast<const float4*>(wbias + c0 + 8 * j + 4);
+            const float* rr = reinterpret_cast<const float*>(r) + 8 * j;
+            __half2 h0 = __floats2half2_rn(fmaf(rr[0], sc0.x, bi0.x), fmaf(rr[1], sc0.y, bi0.y));
+            __half2 h1 = __floats2half2_rn(fmaf(rr[2], sc0.z, bi0.z), fmaf(rr[3], sc0.w, bi0.w));
+            __half2 h2 = __floats2half2_rn(fmaf(rr[4], sc1.x, bi1.x), fmaf(rr[5], sc1.y, bi1.y));
+            __half2 h3 = __floats2half2_rn(fmaf(rr[6], sc1.z, bi1.z), fmaf(rr[7], sc1.w, bi1.w));
+            *reinterpret_cast<uint4*>(dst + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                make_uint4(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1),
+                           *reinterpret_cast<uint32_t*>(&h2), *reinterpret_cast<uint32_t*>(&h3));
+          }
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          if (raw)
+            tma_store_3d(&mapY, dst, n0 + c0, m0 + q * 32, tc.split);
+          else
+            tma_store_2d(&mapY, dst, n0 + c0, m0 + q * 32);
+          bulk_commit_group();
+        }
+        __syncwarp();
+      }
     }
+    if (lane == 0) bulk_wait_group_all();
   }
 
   tc_fence_before();
@@ -286,8 +445,8 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
     const int n = static_cast<int>(q - t * (p.N / 4)) * 4;
     float4 acc = *reinterpret_cast<const float4*>(p.partial + t * p.N + n);
     for (int s = 1; s < splits; ++s) {
-      const float4 v =
-          *reinterpret_cast<const float4*>(p.partial + (static_cast<int64_t>(s) * p.T + t) * p.N + n);
+      const float4 v = *reinterpret_cast<const float4*>(
+          p.partial + (static_cast<int64_t>(s) * p.T + t) * p.N + n);
       acc.x += v.x;
       acc.y += v.y;
       acc.z += v.z;
@@ -312,17 +471,17 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
   }
 }
 
-cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const GemmParams& p,
-                        int n_tiles, int m_tiles, int splits, cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
+                        const GemmParams& p, int grid, cudaStream_t st) {
+  static int configured_bytes = 0;
+  const size_t bytes = gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr);
+  if (static_cast<int>(bytes) > configured_bytes) {
     cudaError_t e = cudaFuncSetAttribute(aq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kGemmSmemBytes));
+                                         static_cast<int>(bytes));
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    configured_bytes = static_cast<int>(bytes);
   }
-  dim3 grid(n_tiles, m_tiles, splits);
-  aq_gemm_kernel<<<grid, 192, kGemmSmemBytes, st>>>(mapA, mapB, p);
+  aq_gemm_kernel<<<grid, kThreads, bytes, st>>>(mapA, mapB, mapY, p);
   return cudaGetLastError();
 }
 

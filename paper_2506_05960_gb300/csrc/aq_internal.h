@@ -11,15 +11,21 @@ namespace aq {
 
 // ---- tile geometry of the tensor-core GEMM
 constexpr int kBM = 128;        // rows (tokens / output pixels) per tile = TMEM lanes
-constexpr int kBK = 64;         // K per pipeline stage (128 bytes of fp16 = one swizzle row)
-constexpr int kMaxBN = 256;     // widest N tile (TMEM columns of the fp32 accumulator)
+constexpr int kBK = 64;         // K per TMA box / swizzle row (128 bytes of fp16)
+constexpr int kStageBlocks = 2; // 64-wide K blocks per pipeline stage (8 MMAs of K = 16)
+constexpr int kMaxBN = 192;     // widest N tile: 2 fp32 accumulators + >= 2 A stages in TMEM
+constexpr int kMaxStages = 8;   // pipeline ring depth bound
 
 // Parameters of one GEMM launch (passed by value).
 struct GemmParams {
   int T, N, K;                  // rows, output channels, reduction length
-  int BN;                       // N tile (multiple of 16, <= 256)
+  int BN;                       // N tile (multiple of 32, <= kMaxBN)
   int num_kb;                   // ceil(K / 64)
-  int kb_per_split;             // K blocks per split (grid.z splits)
+  int kb_per_split;             // K blocks per split
+  int m_tiles, n_tiles, splits, total_tiles;
+  int stages;                   // smem ring depth (TMA stages of 128 K)
+  int a_stages;                 // TMEM A ring depth (slots of 128 K = 64 columns)
+  int acc_stride, a_col;        // TMEM columns: accumulator buffer stride, first A slot
   // implicit-GEMM convolution (conv != 0): A is loaded per tap with a 4-D TMA box
   int conv, cin_blocks, pad, tiles_per_img, rows_per_tile, imgs_per_tile;
   // epilogue
@@ -37,8 +43,11 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
-cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const GemmParams& p,
-                        int n_tiles, int m_tiles, int splits, cudaStream_t st);
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out);
+int gemm_max_stages(int BN, bool f32_out);   // smem ring depth that fits shared memory
+int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-column accumulators
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
+                        const GemmParams& p, int grid, cudaStream_t st);
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st);
 
 // Device error words of each translation unit (read and cleared, synchronising).
