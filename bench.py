@@ -12,8 +12,8 @@ Timing: CUDA-graph replay of 8 steps that rotate over 8 independent buffer
 sets (inputs, codes, outputs: > 300 MB together, larger than the 129 MB L2),
 CUDA events on the launching stream, warm-up first, barrier + synchronize on
 both sides, max over ranks.  The dominant kernel (the tensor-core GEMM) is
-timed by the library's own event pairs in a second captured graph inside the
-same timed region.  `e2e` repeats the step through the public C ABI with the
+timed by the library's own event pairs, captured as event-record nodes into a
+second graph that is replayed once inside the same timed region.  `e2e` repeats the step through the public C ABI with the
 input copied from pinned host memory and the output copied back every step.
 
 --impl reference times the CPU oracle (plain numpy fp64) on the same workload.
@@ -293,9 +293,15 @@ def main():
     aq.aq_profile_enable(False)
     assert aq.aq_device_error() == 0
 
-    # capture the main graph (NSETS steps, one per buffer set)
+    # capture the main graph (NSETS steps, one per buffer set) and a copy whose library
+    # calls carry event-record nodes around every kernel (for per-kernel device time)
     g_main = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_main, stream=stream):
+        for i in range(NSETS):
+            step(bufs[i], stream)
+    aq.aq_profile_enable(True)
+    g_prof = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_prof, stream=stream):
         for i in range(NSETS):
             step(bufs[i], stream)
     for _ in range(2):
@@ -316,14 +322,7 @@ def main():
         for _ in range(reps):
             g_main.replay()
         ev1.record(stream)
-        pad_reps = max(0, 64 - reps)       # keep >= 64 replays queued ahead of the timed kernels
-        for _ in range(pad_reps):
-            g_main.replay()
-        # kernel timing: eager steps with the library's event pairs, enqueued while the GPU
-        # is still busy with the replays above, so they run back to back like the graph
-        aq.aq_profile_enable(True)
-        for i in range(2 * NSETS):
-            step(bufs[i % NSETS], stream)
+        g_prof.replay()          # per-kernel event pairs (read below)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
@@ -346,7 +345,7 @@ def main():
     achieved = fl / (gemm_avg_ms * 1e-3) / 1e12
     tr = TRAFFIC.get(args.workload, {})
     traffic = tr.get("bytes") if tr.get("sources_sha") == sources_sha() else None
-    launches_per_step = sum(n for k, (ms, n) in prof.items()) / (2 * NSETS)
+    launches_per_step = sum(n for k, (ms, n) in prof.items()) / NSETS
 
     # e2e through the public API: pinned host input -> device, step, device -> pinned host
     h_x = [torch.from_numpy(inp["x16"]).pin_memory() for inp in sets[:2]]
@@ -400,8 +399,7 @@ def main():
             "e2e": {"value": world * fl / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                     "ms_per_step": e2e_ms, "h2d_bytes_per_step": T * K * 2,
                     "d2h_bytes_per_step": T * N * 2},
-            "gpu_launches": int(round(launches_per_step * (steps + pad_reps * NSETS)))
-            + sum(n for _, n in prof.values()),
+            "gpu_launches": int(round(launches_per_step * steps)) + sum(n for _, n in prof.values()),
             "clocks": clocks,
         }
         print(json.dumps(line), flush=True)

@@ -96,7 +96,10 @@ AQ_API int aq_device_error(int* code_out);
  * milliseconds and the number of launches since the last aq_profile_enable().
  * Kinds: 0 quantizer, 1 pack, 2 decode, 3 tensor-core GEMM, 4 split-K reduce,
  * 5 LUT build, 6 LUT gather, 7 fused-decode GEMM.  Uses host-side CUDA events
- * only (no device memory).  Not for use inside CUDA graph capture.          */
+ * only (no device memory).  Calls captured into a CUDA graph record external
+ * event nodes: replay the graph once, then read (a read reports the last
+ * replay).  Event creation happens on first use: make one uncaptured call
+ * with timing enabled before capturing.                                      */
 #define AQ_PROFILE_KINDS 8
 AQ_API int aq_profile_enable(int on);
 AQ_API int aq_profile_read(double* ms_out, int64_t* launches_out, int n_kinds);

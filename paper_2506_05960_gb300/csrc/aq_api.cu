@@ -80,12 +80,16 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
+// elem_strides (optional): traversal stride per dimension; a box dimension of
+// size b with traversal stride s delivers b / s elements (b a multiple of s).
 int encode(CUtensorMap* map, CUtensorMapDataType dt, int rank, const void* base,
            const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box,
-           CUtensorMapSwizzle sw) {
+           CUtensorMapSwizzle sw, const cuuint32_t* elem_strides = nullptr) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return set_error(AQ_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
   cuuint32_t es[5] = {1, 1, 1, 1, 1};
+  if (elem_strides)
+    for (int i = 0; i < rank; ++i) es[i] = elem_strides[i];
   CUresult r = fn(map, dt, static_cast<cuuint32_t>(rank), const_cast<void*>(base), dims, strides,
                   box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -112,33 +116,48 @@ double stage_cycles(int BN) {
   return 8.0 * mma + exposed;
 }
 
-void finish_plan(Plan& pl, bool f32_out) {
+// Fused path: the four decoder warps rebuild BN x 16 groups per stage, each group
+// about 12 + 12*M instructions (twice that for 2^16-entry books gathered from L2).
+double decode_stage_cycles(int BN, int M, int B) {
+  const double per_group = (12.0 + 12.0 * M) * (B == 16 ? 2.0 : 1.0);
+  return BN * 16.0 * per_group / 128.0;
+}
+
+int book_smem_bytes(bool fused, int M, int B) { return (fused && B == 8) ? M * 256 * 16 : 0; }
+
+void finish_plan(Plan& pl, bool f32_out, int book_bytes) {
   pl.acc_stride = pl.BN;
   pl.a_col = 2 * pl.acc_stride;
   pl.a_stages = aq::gemm_a_stages(pl.BN);
-  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1);
+  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1, book_bytes);
   pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
 }
 
 // Picks the N tile and the K split that minimise a model of the busiest SM's time:
 // waves x (stage cycles x stages per tile + a fixed tile overhead), plus the traffic
-// and launch of the split-K reduction when K is split.  Depends only on the shapes.
-Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out) {
+// and launch of the split-K reduction when K is split.  Depends only on the shapes
+// (and, for the fused path, on the code format).
+Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
+               bool fused = false, int M = 1, int B = 8) {
   const int num_kb = (K + aq::kBK - 1) / aq::kBK;
+  const int book_bytes = book_smem_bytes(fused, M, B);
   double best = 1e30;
   Plan bp{};
   for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
     if (BN == 224) continue;
     if (aq::gemm_a_stages(BN) < 2) continue;
+    if (aq::gemm_max_stages(BN, true, book_bytes) < 2) continue;
     const int n_tiles = (N + BN - 1) / BN;
     const int max_split = allow_split ? std::min(num_kb, 64) : 1;
+    double st_cyc = stage_cycles(BN);
+    if (fused) st_cyc = std::max(st_cyc, decode_stage_cycles(BN, M, B));
     for (int sp = 1; sp <= max_split; ++sp) {
       const int kbps = (num_kb + sp - 1) / sp;
       const int s_eff = (num_kb + kbps - 1) / kbps;
       if (s_eff != sp) continue;
       const long tiles = static_cast<long>(m_tiles) * n_tiles * s_eff;
       const long waves = (tiles + kPlanSMs - 1) / kPlanSMs;
-      const double tile_cycles = (kbps / 2) * stage_cycles(BN) + (kbps & 1) * 0.5 * stage_cycles(BN) + 800.0;
+      const double tile_cycles = (kbps / 2) * st_cyc + (kbps & 1) * 0.5 * st_cyc + 800.0;
       double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
       if (s_eff > 1) t += (s_eff * 8.0 + 2.0) * T * static_cast<double>(N) / 6.0e12 + 2.0e-6;
       if (t < best * 0.999) {
@@ -153,7 +172,7 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out)
       }
     }
   }
-  finish_plan(bp, f32_out);
+  finish_plan(bp, f32_out, book_bytes);
   return bp;
 }
 
@@ -163,10 +182,78 @@ size_t dense_ws_bytes(int T, int N, int K, const Plan& pl) {
   return b;
 }
 
-int resolve_path(int path) {
-  if (path == AQ_PATH_AUTO) return AQ_PATH_DENSE;
-  if (path == AQ_PATH_DENSE) return AQ_PATH_DENSE;
-  return -1;
+// Fused path workspace: only the split-K partial sums (no decoded weights).
+size_t fused_ws_bytes(int T, int N, const Plan& pl) {
+  return pl.splits > 1 ? align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024) : 0;
+}
+
+// AUTO decodes inside the GEMM (fused path) when every weight tile is decoded by at
+// most this many CTAs (one per 128-row M tile); beyond it a separate decode pass
+// into the workspace is cheaper.
+constexpr int kFusedAutoMaxMTiles = 1;
+
+// Path of a convolution: -1 unknown path, -2 path cannot run this layer.
+int resolve_conv_path(int path, int m_tiles) {
+  switch (path) {
+    case AQ_PATH_AUTO:
+      return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
+    case AQ_PATH_DENSE:
+    case AQ_PATH_FUSED:
+      return path;
+    case AQ_PATH_LUT:
+      return -2;
+    default:
+      return -1;
+  }
+}
+
+// ---- lookup-table path (linear layers, 8-bit codes, T <= 16)
+constexpr int kLutMaxT = 16;       // tokens per call the LUT kernel handles
+constexpr int kLutAutoMaxT = 8;    // AUTO takes the LUT path up to this many tokens
+
+struct LutPlan {
+  int J, Tp, chunks, rows_per_cta;
+  size_t ws_bytes;
+};
+
+LutPlan plan_lut(int T, int K, int N, int M) {
+  LutPlan lp{};
+  lp.Tp = T <= 4 ? 4 : (T <= 8 ? 8 : 16);
+  lp.J = 8;
+  while (lp.J > 1 && static_cast<size_t>(lp.J) * M * 256 * lp.Tp * 4 > 160 * 1024) lp.J >>= 1;
+  const int G = K / 8;
+  lp.chunks = (G + lp.J - 1) / lp.J;
+  int n_slices = (2 * kPlanSMs + lp.chunks - 1) / lp.chunks;
+  if (n_slices < 1) n_slices = 1;
+  lp.rows_per_cta = ((N + n_slices - 1) / n_slices + 31) / 32 * 32;
+  lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * T * N * 4, 1024);
+  return lp;
+}
+
+// AUTO / explicit path of a linear layer: -1 unknown path, -2 path cannot run this layer.
+int resolve_linear_path(int path, int T, int B) {
+  const int m_tiles = (T + aq::kBM - 1) / aq::kBM;
+  switch (path) {
+    case AQ_PATH_AUTO:
+      if (B == 8 && T <= kLutAutoMaxT) return AQ_PATH_LUT;
+      return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
+    case AQ_PATH_DENSE:
+    case AQ_PATH_FUSED:
+      return path;
+    case AQ_PATH_LUT:
+      return (B == 8 && T <= kLutMaxT) ? AQ_PATH_LUT : -2;
+    default:
+      return -1;
+  }
+}
+
+int path_error(int rp, int path) {
+  if (rp == -2)
+    return set_error(AQ_ERR_UNSUPPORTED,
+                     "path %d cannot run this layer (the table path is for linear layers with "
+                     "8-bit codes and T <= %d)",
+                     path, kLutMaxT);
+  return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
 }
 
 // Conv tile geometry: 128 output pixels per tile as one 4-D box.
@@ -177,8 +264,8 @@ struct ConvGeom {
 int conv_geometry(int Nb, int H, int W, int kh, int kw, int stride, int pad, ConvGeom* g) {
   g->Ho = (H + 2 * pad - kh) / stride + 1;
   g->Wo = (W + 2 * pad - kw) / stride + 1;
-  if (stride != 1) return set_error(AQ_ERR_UNSUPPORTED, "conv stride %d not supported yet", stride);
   const int Wo = g->Wo, Ho = g->Ho;
+  if (stride * Wo > 256) return set_error(AQ_ERR_UNSUPPORTED, "conv output width %d too wide", Wo);
   if (Wo > aq::kBM || aq::kBM % Wo != 0)
     return set_error(AQ_ERR_UNSUPPORTED, "conv output width %d must divide 128", Wo);
   const int rpt = aq::kBM / Wo;
@@ -261,7 +348,16 @@ void fold_locked(bool accumulate) {
 }
 }  // namespace prof
 
-// Records an event pair around the launches made while it is alive.
+// Records an event pair around the launches made while it is alive.  Under stream
+// capture the records become external event-record nodes of the graph, so each
+// replay of the graph stamps them again (the last replay is what a read sees).
+cudaError_t record_event(cudaEvent_t e, cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+    return cudaEventRecordWithFlags(e, st, cudaEventRecordExternal);
+  return cudaEventRecord(e, st);
+}
+
 struct ProfScope {
   cudaStream_t st;
   int kind;
@@ -270,7 +366,8 @@ struct ProfScope {
     if (!prof::enabled.load(std::memory_order_relaxed)) return;
     std::lock_guard<std::mutex> g(prof::mu);
     a = prof::take_locked();
-    if (a && cudaEventRecord(a, st) != cudaSuccess) {
+    if (a && record_event(a, st) != cudaSuccess) {
+      (void)cudaGetLastError();
       prof::pool.push_back(a);
       a = nullptr;
     }
@@ -279,13 +376,17 @@ struct ProfScope {
     if (!a) return;
     std::lock_guard<std::mutex> g(prof::mu);
     cudaEvent_t b = prof::take_locked();
-    if (!b || cudaEventRecord(b, st) != cudaSuccess) {
+    if (!b || record_event(b, st) != cudaSuccess) {
+      (void)cudaGetLastError();
       prof::pool.push_back(a);
       if (b) prof::pool.push_back(b);
       return;
     }
     prof::pending.push_back({a, b, kind});
-    if (prof::pending.size() > 16384) prof::fold_locked(true);
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (prof::pending.size() > 16384 && cudaStreamIsCapturing(st, &cs) == cudaSuccess &&
+        cs == cudaStreamCaptureStatusNone)
+      prof::fold_locked(true);
   }
 };
 
@@ -312,8 +413,18 @@ int sm_count() {
 
 // Dense path after the activation map is built: decode W-hat into the workspace,
 // then the tensor-core GEMM with the fused epilogue (or split-K partials + reduce).
-int run_dense(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
-              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st) {
+// Tensor-core path after the activation map is built.  Dense: decode W-hat into the
+// workspace (Wdec), then the GEMM streams it with TMA.  Fused (Wdec == nullptr): the
+// GEMM's decoder warps rebuild each weight tile in shared memory from the codes.
+int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
+             const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st) {
+  const bool fused = Wdec == nullptr;
+  p.fused = fused ? 1 : 0;
+  p.codes = codes_packed;
+  p.books = codebooks;
+  p.M = M;
+  p.B = B;
+  p.book_bytes = book_smem_bytes(fused, M, B);
   p.BN = pl.BN;
   p.num_kb = pl.num_kb;
   p.kb_per_split = pl.kb_per_split;
@@ -329,7 +440,8 @@ int run_dense(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const v
   const int T = p.T, N = p.N, K = p.K;
   int r;
   CUtensorMap mapB, mapY;
-  {
+  std::memset(&mapB, 0, sizeof(mapB));
+  if (!fused) {
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
     cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(pl.BN)};
@@ -359,13 +471,13 @@ int run_dense(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const v
   }
   if (r) return r;
   cudaError_t e;
-  {
+  if (!fused) {
     ProfScope ps(kProfDecode, st);
     e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+    if (e != cudaSuccess) return cuda_status(e, "decode launch");
   }
-  if (e != cudaSuccess) return cuda_status(e, "decode launch");
   {
-    ProfScope ps(kProfGemm, st);
+    ProfScope ps(fused ? kProfFused : kProfGemm, st);
     e = aq::launch_gemm(mapA, mapB, mapY, p, std::min(pl.total_tiles, sm_count()), st);
   }
   if (e != cudaSuccess) return cuda_status(e, "gemm launch");
@@ -375,6 +487,40 @@ int run_dense(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const v
     if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
   }
   return ok();
+}
+
+// Plan and workspace layout of a tensor-core call on the dense or the fused path.
+struct Route {
+  bool fused;
+  Plan pl;
+  size_t ws;
+};
+
+Route route_gemm(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, int B) {
+  Route rt;
+  rt.fused = rp == AQ_PATH_FUSED;
+  rt.pl = plan_gemm(T, N, K, m_tiles, true, f32_out, rt.fused, M, B);
+  rt.ws = rt.fused ? fused_ws_bytes(T, N, rt.pl) : dense_ws_bytes(T, N, K, rt.pl);
+  return rt;
+}
+
+int check_workspace(const void* workspace, size_t workspace_bytes, size_t need) {
+  if (need == 0) return AQ_OK;
+  if (!workspace || workspace_bytes < need || !aligned16(workspace))
+    return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+  return AQ_OK;
+}
+
+// Dense: [decoded W-hat fp16 (N x K)][split-K partials]; fused: [split-K partials].
+void ws_pointers(const Route& rt, void* workspace, int N, int K, void** Wdec, float** partial) {
+  if (rt.fused) {
+    *Wdec = nullptr;
+    *partial = static_cast<float*>(workspace);
+  } else {
+    *Wdec = workspace;
+    *partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
+                                        align_up(static_cast<size_t>(N) * K * 2, 1024));
+  }
 }
 
 int encode_linear_a(CUtensorMap* mapA, const int8_t* xq, int T, int K) {
@@ -481,10 +627,13 @@ int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  const int rp = resolve_path(path);
-  if (rp < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
-  const Plan pl = plan_gemm(T, N, K, (T + aq::kBM - 1) / aq::kBM, true, false);
-  *bytes = dense_ws_bytes(T, N, K, pl);
+  const int rp = resolve_linear_path(path, T, B);
+  if (rp < 0) return path_error(rp, path);
+  if (rp == AQ_PATH_LUT) {
+    *bytes = plan_lut(T, K, N, M).ws_bytes;
+    return ok();
+  }
+  *bytes = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B).ws;
   return ok();
 }
 
@@ -500,21 +649,63 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
     return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
   if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite");
-  const int rp = resolve_path(path);
-  if (rp < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
+  const int rp = resolve_linear_path(path, T, B);
+  if (rp < 0) return path_error(rp, path);
   if (T == 0) return ok();
   if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
   if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
-  const Plan pl = plan_gemm(T, N, K, (T + aq::kBM - 1) / aq::kBM, true, out_dtype == AQ_DTYPE_F32);
-  const size_t need = dense_ws_bytes(T, N, K, pl);
-  if (!workspace || workspace_bytes < need || !aligned16(workspace))
-    return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+  if (rp == AQ_PATH_LUT) {
+    const LutPlan lp = plan_lut(T, K, N, M);
+    if (!workspace || workspace_bytes < lp.ws_bytes || !aligned16(workspace))
+      return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", lp.ws_bytes,
+                       workspace_bytes);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    aq::LutParams lpar{};
+    lpar.xq = xq;
+    lpar.packed = static_cast<const uint8_t*>(codes_packed);
+    lpar.books = static_cast<const __half*>(codebooks);
+    lpar.partial = static_cast<float*>(workspace);
+    lpar.T = T;
+    lpar.K = K;
+    lpar.N = N;
+    lpar.M = M;
+    lpar.Tp = lp.Tp;
+    lpar.J = lp.J;
+    lpar.G = K / 8;
+    lpar.chunks = lp.chunks;
+    lpar.rows_per_cta = lp.rows_per_cta;
+    cudaError_t e;
+    {
+      ProfScope ps(kProfLutGather, st);
+      e = aq::launch_lut(lpar, st);
+    }
+    if (e != cudaSuccess) return cuda_status(e, "LUT launch");
+    aq::GemmParams rpar{};
+    rpar.T = T;
+    rpar.N = N;
+    rpar.s_x = s_x;
+    rpar.scale = static_cast<const __half*>(scale);
+    rpar.bias = static_cast<const __half*>(bias);
+    rpar.y = y;
+    rpar.out_f32 = out_dtype == AQ_DTYPE_F32;
+    rpar.partial = lpar.partial;
+    {
+      ProfScope ps(kProfSplitK, st);
+      e = aq::launch_splitk_reduce(rpar, lp.chunks, st);
+    }
+    if (e != cudaSuccess) return cuda_status(e, "LUT reduce launch");
+    return ok();
+  }
+  const Route rt =
+      route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, out_dtype == AQ_DTYPE_F32, M, B);
+  r = check_workspace(workspace, workspace_bytes, rt.ws);
+  if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  void* Wdec = workspace;
-  float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
-                                            align_up(static_cast<size_t>(N) * K * 2, 1024));
+  void* Wdec = nullptr;
+  float* partial = nullptr;
+  ws_pointers(rt, workspace, N, K, &Wdec, &partial);
   CUtensorMap mapA;
   r = encode_linear_a(&mapA, xq, T, K);
   if (r) return r;
@@ -528,7 +719,7 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, partial, st);
+  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st);
 }
 
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
@@ -538,14 +729,14 @@ int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, in
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
   if (r) return r;
-  if (resolve_path(path) < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
+  const int rp = resolve_conv_path(path, cg.m_tiles);
+  if (rp < 0) return path_error(rp, path);
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  const Plan pl = plan_gemm(T, Cout, K, cg.m_tiles, true, false);
-  *bytes = dense_ws_bytes(T, Cout, K, pl);
+  *bytes = route_gemm(rp, T, Cout, K, cg.m_tiles, false, M, B).ws;
   return ok();
 }
 
@@ -561,10 +752,11 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
     return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
   if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite");
-  if (resolve_path(path) < 0) return set_error(AQ_ERR_UNSUPPORTED, "path %d not available", path);
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
+  const int rp = resolve_conv_path(path, cg.m_tiles);
+  if (rp < 0) return path_error(rp, path);
   if (Nb == 0) return ok();
   if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
   if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
@@ -572,24 +764,25 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  const Plan pl = plan_gemm(T, Cout, K, cg.m_tiles, true, out_dtype == AQ_DTYPE_F32);
-  const size_t need = dense_ws_bytes(T, Cout, K, pl);
-  if (!workspace || workspace_bytes < need || !aligned16(workspace))
-    return set_error(AQ_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+  const Route rt = route_gemm(rp, T, Cout, K, cg.m_tiles, out_dtype == AQ_DTYPE_F32, M, B);
+  r = check_workspace(workspace, workspace_bytes, rt.ws);
+  if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  void* Wdec = workspace;
-  float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) +
-                                            align_up(static_cast<size_t>(Cout) * K * 2, 1024));
+  void* Wdec = nullptr;
+  float* partial = nullptr;
+  ws_pointers(rt, workspace, Cout, K, &Wdec, &partial);
   CUtensorMap mapA;
   {
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W),
                           static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(Nb)};
     cuuint64_t strides[3] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W) * Cin,
                              static_cast<cuuint64_t>(H) * W * Cin};
-    cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(cg.bw),
-                         static_cast<cuuint32_t>(cg.bh), static_cast<cuuint32_t>(cg.bn)};
+    // stride s: the box spans s*bw x s*bh input pixels and delivers every s-th one
+    cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(stride * cg.bw),
+                         static_cast<cuuint32_t>(stride * cg.bh), static_cast<cuuint32_t>(cg.bn)};
+    cuuint32_t es[4] = {1, static_cast<cuuint32_t>(stride), static_cast<cuuint32_t>(stride), 1};
     r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_64B);
+               CU_TENSOR_MAP_SWIZZLE_64B, es);
     if (r) return r;
   }
   aq::GemmParams p{};
@@ -599,6 +792,7 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   p.conv = 1;
   p.cin_blocks = Cin / aq::kBK;
   p.pad = pad;
+  p.stride = stride;
   p.tiles_per_img = cg.tiles_per_img;
   p.rows_per_tile = cg.rows_per_tile;
   p.imgs_per_tile = cg.imgs_per_tile;
@@ -607,7 +801,7 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, partial, st);
+  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st);
 }
 
 }  // extern "C"
@@ -679,5 +873,5 @@ extern "C" int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  return run_dense(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, nullptr, st);
+  return run_gemm(mapA, p, pl, codes_packed, codebooks, M, B, Wdec, nullptr, st);
 }

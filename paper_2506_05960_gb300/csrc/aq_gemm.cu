@@ -36,7 +36,8 @@ namespace aq {
 
 __device__ unsigned g_gemm_err = 0;
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 448;                   // 14 warps (warps 10..13 decode on the fused path)
+constexpr int kDecodeThreads = 128;
 constexpr int kA8Half = kBM * 64;               // one 64-wide int8 box: 128 rows x 64 B
 constexpr int kA8Stage = kStageBlocks * kA8Half;
 constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A slot
@@ -57,13 +58,14 @@ struct alignas(8) GemmBarriers {
   int abort_flag;
 };
 
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out) {
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes) {
   return 1024 + static_cast<size_t>(stages) * (kStageBlocks * BN * 128 + kA8Stage) +
-         4 * 2 * (f32_out ? kEpiBuf32 : kEpiBuf16) + kScaleBytes + sizeof(GemmBarriers);
+         4 * 2 * (f32_out ? kEpiBuf32 : kEpiBuf16) + kScaleBytes + book_bytes +
+         sizeof(GemmBarriers);
 }
 
-int gemm_max_stages(int BN, bool f32_out) {
-  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out);
+int gemm_max_stages(int BN, bool f32_out, int book_bytes) {
+  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes);
   const size_t per = static_cast<size_t>(kStageBlocks) * BN * 128 + kA8Stage;
   const int s = static_cast<int>((232448 - fixed) / per);
   return s < kMaxStages ? s : kMaxStages;
@@ -128,16 +130,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* aring = bring + S * b_stage;
   uint8_t* epi = aring + S * kA8Stage;
   float* sscale = reinterpret_cast<float*>(epi + 4 * 2 * epi_buf);
+  uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) + kScaleBytes);
   GemmBarriers* bar =
-      reinterpret_cast<GemmBarriers*>(reinterpret_cast<uint8_t*>(sscale) + kScaleBytes);
+      reinterpret_cast<GemmBarriers*>(reinterpret_cast<uint8_t*>(sbook) + p.book_bytes);
   const volatile int* abort_flag = &bar->abort_flag;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
+  if (p.fused && p.book_bytes > 0) {
+    // 8-bit codebooks of the fused path live in shared memory for the whole kernel
+    for (int i = threadIdx.x; i < p.book_bytes / 16; i += blockDim.x)
+      sbook[i] = reinterpret_cast<const uint4*>(p.books)[i];
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&bar->full[s], 1);
+      // fused path: the producer's expect_tx arrival + one arrival per decoder warp
+      mbar_init(&bar->full[s], p.fused ? 1 + kDecodeThreads / 32 : 1);
       mbar_init(&bar->empty[s], 5);
     }
     for (int s = 0; s < SA; ++s) {
@@ -152,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bar->abort_flag = 0;
     mbar_fence_init();
     tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapB);
+    if (!p.fused) tma_prefetch_desc(&mapB);
     tma_prefetch_desc(&mapY);
   }
   if (warp == 1) {
@@ -193,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           uint64_t* fb = &bar->full[rg.s];
-          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (kA8Half + b_half)));
+          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (kA8Half + (p.fused ? 0 : b_half))));
           uint8_t* a_dst = aring + rg.s * kA8Stage;
           uint8_t* b_dst = bring + rg.s * b_stage;
           for (int h = 0; h < nb; ++h) {
@@ -202,13 +211,13 @@ __global__ void __launch_bounds__(kThreads, 1)
               tma_load_2d(a_dst + h * kA8Half, &mapA, fb, k * kBK, m0);
             } else {
               const int kh = tap / 3, kw = tap - 3 * (tap / 3);
-              tma_load_4d(a_dst + h * kA8Half, &mapA, fb, cb * kBK, kw - p.pad, ho0 + kh - p.pad, b0);
+              tma_load_4d(a_dst + h * kA8Half, &mapA, fb, cb * kBK, kw - p.pad, ho0 * p.stride + kh - p.pad, b0);
               if (++cb == p.cin_blocks) {
                 cb = 0;
                 ++tap;
               }
             }
-            tma_load_2d(b_dst + h * b_half, &mapB, fb, k * kBK, n0);
+            if (!p.fused) tma_load_2d(b_dst + h * b_half, &mapB, fb, k * kBK, n0);
           }
           ++issued;
           rg.next(S);
@@ -336,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ra.next(SA);
       }
     }
-  } else {
+  } else if (warp < 10) {
     // ================================================================ epilogue
     const int q = warp & 3;
     const int ew = warp - 6;
@@ -426,6 +435,72 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (lane == 0) bulk_wait_group_all();
+  } else if (p.fused) {
+    // ================================================================ decoders (fused path)
+    // Each decoded group (8 consecutive k of one output row) is written as one
+    // 16-byte chunk of the 128B-swizzled K-major B stage, so W-hat never leaves
+    // shared memory.  Same arithmetic as the decode kernel: fp32 sum of the M
+    // codewords in ascending m, one round to fp16.
+    const int dt = threadIdx.x - 320;
+    const int eb = p.B >> 3;                         // bytes per code
+    const int G = p.K >> 3;
+    Ring rg;
+    bool failed = false;
+    for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
+      const TileCoord tc = tile_coord(p, t);
+      const int n0 = tc.n_tile * BN;
+      for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
+        const int nb = min(kStageBlocks, tc.kb_end - kb);
+        if (!rg.lap0 && !mbar_wait(&bar->empty[rg.s], rg.ph ^ 1u, abort_flag)) {
+          if (!*abort_flag) record_failure(bar, kDevErrTimeoutEmpty);
+          failed = true;
+          break;
+        }
+        uint8_t* b_dst = bring + rg.s * b_stage;
+        const int groups = nb * BN * 8;
+        for (int gi = dt; gi < groups; gi += kDecodeThreads) {
+          const int h = gi / (BN * 8);
+          const int r = gi - h * (BN * 8);
+          const int n = r >> 3;
+          const int j = r & 7;
+          const int grow = n0 + n;
+          const int gk = (kb + h) * 8 + j;             // group index along K
+          uint4 out = make_uint4(0u, 0u, 0u, 0u);
+          if (grow < p.N && gk < G) {
+            const uint8_t* c = static_cast<const uint8_t*>(p.codes) +
+                               ((static_cast<int64_t>(kb + h) * p.N + grow) * 8 + j) * p.M * eb;
+            float acc[8];
+            for (int m = 0; m < p.M; ++m) {
+              uint4 cw;
+              if (eb == 1) {
+                cw = sbook[m * 256 + c[m]];
+              } else {
+                const int code = c[2 * m] | (c[2 * m + 1] << 8);
+                cw = __ldg(reinterpret_cast<const uint4*>(p.books) + (static_cast<int64_t>(m) << 16) + code);
+              }
+              const __half2* h2 = reinterpret_cast<const __half2*>(&cw);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const float2 f = __half22float2(h2[i]);
+                acc[2 * i] = m == 0 ? f.x : __fadd_rn(acc[2 * i], f.x);
+                acc[2 * i + 1] = m == 0 ? f.y : __fadd_rn(acc[2 * i + 1], f.y);
+              }
+            }
+            uint32_t* o = reinterpret_cast<uint32_t*>(&out);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              __half2 hh = __floats2half2_rn(acc[2 * i], acc[2 * i + 1]);
+              o[i] = *reinterpret_cast<uint32_t*>(&hh);
+            }
+          }
+          *reinterpret_cast<uint4*>(b_dst + h * b_half + n * 128 + ((j ^ (n & 7)) << 4)) = out;
+        }
+        fence_proxy_async_smem();     // generic writes -> visible to the tensor core
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar->full[rg.s]);
+        rg.next(S);
+      }
+    }
   }
 
   tc_fence_before();
@@ -474,7 +549,8 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st) {
   static int configured_bytes = 0;
-  const size_t bytes = gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr);
+  const size_t bytes =
+      gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes);
   if (static_cast<int>(bytes) > configured_bytes) {
     cudaError_t e = cudaFuncSetAttribute(aq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(bytes));

@@ -27,7 +27,7 @@ struct GemmParams {
   int a_stages;                 // TMEM A ring depth (slots of 128 K = 64 columns)
   int acc_stride, a_col;        // TMEM columns: accumulator buffer stride, first A slot
   // implicit-GEMM convolution (conv != 0): A is loaded per tap with a 4-D TMA box
-  int conv, cin_blocks, pad, tiles_per_img, rows_per_tile, imgs_per_tile;
+  int conv, cin_blocks, pad, stride, tiles_per_img, rows_per_tile, imgs_per_tile;
   // epilogue
   float s_x;
   const __half* scale;
@@ -35,6 +35,25 @@ struct GemmParams {
   void* y;
   int out_f32;
   float* partial;               // split-K partial sums [splits][T][N] (null: fused epilogue)
+  // fused decode (B stages written by decoder warps instead of TMA from a decoded W)
+  int fused;
+  const void* codes;            // packed codes
+  const void* books;            // codebooks [M][2^B][8] fp16
+  int M, B;
+  int book_bytes;               // codebooks staged in shared memory (8-bit codes), else 0
+};
+
+// Parameters of the lookup-table kernel (linear layer, 8-bit codes, T <= 16).
+struct LutParams {
+  const int8_t* xq;             // [T][K]
+  const uint8_t* packed;        // packed codes [K/64][N][8][M]
+  const __half* books;          // [M][256][8]
+  float* partial;               // [chunks][T][N] partial sums
+  int T, K, N, M;
+  int Tp;                       // T rounded up to 4, 8 or 16 (floats per table entry)
+  int J;                        // groups per chunk (divides 8)
+  int G;                        // K / 8
+  int chunks, rows_per_cta;
 };
 
 // Launchers (return the launch status; they never synchronise).
@@ -43,12 +62,13 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out);
-int gemm_max_stages(int BN, bool f32_out);   // smem ring depth that fits shared memory
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes);
+int gemm_max_stages(int BN, bool f32_out, int book_bytes);  // smem ring depth that fits
 int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-column accumulators
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st);
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st);
+cudaError_t launch_lut(const LutParams& p, cudaStream_t st);
 
 // Device error words of each translation unit (read and cleared, synchronising).
 cudaError_t read_clear_gemm_error(unsigned* out);

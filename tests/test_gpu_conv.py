@@ -32,6 +32,20 @@ def test_conv_shapes(Nb, H, W, Cin, Cout, M):
     assert_close(y, O.layer_f64(inp), spec)
 
 
+@pytest.mark.parametrize("Nb,H,W,Cin,Cout,M", [
+    (2, 64, 64, 192, 192, 2),   # UNet downsample 64 -> 32 (4 output rows per tile)
+    (2, 16, 16, 64, 64, 4),     # 16 -> 8: two 8x8 output images per tile
+    (3, 32, 32, 128, 96, 2),    # 32 -> 16, N tile tail
+    (3, 16, 16, 576, 576, 2),   # UNet downsample 16 -> 8 at 576 channels, ragged images
+])
+def test_conv_stride2(Nb, H, W, Cin, Cout, M):
+    spec = ConvSpec(Nb=Nb, H=H, W=W, Cin=Cin, Cout=Cout, stride=2, M=M, cb_std=0.05 / M ** 0.5)
+    inp = make_conv(spec, seed=7 * Nb + H + Cin)
+    assert (spec.Ho, spec.Wo) == (H // 2, W // 2)
+    y = run_conv(inp)
+    assert_close(y, O.layer_f64(inp), spec)
+
+
 def test_conv_fp32_no_bias():
     spec = ConvSpec(Nb=2, H=16, W=16, Cin=64, Cout=48, M=2)
     inp = make_conv(spec, seed=77)

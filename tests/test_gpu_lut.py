@@ -1,0 +1,68 @@
+"""GPU parity of the lookup-table path (App. A.1, Eq. A5-A6) of aq_linear
+against the fp64 oracle, and its path-selection rules."""
+
+import numpy as np
+import pytest
+
+from aq_synth import LinearSpec, make_linear
+from oracle import aq_oracle as O
+
+from gpu_util import assert_close, run_linear
+
+pytestmark = pytest.mark.gpu
+
+LUT = 3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import paper_2506_05960_gb300 as aq
+    aq.load_library()
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4, 5, 8, 9, 16])
+def test_lut_qkv_shape_small_batches(T):
+    inp = make_linear(LinearSpec(T=T, K=960, N=2880, M=2, B=8), seed=100 + T)
+    y = run_linear(inp, path=LUT)
+    assert_close(y, O.layer_f64(inp), T)
+
+
+@pytest.mark.parametrize("M", [1, 3, 4, 8])
+@pytest.mark.parametrize("out_f32", [False, True])
+def test_lut_codebook_counts(M, out_f32):
+    inp = make_linear(LinearSpec(T=6, K=576, N=1728, M=M, B=8, cb_std=0.05 / M ** 0.5),
+                      seed=200 + M)
+    y = run_linear(inp, path=LUT, out_f32=out_f32)
+    assert_close(y, O.layer_f64(inp), M)
+
+
+def test_lut_ragged_k_and_no_bias():
+    inp = make_linear(LinearSpec(T=7, K=208, N=40, M=2, B=8), seed=5)   # 26 groups
+    y = run_linear(inp, path=LUT, with_bias=False)
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    assert_close(y, O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], None))
+
+
+def test_lut_matches_oracle_lut_order():
+    """The kernel sums in the table order of Eq. A6; the oracle's table-order sum and its
+    decode-order sum agree, and the GPU result is within tolerance of both."""
+    inp = make_linear(LinearSpec(T=4, K=256, N=64, M=2, B=8), seed=9)
+    y = run_linear(inp, path=LUT)
+    y_lut = O.lut_linear_f64(inp["xq"], inp["s_x"], inp["codes"], inp["codebooks"],
+                             inp["scale"], inp["bias"])
+    assert_close(y, y_lut)
+
+
+def test_lut_path_selection():
+    import paper_2506_05960_gb300 as aq
+    # AUTO uses the table path for a handful of tokens, the tensor-core path beyond
+    assert aq.aq_linear_workspace_size(8, 960, 2880, 8, 2, 8, 0) == \
+        aq.aq_linear_workspace_size(8, 960, 2880, 8, 2, 8, LUT)
+    assert aq.aq_linear_workspace_size(256, 960, 2880, 8, 2, 8, 0) == \
+        aq.aq_linear_workspace_size(256, 960, 2880, 8, 2, 8, 1)
+    with pytest.raises(aq.AQError) as e:
+        aq.aq_linear_workspace_size(4, 960, 960, 8, 1, 16, LUT)      # 2^16 codebook
+    assert e.value.status == -3
+    with pytest.raises(aq.AQError) as e:
+        aq.aq_linear_workspace_size(17, 960, 960, 8, 2, 8, LUT)      # too many tokens
+    assert e.value.status == -3
