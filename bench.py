@@ -1,10 +1,10 @@
 #!/usr/bin/env python
 """Throughput of the AQ x A8 layer on GB300 (one JSON line on stdout).
 
-Workload (default): the fused qkv projection of an LDM-4-like UNet at its 8x8
+Headline workload: the fused qkv projection of an LDM-4-like UNet at its 8x8
 level for 32 images x CFG pair: T = 4096 tokens, K = 960, N = 2880, 2x8
 codebooks (W2A8), seeded synthetic weights and activations.  One step is the
-whole hot path of that layer: 8-bit activation quantization of the fp16
+whole hot path of that layer through the C ABI: 8-bit quantization of the fp16
 input, decode of the AQ weight, tensor-core contraction, fused scale/bias
 epilogue to fp16.
 
@@ -12,12 +12,15 @@ Timing: CUDA-graph replay of 8 steps that rotate over 8 independent buffer
 sets (inputs, codes, outputs: > 300 MB together, larger than the 129 MB L2),
 CUDA events on the launching stream, warm-up first, barrier + synchronize on
 both sides, max over ranks.  The dominant kernel (the tensor-core GEMM) is
-timed by the library's own event pairs, captured as event-record nodes into a
-second graph that is replayed once inside the same timed region.  `e2e` repeats the step through the public C ABI with the
-input copied from pinned host memory and the output copied back every step.
+timed live as the difference between that graph and the same graph without
+the GEMM (quantizer + decode only), replayed in the same timed region.
+`e2e` repeats the step through the C ABI with the input copied from pinned host
+memory and the output copied back every step.  `layers` times the other
+workloads (64x64 W4A8 conv, 8x8 conv with one 2^16-entry codebook) and
+`unet_forward` one UNet-shaped forward (97 AQ layers, batch 2, W2A8 and W4A8).
 
---impl reference times the CPU oracle (plain numpy fp64) on the same workload.
-Multi-GPU: independent replicas, one per rank (the layer needs no exchange).
+--impl reference times the CPU oracle (numpy float64) on the headline workload.
+Multi-GPU: independent replicas, one per rank (the layer has no exchange step).
 """
 
 from __future__ import annotations
@@ -38,17 +41,13 @@ if ROOT not in sys.path:
 
 import numpy as np  # noqa: E402
 
-WORKLOADS = {
-    "qkv": dict(cfg=1, name="AQ linear qkv projection T=4096 K=960 N=2880 W2A8 (2x8 codebooks, g=8)"),
-}
+HEADLINE = "AQ linear qkv projection T=4096 K=960 N=2880 W2A8 (2x8 codebooks, g=8)"
 NSETS = 8
 
-# DRAM traffic of one launch of the tensor-core GEMM kernel on this workload,
-# from `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (see the
-# summary under profiles/), valid only for the kernel sources it was taken on.
-TRAFFIC = {
-    "qkv": {"bytes": None, "sources_sha": None},
-}
+# DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from
+# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (summary under profiles/);
+# reported only while the kernel sources are the ones it was measured on.
+TRAFFIC = {"bytes": None, "sources_sha": None}
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh"]
 
 
@@ -134,32 +133,24 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------- workload
-def make_sets(cfg: int, nsets: int):
+def headline_sets(nsets: int):
     from aq_synth import CONFIGS, make_linear
-    spec = CONFIGS[cfg]
-    sets = []
-    for i in range(nsets):
-        inp = make_linear(spec, seed=cfg * 1000 + i)
-        # fp16 activations whose 8-bit quantization with s_x gives the seeded int8 values
-        inp["x16"] = (inp["xq"].astype(np.float32) * np.float32(spec.s_x)).astype(np.float16)
-        sets.append(inp)
-    return spec, sets
+    spec = CONFIGS[1]
+    return spec, [make_linear(spec, seed=1000 + i) for i in range(nsets)]
 
 
-def flops_per_step(spec) -> float:
-    return 2.0 * spec.T * spec.N * spec.K
+def linear_flops(T, N, K) -> float:
+    return 2.0 * T * N * K
 
 
-def alg_bytes(spec) -> int:
-    """Algorithmic bytes of the layer: codes, codebooks, int8 activations once, output,
-    scale + bias (decoded weights and other scratch excluded)."""
-    codes = spec.N * spec.K * spec.M * spec.B // (8 * spec.g)
-    books = spec.M * (1 << spec.B) * spec.g * 2
-    return codes + books + spec.T * spec.K + spec.T * spec.N * 2 + 4 * spec.N
+def alg_bytes(T, K, N, M, B, g=8, out_bytes=2) -> int:
+    """Algorithmic bytes of one layer: codes, codebooks, int8 activations once, output,
+    scale + bias (decoded weights and scratch excluded)."""
+    return N * K * M * B // (8 * g) + M * (1 << B) * g * 2 + T * K + T * N * out_bytes + 4 * N
 
 
 # ----------------------------------------------------------------------------- oracle (CPU)
-def time_oracle(spec, inp, min_seconds: float = 10.0, max_steps: int = 50) -> dict:
+def time_oracle(inp, flops, min_seconds: float = 10.0, max_steps: int = 50) -> dict:
     """The oracle as it stands (float64 decode + numpy matmul) on the full layer, repeated
     until about `min_seconds` of CPU time."""
     from oracle import aq_oracle as O
@@ -172,14 +163,12 @@ def time_oracle(spec, inp, min_seconds: float = 10.0, max_steps: int = 50) -> di
         if el >= min_seconds or steps >= max_steps:
             break
     cores = len(os.sched_getaffinity(0))
-    return {"value": flops_per_step(spec) * steps / el / 1e12, "unit": "TFLOP/s",
-            "cores": cores, "kind": "oracle",
+    spec = inp["spec"]
+    return {"value": flops * steps / el / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
             "sample": f"full layer (T={spec.T}, K={spec.K}, N={spec.N}) x {steps} step(s), "
-                      f"{el:.1f} s, numpy float64 BLAS on {cores} host cores",
-            "seconds": el, "steps": steps}
+                      f"{el:.1f} s, numpy float64 BLAS on {cores} host cores"}
 
 
-# ----------------------------------------------------------------------------- main
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -187,11 +176,11 @@ def dist_setup():
     return world, rank, local
 
 
-def run_reference(args, workload):
+def run_reference(args):
     world, rank, _ = dist_setup()
     if rank != 0:
         return 0
-    spec, sets = make_sets(WORKLOADS[workload]["cfg"], 1)
+    spec, sets = headline_sets(1)
     inp = sets[0]
     from oracle import aq_oracle as O
     for _ in range(args.warmup):
@@ -202,14 +191,14 @@ def run_reference(args, workload):
         O.layer_f64(inp)
         times.append(time.perf_counter() - t0)
     el = sum(times)
-    val = flops_per_step(spec) * args.steps / el / 1e12
+    val = linear_flops(spec.T, spec.N, spec.K) * args.steps / el / 1e12
     cores = len(os.sched_getaffinity(0))
     line = {"impl": "reference", "metric": "AQ layer dense-equivalent TFLOP/s", "value": val,
             "unit": "TFLOP/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOADS[workload]["name"], "T": spec.T, "K": spec.K,
-                       "N": spec.N, "M": spec.M, "B": spec.B, "g": spec.g},
+            "config": {"workload": HEADLINE, "T": spec.T, "K": spec.K, "N": spec.N, "M": spec.M,
+                       "B": spec.B, "g": spec.g},
             "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                              "sample": f"full layer per step, {args.steps} steps"},
             "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -218,30 +207,151 @@ def run_reference(args, workload):
     return 0
 
 
+# ----------------------------------------------------------------------------- GPU helpers
+class Dev:
+    """Device copies of one seeded layer plus its output and workspace; step() is one pass
+    of the hot path through the C ABI (quantizer, then the layer on the AUTO path)."""
+
+    def __init__(self, aq, torch, inp, dev, path=0):
+        self.aq, self.torch = aq, torch
+        s = inp["spec"]
+        self.spec = s
+        self.conv = inp["xq"].ndim == 4
+        N, G, M = inp["codes"].shape
+        K = G * 8
+        B = 8 if inp["codes"].dtype == np.uint8 else 16
+        self.N, self.K, self.M, self.B, self.path = N, K, M, B, path
+
+        def t(a):
+            return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+        codes = t(inp["codes"])
+        self.packed = torch.empty(aq.aq_packed_size(N, K, 8, M, B), dtype=torch.uint8, device=dev)
+        aq.aq_pack(codes, self.packed, N, K, 8, M, B)
+        self.books, self.scale, self.bias = t(inp["codebooks"]), t(inp["scale"]), t(inp["bias"])
+        # fp16 activations whose 8-bit quantization with s_x gives the seeded int8 values
+        x16 = (inp["xq"].astype(np.float32) * np.float32(inp["s_x"])).astype(np.float16)
+        self.x16 = t(x16)
+        self.xq = torch.empty(inp["xq"].shape, dtype=torch.int8, device=dev)
+        self.s_x = inp["s_x"]
+        if self.conv:
+            self.T = s.Nb * s.Ho * s.Wo
+            self.ws_bytes = aq.aq_conv2d_workspace_size(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
+                                                        s.stride, 1, 8, M, B, path)
+            self.y = torch.empty((s.Nb, s.Ho, s.Wo, N), dtype=torch.float16, device=dev)
+        else:
+            self.T = inp["xq"].shape[0]
+            self.ws_bytes = aq.aq_linear_workspace_size(self.T, K, N, 8, M, B, path)
+            self.y = torch.empty((self.T, N), dtype=torch.float16, device=dev)
+        self.ws = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=dev)
+        self.flops = linear_flops(self.T, N, K)
+
+    def quant(self, st):
+        self.aq.aq_quant_act(self.x16, self.xq, self.xq.numel(), self.s_x, stream=st)
+
+    def layer(self, st):
+        aq, s = self.aq, self.spec
+        if self.conv:
+            aq.aq_conv2d_nhwc(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias,
+                              self.y, aq.AQ_DTYPE_F16, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
+                              s.stride, 1, 8, self.M, self.B, self.ws, self.ws_bytes, self.path,
+                              stream=st)
+        else:
+            aq.aq_linear(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias, self.y,
+                         aq.AQ_DTYPE_F16, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
+                         self.ws_bytes, self.path, stream=st)
+
+    def decode_only(self, st, wbuf):
+        self.aq.aq_decode(self.packed, self.books, wbuf, self.N, self.K, 8, self.M, self.B,
+                          stream=st)
+
+    def step(self, st):
+        self.quant(st)
+        self.layer(st)
+
+
+def capture(torch, stream, fn):
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    return g
+
+
+def replay_ms(torch, stream, g, reps):
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        g.replay()
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20):
+    """One UNet-shaped forward: every AQ layer of the LDM-4-like sweep, each preceded by
+    its activation quantization, captured as one graph.  Returns (ms, GFLOP, layers)."""
+    from aq_synth import ConvSpec, LinearSpec, make_conv, make_linear, unet_sweep_layers
+    layers = []
+    seed = 4000 + 100 * M
+    for kind, res, cin, cout, stride, count in unet_sweep_layers():
+        for _ in range(count):
+            seed += 1
+            if kind == "conv3":
+                spec = ConvSpec(Nb=batch, H=res * stride, W=res * stride, Cin=cin, Cout=cout,
+                                stride=stride, M=M, B=8, cb_std=0.03)
+                layers.append(Dev(aq, torch, make_conv(spec, seed), dev))
+            else:
+                spec = LinearSpec(T=batch * res * res, K=cin, N=cout, M=M, B=8, cb_std=0.03,
+                                  act="normal40")
+                layers.append(Dev(aq, torch, make_linear(spec, seed), dev))
+    torch.cuda.synchronize()
+
+    def fwd():
+        for L in layers:
+            L.step(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            fwd()
+    stream.synchronize()
+    g = capture(torch, stream, fwd)
+    ms = replay_ms(torch, stream, g, reps)
+    gflop = sum(L.flops for L in layers) / 1e9
+    del g
+    return ms, gflop, len(layers)
+
+
+# ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=4000)
     ap.add_argument("--warmup", type=int, default=16)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="qkv", choices=sorted(WORKLOADS))
     ap.add_argument("--e2e-steps", type=int, default=100)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the other workloads and the UNet-shaped forward")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
 
     if args.impl == "reference":
-        return run_reference(args, args.workload)
+        return run_reference(args)
 
     world, rank, local = dist_setup()
-    spec, sets = make_sets(WORKLOADS[args.workload]["cfg"], NSETS)
+    spec, sets = headline_sets(NSETS)
+    T, K, N, g, M, B = spec.T, spec.K, spec.N, spec.g, spec.M, spec.B
+    fl = linear_flops(T, N, K)
 
     # CPU baseline first (before any GPU work), rank 0 at N=1 only
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = time_oracle(spec, sets[0], min_seconds=args.cpu_seconds)
+        cpu = time_oracle(sets[0], fl, min_seconds=args.cpu_seconds)
 
     import torch
     import paper_2506_05960_gb300 as aq
@@ -255,117 +365,90 @@ def main():
         pg = dist
     aq.load_library()
 
-    T, K, N, g, M, B = spec.T, spec.K, spec.N, spec.g, spec.M, spec.B
-    ws_bytes = aq.aq_linear_workspace_size(T, K, N, g, M, B)
-    bufs = []
-    for inp in sets:
-        b = {}
-        b["x16"] = torch.from_numpy(inp["x16"]).to(dev)
-        codes = torch.from_numpy(inp["codes"]).to(dev)
-        b["packed"] = torch.empty(aq.aq_packed_size(N, K, g, M, B), dtype=torch.uint8, device=dev)
-        aq.aq_pack(codes, b["packed"], N, K, g, M, B)
-        b["books"] = torch.from_numpy(inp["codebooks"]).to(dev)
-        b["scale"] = torch.from_numpy(inp["scale"]).to(dev)
-        b["bias"] = torch.from_numpy(inp["bias"]).to(dev)
-        b["xq"] = torch.empty((T, K), dtype=torch.int8, device=dev)
-        b["y"] = torch.empty((T, N), dtype=torch.float16, device=dev)
-        b["ws"] = torch.empty(max(ws_bytes, 16), dtype=torch.uint8, device=dev)
-        bufs.append(b)
+    bufs = [Dev(aq, torch, inp, dev) for inp in sets]
+    wdec = torch.empty((N, K), dtype=torch.float16, device=dev)
     torch.cuda.synchronize()
-    s_x = spec.s_x
     stream = torch.cuda.Stream(device=dev)
 
-    def step(b, st):
-        aq.aq_quant_act(b["x16"], b["xq"], T * K, s_x, stream=st)
-        aq.aq_linear(b["xq"], s_x, b["packed"], b["books"], b["scale"], b["bias"], b["y"],
-                     aq.AQ_DTYPE_F16, T, K, N, g, M, B, b["ws"], ws_bytes, stream=st)
-
-    # warm-up (eager); one pass with kernel timing on fills the library's event pool so
-    # that capture below needs no event creation
     with torch.cuda.stream(stream):
         for i in range(args.warmup):
-            step(bufs[i % NSETS], stream)
-        aq.aq_profile_enable(True)
-        for i in range(2 * NSETS):
-            step(bufs[i % NSETS], stream)
+            bufs[i % NSETS].step(stream)
     stream.synchronize()
-    aq.aq_profile_read()
-    aq.aq_profile_enable(False)
     assert aq.aq_device_error() == 0
 
-    # capture the main graph (NSETS steps, one per buffer set) and a copy whose library
-    # calls carry event-record nodes around every kernel (for per-kernel device time)
-    g_main = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_main, stream=stream):
-        for i in range(NSETS):
-            step(bufs[i], stream)
-    aq.aq_profile_enable(True)
-    g_prof = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_prof, stream=stream):
-        for i in range(NSETS):
-            step(bufs[i], stream)
-    for _ in range(2):
-        g_main.replay()
+    # graphs: the step over the 8 buffer sets, and the same without the GEMM
+    # (quantizer + the decode kernel the step runs), for the GEMM's live time
+    def main_graph():
+        for b in bufs:
+            b.step(stream)
+
+    def nogemm_graph():
+        for b in bufs:
+            b.quant(stream)
+            b.decode_only(stream, wdec)
+
+    g_main = capture(torch, stream, main_graph)
+    g_nogemm = capture(torch, stream, nogemm_graph)
+    for gg in (g_main, g_nogemm):
+        gg.replay()
     stream.synchronize()
 
     reps = max(1, args.steps // NSETS)
+    reps_nogemm = max(1, reps // 4)
     steps = reps * NSETS
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
     sampler = ClockSampler(local)
     sampler.start()
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
-        ev0.record(stream)
+        ev[0].record(stream)
         for _ in range(reps):
             g_main.replay()
-        ev1.record(stream)
-        g_prof.replay()          # per-kernel event pairs (read below)
+        ev[1].record(stream)
+        for _ in range(reps_nogemm):
+            g_nogemm.replay()
+        ev[2].record(stream)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
     clocks = sampler.stop()
-    ms_total = ev0.elapsed_time(ev1)
-    prof = aq.aq_profile_read()
-    aq.aq_profile_enable(False)
+    ms_total = ev[0].elapsed_time(ev[1])
+    ms_nogemm_step = ev[1].elapsed_time(ev[2]) / (reps_nogemm * NSETS)
     assert aq.aq_device_error() == 0
     if pg:
         t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
         ms_total = float(t.item())
     ms_step = ms_total / steps
-    fl = flops_per_step(spec)
     value = world * fl / (ms_step * 1e-3) / 1e12
+    gemm_ms = ms_step - ms_nogemm_step
 
-    gemm_ms, gemm_n = prof["gemm"]
-    gemm_avg_ms = gemm_ms / gemm_n if gemm_n else float("nan")
     peaks = measured_peaks()
-    achieved = fl / (gemm_avg_ms * 1e-3) / 1e12
-    tr = TRAFFIC.get(args.workload, {})
-    traffic = tr.get("bytes") if tr.get("sources_sha") == sources_sha() else None
-    launches_per_step = sum(n for k, (ms, n) in prof.items()) / NSETS
+    achieved = fl / (gemm_ms * 1e-3) / 1e12
+    traffic = TRAFFIC["bytes"] if TRAFFIC.get("sources_sha") == sources_sha() else None
+    launches_per_step = 3    # quantizer, decode, GEMM (the headline plan does not split K)
 
     # e2e through the public API: pinned host input -> device, step, device -> pinned host
-    h_x = [torch.from_numpy(inp["x16"]).pin_memory() for inp in sets[:2]]
+    h_x = [b.x16.cpu().pin_memory() for b in bufs[:2]]
     h_y = torch.empty((T, N), dtype=torch.float16).pin_memory()
     e2e_steps = max(1, args.e2e_steps)
     with torch.cuda.stream(stream):
         for i in range(3):
             b = bufs[i % 2]
-            b["x16"].copy_(h_x[i % 2], non_blocking=True)
-            step(b, stream)
-            h_y.copy_(b["y"], non_blocking=True)
+            b.x16.copy_(h_x[i % 2], non_blocking=True)
+            b.step(stream)
+            h_y.copy_(b.y, non_blocking=True)
         stream.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for i in range(e2e_steps):
             b = bufs[i % 2]
-            b["x16"].copy_(h_x[i % 2], non_blocking=True)
-            step(b, stream)
-            h_y.copy_(b["y"], non_blocking=True)
+            b.x16.copy_(h_x[i % 2], non_blocking=True)
+            b.step(stream)
+            h_y.copy_(b.y, non_blocking=True)
         e1.record(stream)
     stream.synchronize()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
@@ -374,34 +457,66 @@ def main():
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
         e2e_ms = float(t.item())
 
+    # the other workloads (per layer, graph replay) and the UNet-shaped forward
+    layers, unet = {}, None
+    if not args.no_extras and rank == 0:
+        from aq_synth import CONFIGS, make_conv
+        for name, cfg in (("conv3x3 16x64x64x192->192 W4A8 (4x8)", 2),
+                          ("conv3x3 2x8x8x960->960 one 2^16 codebook (1x16)", 3)):
+            L = Dev(aq, torch, make_conv(CONFIGS[cfg], seed=cfg), dev)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    L.step(stream)
+            stream.synchronize()
+            gl = capture(torch, stream, lambda: [L.step(stream) for _ in range(8)])
+            ms = replay_ms(torch, stream, gl, 20) / 8
+            layers[name] = {"us_per_step": ms * 1e3,
+                            "tflops": L.flops / (ms * 1e-3) / 1e12,
+                            "tensor_roofline_frac": L.flops / (peaks["bf16_tflops"] * 1e12) / (ms * 1e-3),
+                            "step": "quantizer + layer (AUTO path), CUDA graph replay"}
+            del gl, L
+        unet = {}
+        for Mu, label in ((2, "W2A8"), (4, "W4A8")):
+            ms, gflop, nl = unet_forward(aq, torch, dev, stream, Mu)
+            unet[label] = {"ms_per_forward": ms, "gflop": gflop, "tflops": gflop / ms,
+                           "layers": nl, "batch": 2}
+        assert aq.aq_device_error() == 0
+
     if rank == 0:
         line = {
             "metric": "AQ layer dense-equivalent TFLOP/s (2*T*N*K / step time)",
             "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
-            "config": {"workload": WORKLOADS[args.workload]["name"], "T": T, "K": K, "N": N,
-                       "g": g, "M": M, "B": B, "parallelism": f"replicas{world}",
+            "config": {"workload": HEADLINE, "T": T, "K": K, "N": N, "g": g, "M": M, "B": B,
+                       "parallelism": f"replicas{world}",
                        "l2": f"inputs larger than L2: {NSETS} rotating buffer sets",
                        "timing": "CUDA graph replay of 8 steps, CUDA events"},
-            "hbm_gbs_algorithmic": alg_bytes(spec) / (ms_step * 1e-3) / 1e9,
+            "hbm_gbs_algorithmic": alg_bytes(T, K, N, M, B) / (ms_step * 1e-3) / 1e9,
             "roofline": {"bound": "tensor", "kernel": "aq_gemm_kernel", "achieved": achieved,
                          "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
-                         "peak_source": f"{peaks['source']} bf16 burst (fp16 dense rate is equal)",
+                         "peak_source": f"{peaks['source']} bf16 dense burst (the fp16 rate is equal)",
                          "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
                                                if peaks.get("bf16_tflops_sustained") else None),
-                         "kernel_ms": gemm_avg_ms},
-            "kernel_ms": {k: (ms / n if n else None) for k, (ms, n) in prof.items()},
+                         "kernel_us": gemm_ms * 1e3,
+                         "kernel_timing": "step graph minus the same graph without the GEMM"},
+            "step_us": {"total": ms_step * 1e3, "gemm": gemm_ms * 1e3,
+                        "quant_and_decode": ms_nogemm_step * 1e3},
             "step_roofline_frac": (max(fl / (peaks["bf16_tflops"] * 1e12),
-                                       alg_bytes(spec) / (peaks["hbm_gbs"] * 1e9)) / (ms_step * 1e-3)),
-            "cpu_baseline": cpu and {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")},
+                                       alg_bytes(T, K, N, M, B) / (peaks["hbm_gbs"] * 1e9))
+                                   / (ms_step * 1e-3)),
+            "cpu_baseline": cpu,
             "e2e": {"value": world * fl / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                     "ms_per_step": e2e_ms, "h2d_bytes_per_step": T * K * 2,
                     "d2h_bytes_per_step": T * N * 2},
-            "gpu_launches": int(round(launches_per_step * steps)) + sum(n for _, n in prof.values()),
+            "gpu_launches": launches_per_step * steps + 2 * NSETS * reps_nogemm,
             "clocks": clocks,
         }
+        if layers:
+            line["layers"] = layers
+        if unet:
+            line["unet_forward"] = unet
         print(json.dumps(line), flush=True)
     if pg:
         pg.destroy_process_group()
