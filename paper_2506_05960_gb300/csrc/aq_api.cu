@@ -159,7 +159,11 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
       const long waves = (tiles + kPlanSMs - 1) / kPlanSMs;
       const double tile_cycles = (kbps / 2) * st_cyc + (kbps & 1) * 0.5 * st_cyc + 800.0;
       double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
-      if (s_eff > 1) t += (s_eff * 8.0 + 2.0) * T * static_cast<double>(N) / 6.0e12 + 2.0e-6;
+      if (s_eff > 1) {
+        // partials written and read back (mostly from L2) + the reduce launch
+        const double part_bytes = s_eff * 8.0 * T * static_cast<double>(N);
+        t += part_bytes / (part_bytes < 64e6 ? 15.0e12 : 6.0e12) + 2.0 * T * N / 6.0e12 + 1.0e-6;
+      }
       if (t < best * 0.999) {
         best = t;
         bp = Plan{};

@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include "aq_internal.h"
+#include "aq_ptx.cuh"
 
 namespace aq {
 
@@ -32,6 +33,8 @@ __device__ __forceinline__ int8_t quant_one(__half h, float s, float rs) {
 __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
                                                         int8_t* __restrict__ xq,
                                                         int64_t nvec, int64_t numel, float s) {
+  grid_dependency_wait();
+  allow_dependents();
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec;
        v += stride) {
@@ -67,15 +70,16 @@ cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s,
   const int64_t cap = 152 * 16;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  quant_act_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(
-      static_cast<const __half*>(x), xq, nvec, numel, s);
-  return cudaGetLastError();
+  return launch_pdl(quant_act_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st,
+                    static_cast<const __half*>(x), xq, nvec, numel, s);
 }
 
 // ============================================================== packing
 // canonical [N][G][M] (elem bytes eb) -> packed [KB][N][8][M]; one thread per (kb, n).
 __global__ void pack_kernel(const uint8_t* __restrict__ canon, uint8_t* __restrict__ packed,
                             int N, int G, int M, int eb, int KB) {
+  grid_dependency_wait();
+  allow_dependents();
   const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (idx >= static_cast<int64_t>(KB) * N) return;
   const int kb = static_cast<int>(idx / N);
@@ -96,9 +100,9 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
   const int64_t total = static_cast<int64_t>(KB) * N;
   const int threads = 256;
   const int64_t blocks = (total + threads - 1) / threads;
-  pack_kernel<<<static_cast<unsigned>(blocks), threads, 0, st>>>(
-      static_cast<const uint8_t*>(canon), static_cast<uint8_t*>(packed), N, G, M, B / 8, KB);
-  return cudaGetLastError();
+  return launch_pdl(pack_kernel, dim3(static_cast<unsigned>(blocks)), dim3(threads), 0, st,
+                    static_cast<const uint8_t*>(canon), static_cast<uint8_t*>(packed), N, G, M,
+                    B / 8, KB);
 }
 
 // ============================================================== decode
@@ -143,6 +147,8 @@ __global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restric
                                                         __half* __restrict__ W, int N, int K,
                                                         int M, int KB) {
   extern __shared__ uint4 sbook[];                       // [M][256]
+  grid_dependency_wait();
+  allow_dependents();
   for (int i = threadIdx.x; i < M * 256; i += blockDim.x) sbook[i] = books[i];
   __syncthreads();
   const int G = K / 8;
@@ -167,6 +173,8 @@ __global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restr
                                                          const uint4* __restrict__ books,
                                                          __half* __restrict__ W, int N, int K,
                                                          int M, int KB) {
+  grid_dependency_wait();
+  allow_dependents();
   const int G = K / 8;
   const int64_t total = static_cast<int64_t>(KB) * N * 8;
   for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
@@ -193,16 +201,13 @@ cudaError_t launch_decode(const void* packed, const void* books, void* W, int N,
   int64_t blocks = (total + threads - 1) / threads;
   if (blocks > 152 * 4) blocks = 152 * 4;
   if (blocks < 1) blocks = 1;
-  if (B == 8) {
-    decode_b8_kernel<<<static_cast<unsigned>(blocks), threads, M * 256 * 16, st>>>(
-        static_cast<const uint8_t*>(packed), static_cast<const uint4*>(books),
-        static_cast<__half*>(W), N, K, M, KB);
-  } else {
-    decode_b16_kernel<<<static_cast<unsigned>(blocks), threads, 0, st>>>(
-        static_cast<const uint16_t*>(packed), static_cast<const uint4*>(books),
-        static_cast<__half*>(W), N, K, M, KB);
-  }
-  return cudaGetLastError();
+  if (B == 8)
+    return launch_pdl(decode_b8_kernel, dim3(static_cast<unsigned>(blocks)), dim3(threads),
+                      static_cast<size_t>(M) * 256 * 16, st, static_cast<const uint8_t*>(packed),
+                      static_cast<const uint4*>(books), static_cast<__half*>(W), N, K, M, KB);
+  return launch_pdl(decode_b16_kernel, dim3(static_cast<unsigned>(blocks)), dim3(threads), 0, st,
+                    static_cast<const uint16_t*>(packed), static_cast<const uint4*>(books),
+                    static_cast<__half*>(W), N, K, M, KB);
 }
 
 }  // namespace aq

@@ -111,6 +111,100 @@ struct Ring {
   }
 };
 
+// Fused path: decode the 8 groups of one output row in one 64-wide K block into the
+// row's 128-byte line of the swizzled B stage.  Codes: 8*M*EB contiguous bytes
+// (EB = bytes per code), read as 32-bit words and unpacked with constant shifts;
+// all codeword reads are issued before the fp32 sums (ascending m, one RNE to fp16).
+template <int M, int EB>
+__device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* sbook,
+                                            const uint4* gbooks, uint8_t* rowp, int n,
+                                            int gvalid) {
+  constexpr int kWords = 2 * M * EB;
+  uint32_t w[kWords];
+  if constexpr (kWords % 4 == 0) {
+#pragma unroll
+    for (int i = 0; i < kWords / 4; ++i) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4*>(codes) + i);
+      w[4 * i] = v.x;
+      w[4 * i + 1] = v.y;
+      w[4 * i + 2] = v.z;
+      w[4 * i + 3] = v.w;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < kWords / 2; ++i) {
+      const uint2 v = __ldg(reinterpret_cast<const uint2*>(codes) + i);
+      w[2 * i] = v.x;
+      w[2 * i + 1] = v.y;
+    }
+  }
+  // 16-bit codes gather from L2: issue all 8*M reads first.  8-bit codes read the
+  // codebooks from shared memory as they are summed.
+  constexpr int kPre = EB == 2 ? 8 * M : 1;
+  uint4 cw[kPre];
+  if (EB == 2) {
+#pragma unroll
+    for (int idx = 0; idx < 8 * M; ++idx) {
+      const uint32_t c = (w[idx >> 1] >> (16 * (idx & 1))) & 0xFFFFu;
+      const int m = idx % M;
+      cw[idx % kPre] = (idx / M) < gvalid ? __ldg(gbooks + (static_cast<int64_t>(m) << 16) + c)
+                                          : make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    uint4 out = make_uint4(0u, 0u, 0u, 0u);
+    if (j < gvalid) {
+      float acc[8];
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        const int idx = j * M + m;
+        uint4 word;
+        if (EB == 1)
+          word = sbook[m * 256 + ((w[idx >> 2] >> (8 * (idx & 3))) & 0xFFu)];
+        else
+          word = cw[idx % kPre];
+        const __half2* h2 = reinterpret_cast<const __half2*>(&word);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = __half22float2(h2[i]);
+          acc[2 * i] = m == 0 ? f.x : __fadd_rn(acc[2 * i], f.x);
+          acc[2 * i + 1] = m == 0 ? f.y : __fadd_rn(acc[2 * i + 1], f.y);
+        }
+      }
+      uint32_t* o = reinterpret_cast<uint32_t*>(&out);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        __half2 hh = __floats2half2_rn(acc[2 * i], acc[2 * i + 1]);
+        o[i] = *reinterpret_cast<uint32_t*>(&hh);
+      }
+    }
+    *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = out;
+  }
+}
+
+__device__ __forceinline__ void decode_unit_dispatch(int M, int EB, const uint8_t* codes,
+                                                     const uint4* sbook, const uint4* gbooks,
+                                                     uint8_t* rowp, int n, int gvalid) {
+  if (EB == 1) {
+    switch (M) {
+      case 1: decode_unit<1, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 2: decode_unit<2, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 3: decode_unit<3, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 4: decode_unit<4, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 5: decode_unit<5, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 6: decode_unit<6, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 7: decode_unit<7, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      default: decode_unit<8, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+    }
+  } else {
+    if (M == 1)
+      decode_unit<1, 2>(codes, sbook, gbooks, rowp, n, gvalid);
+    else
+      decode_unit<2, 2>(codes, sbook, gbooks, rowp, n, gvalid);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     aq_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                    const __grid_constant__ CUtensorMap mapB,
@@ -138,6 +232,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
+  // nothing in global memory is touched before the previous kernel in the stream is done
+  grid_dependency_wait();
+  allow_dependents();
   if (p.fused && p.book_bytes > 0) {
     // 8-bit codebooks of the fused path live in shared memory for the whole kernel
     for (int i = threadIdx.x; i < p.book_bytes / 16; i += blockDim.x)
@@ -457,43 +554,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         uint8_t* b_dst = bring + rg.s * b_stage;
-        const int groups = nb * BN * 8;
-        for (int gi = dt; gi < groups; gi += kDecodeThreads) {
-          const int h = gi / (BN * 8);
-          const int r = gi - h * (BN * 8);
-          const int n = r >> 3;
-          const int j = r & 7;
+        // unit = (64-wide K block h, output row n): its 8 groups' codes are contiguous
+        // (8*M*eb bytes, 16-byte aligned) and are read with vector loads; all of the
+        // unit's codeword reads are issued before any is used.
+        const int units = nb * BN;
+        const int code_bytes = 8 * p.M * eb;
+        for (int u = dt; u < units; u += kDecodeThreads) {
+          const int h = u / BN;
+          const int n = u - h * BN;
           const int grow = n0 + n;
-          const int gk = (kb + h) * 8 + j;             // group index along K
-          uint4 out = make_uint4(0u, 0u, 0u, 0u);
-          if (grow < p.N && gk < G) {
-            const uint8_t* c = static_cast<const uint8_t*>(p.codes) +
-                               ((static_cast<int64_t>(kb + h) * p.N + grow) * 8 + j) * p.M * eb;
-            float acc[8];
-            for (int m = 0; m < p.M; ++m) {
-              uint4 cw;
-              if (eb == 1) {
-                cw = sbook[m * 256 + c[m]];
-              } else {
-                const int code = c[2 * m] | (c[2 * m + 1] << 8);
-                cw = __ldg(reinterpret_cast<const uint4*>(p.books) + (static_cast<int64_t>(m) << 16) + code);
-              }
-              const __half2* h2 = reinterpret_cast<const __half2*>(&cw);
+          const int gk0 = (kb + h) * 8;                // first group of this K block
+          uint8_t* rowp = b_dst + h * b_half + n * 128;
+          if (grow >= p.N || gk0 >= G) {
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                const float2 f = __half22float2(h2[i]);
-                acc[2 * i] = m == 0 ? f.x : __fadd_rn(acc[2 * i], f.x);
-                acc[2 * i + 1] = m == 0 ? f.y : __fadd_rn(acc[2 * i + 1], f.y);
-              }
-            }
-            uint32_t* o = reinterpret_cast<uint32_t*>(&out);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              __half2 hh = __floats2half2_rn(acc[2 * i], acc[2 * i + 1]);
-              o[i] = *reinterpret_cast<uint32_t*>(&hh);
-            }
+            for (int j = 0; j < 8; ++j)
+              *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = make_uint4(0u, 0u, 0u, 0u);
+            continue;
           }
-          *reinterpret_cast<uint4*>(b_dst + h * b_half + n * 128 + ((j ^ (n & 7)) << 4)) = out;
+          const uint8_t* cp = static_cast<const uint8_t*>(p.codes) +
+                              (static_cast<int64_t>(kb + h) * p.N + grow) * code_bytes;
+          decode_unit_dispatch(p.M, eb, cp, sbook, reinterpret_cast<const uint4*>(p.books), rowp,
+                               n, min(8, G - gk0));
         }
         fence_proxy_async_smem();     // generic writes -> visible to the tensor core
         __syncwarp();
@@ -513,6 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // Sum of the split-K partials, then the fused epilogue.  One thread per 4 outputs.
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, int splits) {
+  grid_dependency_wait();
+  allow_dependents();
   const int64_t nq = static_cast<int64_t>(p.T) * (p.N / 4);
   for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < nq;
        q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -557,8 +640,9 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
     if (e != cudaSuccess) return e;
     configured_bytes = static_cast<int>(bytes);
   }
-  aq_gemm_kernel<<<grid, kThreads, bytes, st>>>(mapA, mapB, mapY, p);
-  return cudaGetLastError();
+  // the decoder warps (10..13) exist only on the fused path
+  const int threads = p.fused ? kThreads : kThreads - kDecodeThreads;
+  return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
 }
 
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st) {
@@ -566,8 +650,8 @@ cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t s
   int64_t blocks = (nq + 255) / 256;
   if (blocks > 152 * 8) blocks = 152 * 8;
   if (blocks < 1) blocks = 1;
-  splitk_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(p, splits);
-  return cudaGetLastError();
+  return launch_pdl(splitk_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, p,
+                    splits);
 }
 
 cudaError_t read_clear_gemm_error(unsigned* out) {

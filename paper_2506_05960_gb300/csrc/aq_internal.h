@@ -6,6 +6,7 @@
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
+#include <utility>
 
 namespace aq {
 
@@ -55,6 +56,24 @@ struct LutParams {
   int G;                        // K / 8
   int chunks, rows_per_cta;
 };
+
+// Launch with programmatic stream serialization (the kernel must call
+// grid_dependency_wait() before touching global memory).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Launchers (return the launch status; they never synchronise).
 cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s, cudaStream_t st);

@@ -18,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include "aq_internal.h"
+#include "aq_ptx.cuh"
 
 namespace aq {
 
@@ -26,6 +27,8 @@ __global__ void __launch_bounds__(256) lut_kernel(const LutParams p) {
   float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256][Tp]
   const int J = p.J, M = p.M, Tp = p.Tp, T = p.T;
   float* xs = L + static_cast<size_t>(J) * M * 256 * Tp;       // [T][J*8]
+  grid_dependency_wait();
+  allow_dependents();
   const int chunk = blockIdx.x;
   const int g0 = chunk * J;
   const int nj = min(J, p.G - g0);
@@ -125,8 +128,7 @@ cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
   }
   const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
   dim3 grid(p.chunks, n_slices);
-  lut_kernel<<<grid, 256, bytes, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(lut_kernel, grid, dim3(256), bytes, st, p);
 }
 
 }  // namespace aq

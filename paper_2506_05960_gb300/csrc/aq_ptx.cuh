@@ -76,6 +76,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
   }
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Kernels are launched with programmatic stream serialization: a kernel may start while
+// its predecessor in the stream still runs, so it waits (grid_dependency_wait) for the
+// predecessor to complete and flush its memory before reading or writing global memory,
+// and lets its own successor start launching early (allow_dependents).  Both are no-ops
+// for a kernel launched without the attribute.
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+__device__ __forceinline__ void allow_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- shared-memory counters
 // A release-add by a producer and an acquire-poll by a consumer: a cheaper hand-off
 // than an mbarrier for a single waiting thread that must stay lean.
