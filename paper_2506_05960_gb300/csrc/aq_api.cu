@@ -125,11 +125,14 @@ double decode_stage_cycles(int BN, int M, int B) {
 
 int book_smem_bytes(bool fused, int M, int B) { return (fused && B == 8) ? M * 256 * 16 : 0; }
 
-void finish_plan(Plan& pl, bool f32_out, int book_bytes) {
+// Fused path: packed code bytes of one row for one 64-wide K block, staged per stage.
+int code_smem_bytes(bool fused, int M, int B) { return fused ? 8 * M * (B / 8) : 0; }
+
+void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes) {
   pl.acc_stride = pl.BN;
   pl.a_col = 2 * pl.acc_stride;
   pl.a_stages = aq::gemm_a_stages(pl.BN);
-  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1, book_bytes);
+  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1, book_bytes, code_bytes);
   pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
 }
 
@@ -141,12 +144,13 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
                bool fused = false, int M = 1, int B = 8) {
   const int num_kb = (K + aq::kBK - 1) / aq::kBK;
   const int book_bytes = book_smem_bytes(fused, M, B);
+  const int code_bytes = code_smem_bytes(fused, M, B);
   double best = 1e30;
   Plan bp{};
   for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
     if (BN == 224) continue;
     if (aq::gemm_a_stages(BN) < 2) continue;
-    if (aq::gemm_max_stages(BN, true, book_bytes) < 2) continue;
+    if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes) < 2) continue;
     const int n_tiles = (N + BN - 1) / BN;
     const int max_split = allow_split ? std::min(num_kb, 64) : 1;
     double st_cyc = stage_cycles(BN);
@@ -176,7 +180,7 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
       }
     }
   }
-  finish_plan(bp, f32_out, book_bytes);
+  finish_plan(bp, f32_out, book_bytes, code_bytes);
   return bp;
 }
 

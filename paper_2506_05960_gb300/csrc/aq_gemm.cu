@@ -54,19 +54,24 @@ struct alignas(8) GemmBarriers {
   uint64_t acc_full[2];          // accumulator buffer complete (commit)
   uint64_t acc_empty[2];         // accumulator buffer drained (4 epilogue warps)
   uint64_t drain;                // all MMAs of this CTA complete (teardown)
+  uint64_t codes_full[kMaxStages];  // fused path: a stage's packed codes landed in smem
   uint32_t tmem_base;
   int abort_flag;
 };
 
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes) {
-  return 1024 + static_cast<size_t>(stages) * (kStageBlocks * BN * 128 + kA8Stage) +
+// code_bytes: packed code bytes of one row for one 64-wide K block on the fused path
+// (8 * M * bytes per code), 0 on the dense path.
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes) {
+  return 1024 +
+         static_cast<size_t>(stages) *
+             (kStageBlocks * BN * 128 + kA8Stage + kStageBlocks * BN * code_bytes) +
          4 * 2 * (f32_out ? kEpiBuf32 : kEpiBuf16) + kScaleBytes + book_bytes +
          sizeof(GemmBarriers);
 }
 
-int gemm_max_stages(int BN, bool f32_out, int book_bytes) {
-  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes);
-  const size_t per = static_cast<size_t>(kStageBlocks) * BN * 128 + kA8Stage;
+int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes) {
+  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes, code_bytes);
+  const size_t per = static_cast<size_t>(kStageBlocks) * BN * (128 + code_bytes) + kA8Stage;
   const int s = static_cast<int>((232448 - fixed) / per);
   return s < kMaxStages ? s : kMaxStages;
 }
@@ -111,10 +116,50 @@ struct Ring {
   }
 };
 
+// Sum of the M codewords of one group in fp32 (ascending m), one RNE to fp16 (Eq. 4).
+// For M <= 2 the fp16 adds give the same bits: the exact sum of two fp16 values
+// rounded once to fp32 and then to fp16 equals its direct fp16 rounding, since
+// fp32 carries at least 2 * 11 + 2 significand bits (double rounding is innocuous).
+template <int M>
+__device__ __forceinline__ uint4 sum_codewords(const uint4* word) {
+  if constexpr (M == 1) {
+    return word[0];
+  } else if constexpr (M == 2) {
+    uint4 out;
+    const __half2* a = reinterpret_cast<const __half2*>(&word[0]);
+    const __half2* b = reinterpret_cast<const __half2*>(&word[1]);
+    __half2* o = reinterpret_cast<__half2*>(&out);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = __hadd2(a[i], b[i]);
+    return out;
+  } else {
+    float acc[8];
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      const __half2* h2 = reinterpret_cast<const __half2*>(&word[m]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __half22float2(h2[i]);
+        acc[2 * i] = m == 0 ? f.x : __fadd_rn(acc[2 * i], f.x);
+        acc[2 * i + 1] = m == 0 ? f.y : __fadd_rn(acc[2 * i + 1], f.y);
+      }
+    }
+    uint4 out;
+    uint32_t* o = reinterpret_cast<uint32_t*>(&out);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      __half2 hh = __floats2half2_rn(acc[2 * i], acc[2 * i + 1]);
+      o[i] = *reinterpret_cast<uint32_t*>(&hh);
+    }
+    return out;
+  }
+}
+
 // Fused path: decode the 8 groups of one output row in one 64-wide K block into the
-// row's 128-byte line of the swizzled B stage.  Codes: 8*M*EB contiguous bytes
-// (EB = bytes per code), read as 32-bit words and unpacked with constant shifts;
-// all codeword reads are issued before the fp32 sums (ascending m, one RNE to fp16).
+// row's 128-byte line of the swizzled B stage.  Codes: 8*M*EB contiguous bytes in
+// shared memory (EB = bytes per code), read as 32-bit words and unpacked with
+// constant shifts.  8-bit codes index the codebooks staged in shared memory;
+// 16-bit codes gather from L2, all 8*M reads issued before the first sum.
 template <int M, int EB>
 __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* sbook,
                                             const uint4* gbooks, uint8_t* rowp, int n,
@@ -124,7 +169,7 @@ __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* s
   if constexpr (kWords % 4 == 0) {
 #pragma unroll
     for (int i = 0; i < kWords / 4; ++i) {
-      const uint4 v = __ldg(reinterpret_cast<const uint4*>(codes) + i);
+      const uint4 v = reinterpret_cast<const uint4*>(codes)[i];
       w[4 * i] = v.x;
       w[4 * i + 1] = v.y;
       w[4 * i + 2] = v.z;
@@ -133,13 +178,11 @@ __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* s
   } else {
 #pragma unroll
     for (int i = 0; i < kWords / 2; ++i) {
-      const uint2 v = __ldg(reinterpret_cast<const uint2*>(codes) + i);
+      const uint2 v = reinterpret_cast<const uint2*>(codes)[i];
       w[2 * i] = v.x;
       w[2 * i + 1] = v.y;
     }
   }
-  // 16-bit codes gather from L2: issue all 8*M reads first.  8-bit codes read the
-  // codebooks from shared memory as they are summed.
   constexpr int kPre = EB == 2 ? 8 * M : 1;
   uint4 cw[kPre];
   if (EB == 2) {
@@ -155,29 +198,16 @@ __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* s
   for (int j = 0; j < 8; ++j) {
     uint4 out = make_uint4(0u, 0u, 0u, 0u);
     if (j < gvalid) {
-      float acc[8];
+      uint4 word[M];
 #pragma unroll
       for (int m = 0; m < M; ++m) {
         const int idx = j * M + m;
-        uint4 word;
         if (EB == 1)
-          word = sbook[m * 256 + ((w[idx >> 2] >> (8 * (idx & 3))) & 0xFFu)];
+          word[m] = sbook[m * 256 + ((w[idx >> 2] >> (8 * (idx & 3))) & 0xFFu)];
         else
-          word = cw[idx % kPre];
-        const __half2* h2 = reinterpret_cast<const __half2*>(&word);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float2 f = __half22float2(h2[i]);
-          acc[2 * i] = m == 0 ? f.x : __fadd_rn(acc[2 * i], f.x);
-          acc[2 * i + 1] = m == 0 ? f.y : __fadd_rn(acc[2 * i + 1], f.y);
-        }
+          word[m] = cw[idx % kPre];
       }
-      uint32_t* o = reinterpret_cast<uint32_t*>(&out);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        __half2 hh = __floats2half2_rn(acc[2 * i], acc[2 * i + 1]);
-        o[i] = *reinterpret_cast<uint32_t*>(&hh);
-      }
+      out = sum_codewords<M>(word);
     }
     *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = out;
   }
@@ -225,8 +255,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* epi = aring + S * kA8Stage;
   float* sscale = reinterpret_cast<float*>(epi + 4 * 2 * epi_buf);
   uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) + kScaleBytes);
-  GemmBarriers* bar =
-      reinterpret_cast<GemmBarriers*>(reinterpret_cast<uint8_t*>(sbook) + p.book_bytes);
+  // fused path: each stage's packed codes, [h][BN rows][code_bytes] (16-byte aligned)
+  const int code_bytes = p.fused ? 8 * p.M * (p.B >> 3) : 0;
+  const int code_stage = kStageBlocks * BN * code_bytes;
+  uint8_t* scodes = reinterpret_cast<uint8_t*>(sbook) + p.book_bytes;
+  GemmBarriers* bar = reinterpret_cast<GemmBarriers*>(scodes + S * code_stage);
   const volatile int* abort_flag = &bar->abort_flag;
 
   const int warp = threadIdx.x >> 5;
@@ -255,6 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar->acc_empty[b], 4);
     }
     mbar_init(&bar->drain, 1);
+    for (int s = 0; s < S; ++s) mbar_init(&bar->codes_full[s], 1);
     bar->abort_flag = 0;
     mbar_fence_init();
     tma_prefetch_desc(&mapA);
@@ -299,6 +333,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           uint64_t* fb = &bar->full[rg.s];
+          if (p.fused) {
+            // the stage's codes: per K block, rows n0 .. n0+rows-1 are contiguous in
+            // the packed layout (rows is a multiple of 8, so sizes are multiples of 16)
+            const int rows = min(BN, p.N - n0);
+            const uint32_t bytes = static_cast<uint32_t>(rows * code_bytes);
+            uint64_t* cbar = &bar->codes_full[rg.s];
+            mbar_arrive_expect_tx(cbar, nb * bytes);
+            for (int h = 0; h < nb; ++h)
+              bulk_load(scodes + rg.s * code_stage + h * BN * code_bytes,
+                        static_cast<const uint8_t*>(p.codes) +
+                            (static_cast<int64_t>(kb + h) * p.N + n0) * code_bytes,
+                        bytes, cbar);
+          }
           mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (kA8Half + (p.fused ? 0 : b_half))));
           uint8_t* a_dst = aring + rg.s * kA8Stage;
           uint8_t* b_dst = bring + rg.s * b_stage;
@@ -326,7 +373,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         Ring d;
         const uint32_t first = issued > static_cast<uint32_t>(S) ? issued - S : 0u;
         for (uint32_t i = 0; i < issued; ++i) {
-          if (i >= first && !mbar_wait(&bar->full[d.s], d.ph, &zero)) {
+          if (i >= first && (!mbar_wait(&bar->full[d.s], d.ph, &zero) ||
+                             (p.fused && !mbar_wait(&bar->codes_full[d.s], d.ph, &zero)))) {
             atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
             break;
           }
@@ -548,17 +596,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int n0 = tc.n_tile * BN;
       for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
         const int nb = min(kStageBlocks, tc.kb_end - kb);
-        if (!rg.lap0 && !mbar_wait(&bar->empty[rg.s], rg.ph ^ 1u, abort_flag)) {
-          if (!*abort_flag) record_failure(bar, kDevErrTimeoutEmpty);
+        // the producer copies a stage's codes only after the stage is free, so their
+        // arrival also means the B stage may be overwritten
+        if (!mbar_wait(&bar->codes_full[rg.s], rg.ph, abort_flag)) {
+          if (!*abort_flag) record_failure(bar, kDevErrTimeoutFull);
           failed = true;
           break;
         }
         uint8_t* b_dst = bring + rg.s * b_stage;
+        const uint8_t* c_src = scodes + rg.s * code_stage;
         // unit = (64-wide K block h, output row n): its 8 groups' codes are contiguous
-        // (8*M*eb bytes, 16-byte aligned) and are read with vector loads; all of the
-        // unit's codeword reads are issued before any is used.
+        // (8*M*eb bytes, 8-byte aligned) and are read with vector loads.
         const int units = nb * BN;
-        const int code_bytes = 8 * p.M * eb;
         for (int u = dt; u < units; u += kDecodeThreads) {
           const int h = u / BN;
           const int n = u - h * BN;
@@ -571,8 +620,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = make_uint4(0u, 0u, 0u, 0u);
             continue;
           }
-          const uint8_t* cp = static_cast<const uint8_t*>(p.codes) +
-                              (static_cast<int64_t>(kb + h) * p.N + grow) * code_bytes;
+          const uint8_t* cp = c_src + u * code_bytes;
           decode_unit_dispatch(p.M, eb, cp, sbook, reinterpret_cast<const uint4*>(p.books), rowp,
                                n, min(8, G - gk0));
         }
@@ -633,7 +681,8 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
                         const GemmParams& p, int grid, cudaStream_t st) {
   static int configured_bytes = 0;
   const size_t bytes =
-      gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes);
+      gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes,
+                      p.fused ? 8 * p.M * (p.B >> 3) : 0);
   if (static_cast<int>(bytes) > configured_bytes) {
     cudaError_t e = cudaFuncSetAttribute(aq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(bytes));

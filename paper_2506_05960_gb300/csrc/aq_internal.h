@@ -81,8 +81,10 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes);
-int gemm_max_stages(int BN, bool f32_out, int book_bytes);  // smem ring depth that fits
+// code_bytes: packed code bytes per row and 64-wide K block staged per stage on
+// the fused path (8 * M * bytes per code), 0 on the dense path.
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes);
+int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes);  // ring depth that fits
 int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-column accumulators
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st);

@@ -68,3 +68,27 @@ def test_auto_paths_small_tokens_run_fused_or_lut():
     assert aq.aq_linear_workspace_size(128, 960, 2880, 8, 2, 8, 0) == \
         aq.aq_linear_workspace_size(128, 960, 2880, 8, 2, 8, FUSED)
     assert aq.aq_linear_workspace_size(128, 960, 2880, 8, 2, 8, FUSED) < 960 * 2880 * 2
+
+
+@pytest.mark.parametrize("path", [DENSE, FUSED])
+@pytest.mark.parametrize("M,B", [(1, 8), (2, 8), (3, 8), (4, 8), (8, 8), (1, 16), (2, 16)])
+def test_decode_inside_gemm_bit_exact(M, B, path):
+    """Identity activations (x[t][k] = [t == k], s_x = scale = 1, no bias, fp32 out)
+    make the layer return W-hat transposed exactly, so the weights the tensor core
+    multiplied are compared bit for bit (as values: a zero's sign is not kept by
+    the sum) with the decode rule of Eq. 4, on edge-value codebooks: subnormals,
+    halfway cases, large magnitudes whose sums stay finite."""
+    rng = np.random.default_rng(100 * M + B)
+    K = 208                                 # ragged last K block (3.25 blocks)
+    N = 72                                  # ragged N tile
+    special = np.array([8000, -8000, 6e-8, -6e-8, 0.0, -0.0, 1.0, 2 ** -14, 1e-5,
+                        1 + 2 ** -10, -(1 + 2 ** -10), 2049, 0.1, -3.0e-5], dtype=np.float16)
+    books = special[rng.integers(0, special.size, size=(M, 1 << B, 8))].astype(np.float16)
+    codes = rng.integers(0, 1 << B, size=(N, K // 8, M),
+                         dtype=np.uint8 if B == 8 else np.uint16)
+    inp = dict(xq=np.eye(K, dtype=np.int8), s_x=1.0, codebooks=books, codes=codes,
+               scale=np.ones(N, dtype=np.float16), bias=np.zeros(N, dtype=np.float16))
+    y = run_linear(inp, out_f32=True, with_bias=False, path=path)
+    ref = O.decode_rule_f16(codes, books).astype(np.float64)      # [N][K]
+    assert np.isfinite(ref).all()
+    assert np.array_equal(y, ref.T)
