@@ -120,9 +120,11 @@ def make_linear(spec: LinearSpec, seed: int) -> dict:
 
 
 def make_conv(spec: ConvSpec, seed: int) -> dict:
-    """Random AQ conv layer (OHWI groups along Cin per tap) + NHWC int8 input."""
+    """Random AQ conv layer + NHWC int8 input.  g = 8: groups along Cin inside
+    each tap (OHWI); g = 9: one group per (output channel, input channel) 3x3
+    filter, codes [Cout][Cin][M] and codebooks [M][2^B][9]."""
     K = spec.K
-    if spec.Cin % spec.g:
+    if spec.g != 9 and spec.Cin % spec.g:
         raise ValueError("Cin must be a multiple of g")
     rng = np.random.default_rng(seed)
     codebooks, codes, scale, bias = _weights(rng, spec.Cout, K, spec.g, spec.M,

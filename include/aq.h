@@ -20,6 +20,10 @@
  *   - Sizes are element counts.  Arrays are dense, row-major, C-contiguous.
  *   - Every pointer must be 16-byte aligned (AQ_ERR_ALIGN otherwise).
  *   - Supported formats: g = 8; B = 8 with M in 1..8, or B = 16 with M in 1..2.
+ *     g = 9 selects the kernel-aware grouping of a 3x3 convolution (Sec. 3.1.2,
+ *     App. A.1 Eq. A4: one group = the 9 taps of one (output channel, input
+ *     channel) filter); it is accepted by aq_packed_size, aq_pack, aq_decode,
+ *     aq_conv2d_workspace_size and aq_conv2d_nhwc (dense path) only.
  *     Codes of B = 8 are uint8, codes of B = 16 are uint16 (little endian).
  *     Codebooks are fp16 [M][2^B][g].  Per-output-channel scale and bias are
  *     fp16 [N] (bias may be NULL).  The activation scale s_x is fp32.
@@ -111,7 +115,9 @@ AQ_API int aq_profile_read(double* ms_out, int64_t* launches_out, int n_kinds);
  * [ceil(K/64)][N][64/g][M], i.e. for each 64-wide block of K the codes that one
  * output row needs are contiguous (16 bytes for M = 2, B = 8) and consecutive
  * rows follow each other, so a warp reads a block of rows with 128-bit loads.
- * Codes of a zero-padded K tail are 0.                                        */
+ * Codes of a zero-padded K tail are 0.
+ * g = 9 (kernel-aware grouping, K = 9*Cin): canonical codes are [Cout][Cin][M]
+ * and the packed layout is that same array (aq_pack copies it).              */
 
 /* Bytes of the packed buffer for an N x K layer. */
 AQ_API int aq_packed_size(int N, int K, int g, int M, int B, size_t* bytes);
@@ -124,7 +130,10 @@ AQ_API int aq_pack(const void* codes_canon, void* codes_packed,
  * W_out[n][k] = fp16( sum_{m=0..M-1} fp32(C^(m)[b[n, k/g, m]][k mod g]) ), the
  * fp32 sum taken in ascending m and rounded once to fp16 (round to nearest
  * even, overflow to +-inf, subnormals kept).  Bit-exact against that rule.
- * The per-channel scale is NOT folded in.  W_out is fp16 [N][K].             */
+ * The per-channel scale is NOT folded in.  W_out is fp16 [N][K].
+ * g = 9 (kernel-aware grouping): codebooks fp16 [M][2^B][9]; the group of
+ * (n, c) holds the 9 taps t = i*3 + j of that filter and is written in the
+ * convolution's OHWI order, W_out[n][t*Cin + c] with Cin = K/9 (same rule).   */
 AQ_API int aq_decode(const void* codes_packed, const void* codebooks, void* W_out,
               int N, int K, int g, int M, int B, void* stream);
 
@@ -183,7 +192,9 @@ AQ_API int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_pack
  * y[b][ho][wo][n] = (s_x*scale[n]) * sum_{i,j,c} xq[b][ho*s+i-pad][wo*s+j-pad][c]
  *                   * W[n][(i*kw + j)*Cin + c] + bias[n],
  * out-of-image taps read as 0.  The weight is the decoded AQ matrix [Cout][K]
- * with K = kh*kw*Cin in OHWI order, groups of g along Cin inside one tap.
+ * with K = kh*kw*Cin in OHWI order, groups of g = 8 along Cin inside one tap,
+ * or g = 9: one group per (n, c) filter (codes [Cout][Cin][M], dense path;
+ * AQ_PATH_FUSED and AQ_PATH_LUT return AQ_ERR_UNSUPPORTED, AUTO picks dense).
  *   xq int8 [Nb][H][W][Cin];  y [Nb][Ho][Wo][Cout] of out_dtype,
  *   Ho = (H + 2*pad - kh)/stride + 1, Wo likewise.
  *   Supported: kh = kw = 3, pad = 1, stride 1 or 2, Cin % 64 == 0,

@@ -30,7 +30,7 @@ import math
 import numpy as np
 
 __all__ = [
-    "decode_f64", "decode_rule_f16", "decode_kaq_f64", "pack_codes", "packed_nbytes",
+    "decode_f64", "decode_rule_f16", "decode_kaq_f64", "kaq_ohwi", "pack_codes", "packed_nbytes",
     "quant_act", "linear_f64", "conv2d_nhwc_f64", "lut_linear_f64",
     "lut_conv_kaq_counted", "direct_conv_counted", "eq_a7_flops", "eq_a2_flops",
     "paper_lut_breakeven", "eq_a7_breakeven", "bits_per_weight",
@@ -93,6 +93,14 @@ def decode_kaq_f64(codes: np.ndarray, codebooks: np.ndarray) -> np.ndarray:
     for m in range(M):
         F += C[m][codes[:, :, m].astype(np.int64)]
     return F
+
+
+def kaq_ohwi(F: np.ndarray) -> np.ndarray:
+    """Layout only: kernel-aware filters F [Cout][Cin][h1*w1] (taps row-major)
+    -> the OHWI weight matrix [Cout][h1*w1*Cin] of ``conv2d_nhwc_f64``, reduction
+    index k = t*Cin + c for tap t and input channel c."""
+    Cout, Cin, taps = F.shape
+    return np.ascontiguousarray(F.transpose(0, 2, 1)).reshape(Cout, taps * Cin)
 
 
 # --------------------------------------------------------------------------- packing
@@ -210,9 +218,14 @@ def lut_linear_f64(xq: np.ndarray, s_x: float, codes: np.ndarray,
 
 
 def layer_f64(inp: dict) -> np.ndarray:
-    """Reference output of an ``aq_synth`` layer dict (linear or conv)."""
-    W = decode_f64(inp["codes"], inp["codebooks"])
+    """Reference output of an ``aq_synth`` layer dict (linear or conv).  A conv
+    spec with g = 9 uses the kernel-aware grouping (Sec. 3.1.2): one group per
+    (output channel, input channel) 3x3 filter."""
     spec = inp["spec"]
+    if getattr(spec, "g", 8) == 9 and inp["xq"].ndim == 4:
+        W = kaq_ohwi(decode_kaq_f64(inp["codes"], inp["codebooks"]))
+    else:
+        W = decode_f64(inp["codes"], inp["codebooks"])
     if inp["xq"].ndim == 2:
         return linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"])
     return conv2d_nhwc_f64(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"],

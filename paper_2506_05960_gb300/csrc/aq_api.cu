@@ -48,9 +48,17 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-// ---- format checks (g, M, B)
-int check_format(int g, int M, int B) {
-  if (g != 8) return set_error(AQ_ERR_UNSUPPORTED, "group size g=%d unsupported (g=8 only)", g);
+// ---- format checks (g, M, B).  g = 9 is the kernel-aware grouping of a 3x3 conv
+// (one group per (output channel, input channel) filter); only the entry points
+// that can take it pass allow_kaq.
+constexpr int kKaqGroup = 9;
+
+int check_format(int g, int M, int B, bool allow_kaq = false) {
+  if (g != 8 && !(allow_kaq && g == kKaqGroup))
+    return set_error(AQ_ERR_UNSUPPORTED,
+                     allow_kaq ? "group size g=%d unsupported (8, or 9 for 3x3 convolutions)"
+                               : "group size g=%d unsupported here (g=8)",
+                     g);
   if (B == 8) {
     if (M < 1 || M > 8) return set_error(AQ_ERR_UNSUPPORTED, "M=%d unsupported for B=8 (1..8)", M);
   } else if (B == 16) {
@@ -200,14 +208,17 @@ size_t fused_ws_bytes(int T, int N, const Plan& pl) {
 // into the workspace is cheaper.
 constexpr int kFusedAutoMaxMTiles = 1;
 
-// Path of a convolution: -1 unknown path, -2 path cannot run this layer.
-int resolve_conv_path(int path, int m_tiles) {
+// Path of a convolution: -1 unknown path, -2 path cannot run this layer.  The
+// kernel-aware grouping (g = 9) is decoded by its own pass: dense path only.
+int resolve_conv_path(int path, int m_tiles, int g) {
+  const bool kaq = g == kKaqGroup;
   switch (path) {
     case AQ_PATH_AUTO:
-      return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
+      return (m_tiles <= kFusedAutoMaxMTiles && !kaq) ? AQ_PATH_FUSED : AQ_PATH_DENSE;
     case AQ_PATH_DENSE:
-    case AQ_PATH_FUSED:
       return path;
+    case AQ_PATH_FUSED:
+      return kaq ? -2 : path;
     case AQ_PATH_LUT:
       return -2;
     default:
@@ -424,8 +435,10 @@ int sm_count() {
 // Tensor-core path after the activation map is built.  Dense: decode W-hat into the
 // workspace (Wdec), then the GEMM streams it with TMA.  Fused (Wdec == nullptr): the
 // GEMM's decoder warps rebuild each weight tile in shared memory from the codes.
+// kaq: the codes use the kernel-aware grouping (g = 9, dense path only).
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
-             const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st) {
+             const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
+             bool kaq = false) {
   const bool fused = Wdec == nullptr;
   p.fused = fused ? 1 : 0;
   p.codes = codes_packed;
@@ -481,7 +494,8 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   cudaError_t e;
   if (!fused) {
     ProfScope ps(kProfDecode, st);
-    e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+    e = kaq ? aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st)
+            : aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
     if (e != cudaSuccess) return cuda_status(e, "decode launch");
   }
   {
@@ -582,22 +596,33 @@ int aq_device_error(int* code_out) {
 
 int aq_packed_size(int N, int K, int g, int M, int B, size_t* bytes) {
   if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
-  int r = check_format(g, M, B);
+  int r = check_format(g, M, B, true);
   if (r) return r;
   if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
-  *bytes = static_cast<size_t>((K + 63) / 64) * N * (64 / g) * M * (B / 8);
+  if (g == kKaqGroup)
+    *bytes = static_cast<size_t>(N) * (K / g) * M * (B / 8);   // the canonical layout
+  else
+    *bytes = static_cast<size_t>((K + 63) / 64) * N * (64 / g) * M * (B / 8);
   return ok();
 }
 
 int aq_pack(const void* codes_canon, void* codes_packed, int N, int K, int g, int M, int B,
             void* stream) {
   if (!codes_canon || !codes_packed) return set_error(AQ_ERR_NULL, "NULL code buffer");
-  int r = check_format(g, M, B);
+  int r = check_format(g, M, B, true);
   if (r) return r;
   if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
   if (!aligned16(codes_canon) || !aligned16(codes_packed))
     return set_error(AQ_ERR_ALIGN, "code buffers must be 16-byte aligned");
   ProfScope ps(kProfPack, static_cast<cudaStream_t>(stream));
+  if (g == kKaqGroup) {
+    // one group per filter: the decode reads a group's M codes at once, so the
+    // stored layout is the canonical [N][Cin][M] itself
+    const size_t bytes = static_cast<size_t>(N) * (K / g) * M * (B / 8);
+    return cuda_status(cudaMemcpyAsync(codes_packed, codes_canon, bytes, cudaMemcpyDeviceToDevice,
+                                       static_cast<cudaStream_t>(stream)),
+                       "aq_pack copy");
+  }
   return cuda_status(aq::launch_pack(codes_canon, codes_packed, N, K, M, B,
                                      static_cast<cudaStream_t>(stream)),
                      "aq_pack launch");
@@ -606,12 +631,16 @@ int aq_pack(const void* codes_canon, void* codes_packed, int N, int K, int g, in
 int aq_decode(const void* codes_packed, const void* codebooks, void* W_out, int N, int K, int g,
               int M, int B, void* stream) {
   if (!codes_packed || !codebooks || !W_out) return set_error(AQ_ERR_NULL, "NULL argument");
-  int r = check_format(g, M, B);
+  int r = check_format(g, M, B, true);
   if (r) return r;
   if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
   if (!aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(W_out))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   ProfScope ps(kProfDecode, static_cast<cudaStream_t>(stream));
+  if (g == kKaqGroup)
+    return cuda_status(aq::launch_decode_kaq(codes_packed, codebooks, W_out, N, K / g, M, B,
+                                             static_cast<cudaStream_t>(stream)),
+                       "aq_decode launch");
   return cuda_status(aq::launch_decode(codes_packed, codebooks, W_out, N, K, M, B,
                                        static_cast<cudaStream_t>(stream)),
                      "aq_decode launch");
@@ -733,14 +762,14 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
                              int pad, int g, int M, int B, int path, size_t* bytes) {
   if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
-  int r = check_format(g, M, B);
+  int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
   if (r) return r;
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles);
+  const int rp = resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
@@ -752,7 +781,7 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
                    const void* scale, const void* bias, void* y, int out_dtype, int Nb, int H,
                    int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
                    int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
-  int r = check_format(g, M, B);
+  int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
   if (r) return r;
@@ -763,7 +792,7 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles);
+  const int rp = resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
   if (Nb == 0) return ok();
   if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
@@ -809,7 +838,8 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st);
+  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st,
+                  g == kKaqGroup);
 }
 
 }  // extern "C"

@@ -210,4 +210,68 @@ cudaError_t launch_decode(const void* packed, const void* books, void* W, int N,
                     static_cast<__half*>(W), N, K, M, KB);
 }
 
+// ============================================================== kernel-aware decode (g = 9)
+// Sec. 3.1.2 / App. A.1 Eq. A4: one group = the 3x3 taps of one (output channel n,
+// input channel c) filter; codes [N][Cin][M], codebooks [M][2^B][9] fp16.  The
+// decoded filter is written in the K order of the implicit-GEMM convolution,
+// W[n][t*Cin + c] for tap t = i*3 + j, so the tensor-core path is unchanged.  Same
+// rule as the 8-wide decode: fp32 sum in ascending m, one RNE to fp16.  One thread
+// per (n, c): consecutive threads take consecutive c, so each tap's stores are
+// contiguous across the warp.  8-bit books are staged in shared memory.
+template <int EB>
+__global__ void __launch_bounds__(256) decode_kaq_kernel(const uint8_t* __restrict__ codes,
+                                                         const __half* __restrict__ books,
+                                                         __half* __restrict__ W, int N, int Cin,
+                                                         int M) {
+  extern __shared__ __half sbook9[];                     // [M][256][9] for 8-bit codes
+  grid_dependency_wait();
+  allow_dependents();
+  if constexpr (EB == 1) {
+    for (int i = threadIdx.x; i < M * 256 * 9; i += blockDim.x) sbook9[i] = books[i];
+    __syncthreads();
+  }
+  const int K = 9 * Cin;
+  const int64_t total = static_cast<int64_t>(N) * Cin;
+  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int n = static_cast<int>(idx / Cin);
+    const int c = static_cast<int>(idx - static_cast<int64_t>(n) * Cin);
+    float acc[9];
+    for (int m = 0; m < M; ++m) {
+      const __half* cw;
+      if constexpr (EB == 1) {
+        cw = sbook9 + (m * 256 + codes[idx * M + m]) * 9;
+      } else {
+        const uint16_t b = reinterpret_cast<const uint16_t*>(codes)[idx * M + m];
+        cw = books + ((static_cast<int64_t>(m) << 16) + b) * 9;
+      }
+#pragma unroll
+      for (int t = 0; t < 9; ++t) {
+        const float v = __half2float(EB == 1 ? cw[t] : __ldg(cw + t));
+        acc[t] = m == 0 ? v : __fadd_rn(acc[t], v);
+      }
+    }
+    __half* out = W + static_cast<int64_t>(n) * K + c;
+#pragma unroll
+    for (int t = 0; t < 9; ++t) out[static_cast<int64_t>(t) * Cin] = __float2half_rn(acc[t]);
+  }
+}
+
+cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int N, int Cin, int M,
+                              int B, cudaStream_t st) {
+  const int64_t total = static_cast<int64_t>(N) * Cin;
+  int64_t blocks = (total + 255) / 256;
+  const int64_t cap = B == 8 ? 152 * 2 : 152 * 8;       // 8-bit: every block stages the books
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  const uint8_t* c = static_cast<const uint8_t*>(codes);
+  const __half* b = static_cast<const __half*>(books);
+  __half* w = static_cast<__half*>(W);
+  if (B == 8)
+    return launch_pdl(decode_kaq_kernel<1>, dim3(static_cast<unsigned>(blocks)), dim3(256),
+                      static_cast<size_t>(M) * 256 * 9 * 2, st, c, b, w, N, Cin, M);
+  return launch_pdl(decode_kaq_kernel<2>, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, c,
+                    b, w, N, Cin, M);
+}
+
 }  // namespace aq

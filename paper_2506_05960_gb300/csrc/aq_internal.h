@@ -81,6 +81,10 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
+// Kernel-aware grouping (g = 9, 3x3 conv): codes [N][Cin][M], books [M][2^B][9] ->
+// W [N][9*Cin] in the convolution's OHWI K order.
+cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int N, int Cin, int M,
+                              int B, cudaStream_t st);
 // code_bytes: packed code bytes per row and 64-wide K block staged per stage on
 // the fused path (8 * M * bytes per code), 0 on the dense path.
 size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes);

@@ -17,11 +17,11 @@ def poison(shape, dtype):
     return torch.full(shape, float("nan"), dtype=dtype, device="cuda")
 
 
-def pack(codes, N, K, M, B):
+def pack(codes, N, K, M, B, g=8):
     import torch
     import paper_2506_05960_gb300 as aq
-    packed = torch.empty(aq.aq_packed_size(N, K, 8, M, B), dtype=torch.uint8, device="cuda")
-    aq.aq_pack(dev(codes), packed, N, K, 8, M, B)
+    packed = torch.empty(aq.aq_packed_size(N, K, g, M, B), dtype=torch.uint8, device="cuda")
+    aq.aq_pack(dev(codes), packed, N, K, g, M, B)
     return packed
 
 
@@ -52,15 +52,16 @@ def run_conv(inp, out_f32=False, with_bias=True, path=0):
     N, G, M = inp["codes"].shape
     B = 8 if inp["codes"].dtype == np.uint8 else 16
     K = s.kh * s.kw * s.Cin
-    packed = pack(inp["codes"], N, K, M, B)
+    g = s.g                               # 8, or 9 for one group per 3x3 filter
+    packed = pack(inp["codes"], N, K, M, B, g)
     ws_bytes = aq.aq_conv2d_workspace_size(s.Nb, s.H, s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride,
-                                           s.pad, 8, M, B, path)
+                                           s.pad, g, M, B, path)
     ws = torch.empty(max(ws_bytes, 16), dtype=torch.uint8, device="cuda")
     y = poison((s.Nb, s.Ho, s.Wo, s.Cout), torch.float32 if out_f32 else torch.float16)
     aq.aq_conv2d_nhwc(dev(inp["xq"]), inp["s_x"], packed, dev(inp["codebooks"]),
                       dev(inp["scale"]), dev(inp["bias"]) if with_bias else None, y,
                       aq.AQ_DTYPE_F32 if out_f32 else aq.AQ_DTYPE_F16, s.Nb, s.H, s.W, s.Cin,
-                      s.Cout, s.kh, s.kw, s.stride, s.pad, 8, M, B, ws, ws_bytes, path)
+                      s.Cout, s.kh, s.kw, s.stride, s.pad, g, M, B, ws, ws_bytes, path)
     torch.cuda.synchronize()
     assert aq.aq_device_error() == 0
     return y.float().cpu().numpy().astype(np.float64)

@@ -75,7 +75,7 @@ def test_packed_size(lib):
     assert r == 0 and v == 4 * 8 * 8 * 3
 
 
-@pytest.mark.parametrize("g,M,B,code", [(9, 2, 8, -3), (8, 0, 8, -3), (8, 9, 8, -3),
+@pytest.mark.parametrize("g,M,B,code", [(10, 2, 8, -3), (4, 2, 8, -3), (8, 0, 8, -3), (8, 9, 8, -3),
                                         (8, 3, 16, -3), (8, 2, 4, -3)])
 def test_unsupported_formats(lib, g, M, B, code):
     r, _ = _size(lib.aq_packed_size, 64, 64, g, M, B)
@@ -121,3 +121,23 @@ def test_workspace_sizes(lib):
     assert r == 0 and v >= 2880 * 960 * 2
     r, v = _size(lib.aq_conv2d_workspace_size, 16, 64, 64, 192, 192, 3, 3, 1, 1, 8, 4, 8, 0)
     assert r == 0 and v >= 192 * 1728 * 2
+
+
+def test_kernel_aware_grouping_g9(lib):
+    """g = 9 (one group per 3x3 filter): canonical layout stored as is, conv only,
+    dense path only."""
+    r, v = _size(lib.aq_packed_size, 96, 9 * 64, 9, 2, 8)
+    assert r == 0 and v == 96 * 64 * 2
+    r, v = _size(lib.aq_packed_size, 96, 9 * 64, 9, 1, 16)
+    assert r == 0 and v == 96 * 64 * 2
+    assert _size(lib.aq_packed_size, 96, 9 * 64 + 1, 9, 2, 8)[0] == -2          # K % 9
+    # not a linear-layer format
+    assert _size(lib.aq_linear_workspace_size, 128, 576, 64, 9, 2, 8, 0)[0] == -3
+    # conv: AUTO and DENSE run the dense path, FUSED and LUT are refused
+    for path in (0, 1):
+        r, v = _size(lib.aq_conv2d_workspace_size, 2, 16, 16, 64, 96, 3, 3, 1, 1, 9, 2, 8, path)
+        assert r == 0 and v >= 96 * 9 * 64 * 2
+    for path in (2, 3):
+        assert _size(lib.aq_conv2d_workspace_size, 2, 16, 16, 64, 96, 3, 3, 1, 1, 9, 2, 8,
+                     path)[0] == -3
+

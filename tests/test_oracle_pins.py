@@ -386,3 +386,46 @@ def test_breakeven_from_eq_a7():
         assert lut(c_lo) > dense(c_lo)
     assert O.eq_a7_breakeven(2, 8) == 544.0
     assert O.paper_lut_breakeven(2, 8) == pytest.approx(286.875)
+
+
+def _kaq_layer(Nb, H, W, Cin, Cout, M, stride, seed, n_code=16):
+    """A tiny kernel-aware (g = 9) conv layer with a 16-entry codebook."""
+    from aq_synth import ConvSpec
+    rng = np.random.default_rng(seed)
+    spec = ConvSpec(Nb=Nb, H=H, W=W, Cin=Cin, Cout=Cout, stride=stride, g=9, M=M)
+    return dict(codebooks=rng.normal(0, 0.1, size=(M, n_code, 9)).astype(np.float16),
+                codes=rng.integers(0, n_code, size=(Cout, Cin, M), dtype=np.uint8),
+                scale=rng.uniform(0.5, 1.5, size=Cout).astype(np.float16),
+                bias=rng.normal(0, 0.01, size=Cout).astype(np.float16),
+                xq=rng.integers(-127, 128, size=(Nb, H, W, Cin), dtype=np.int8),
+                s_x=0.02, spec=spec)
+
+
+def test_kaq_layer_equals_appendix_lut_kernel():
+    """Sec. 3.1.2 / App. A.1: the kernel-aware conv layer (decode, OHWI layout,
+    direct NHWC conv) equals the appendix's LUT kernel run image by image on the
+    channels-first input, then the per-channel scale and bias."""
+    inp = _kaq_layer(2, 5, 6, 3, 4, 2, 1, seed=91)
+    y = O.layer_f64(inp)
+    for b in range(2):
+        Hc = inp["xq"][b].astype(np.float64).transpose(2, 0, 1) * inp["s_x"]
+        G, _, _ = O.lut_conv_kaq_counted(Hc, inp["codes"], inp["codebooks"])
+        ref = G.transpose(1, 2, 0) * inp["scale"].astype(np.float64) + inp["bias"].astype(np.float64)
+        np.testing.assert_allclose(y[b], ref, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_kaq_layer_equals_torch_conv_on_oihw_filters(stride):
+    """kaq_ohwi is a pure relayout: the NHWC layer equals torch's NCHW conv with
+    the decoded filters F [Cout][Cin][3][3] (float64)."""
+    torch = pytest.importorskip("torch")
+    inp = _kaq_layer(2, 7, 6, 5, 3, 3, stride, seed=92 + stride)
+    y = O.layer_f64(inp)
+    F = O.decode_kaq_f64(inp["codes"], inp["codebooks"]).reshape(3, 5, 3, 3)
+    X = torch.from_numpy(inp["xq"].astype(np.float64).transpose(0, 3, 1, 2) * inp["s_x"])
+    ref = torch.nn.functional.conv2d(X, torch.from_numpy(F), stride=stride, padding=1).numpy()
+    ref = ref.transpose(0, 2, 3, 1) * inp["scale"].astype(np.float64) + inp["bias"].astype(np.float64)
+    np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-12)
+    # and the layout itself: W[n][t*Cin + c] = F[n][c][t]
+    Wm = O.kaq_ohwi(F.reshape(3, 5, 9))
+    assert Wm[2, 7 * 5 + 4] == F.reshape(3, 5, 9)[2, 4, 7]
