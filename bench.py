@@ -17,7 +17,9 @@ the GEMM (quantizer + decode only), replayed in the same timed region.
 `e2e` repeats the step through the C ABI with the input copied from pinned host
 memory and the output copied back every step.  `layers` times the other
 workloads (64x64 W4A8 conv, 8x8 conv with one 2^16-entry codebook) and
-`unet_forward` one UNet-shaped forward (97 AQ layers, batch 2, W2A8 and W4A8).
+`unet_forward` one UNet-shaped forward (97 AQ layers, W2A8 and W4A8, batches 2 and
+16), with each layer preceded by the quantizer, or writing the next layer's int8
+activations from its epilogue.
 
 --impl reference times the CPU oracle (numpy float64) on the headline workload.
 Multi-GPU: independent replicas, one per rank (the layer has no exchange step).
@@ -223,7 +225,9 @@ class Dev:
     """Device copies of one seeded layer plus its output and workspace; step() is one pass
     of the hot path through the C ABI (quantizer, then the layer on the AUTO path)."""
 
-    def __init__(self, aq, torch, inp, dev, path=0):
+    def __init__(self, aq, torch, inp, dev, path=0, xq_dev=None):
+        """xq_dev: int8 activations already on the device (shape of the layer's input),
+        used instead of inp["xq"] for large batches (inp then only supplies weights)."""
         self.aq, self.torch = aq, torch
         s = inp["spec"]
         self.spec = s
@@ -241,17 +245,21 @@ class Dev:
         aq.aq_pack(codes, self.packed, N, K, 8, M, B)
         self.books, self.scale, self.bias = t(inp["codebooks"]), t(inp["scale"]), t(inp["bias"])
         # fp16 activations whose 8-bit quantization with s_x gives the seeded int8 values
-        x16 = (inp["xq"].astype(np.float32) * np.float32(inp["s_x"])).astype(np.float16)
-        self.x16 = t(x16)
-        self.xq = torch.empty(inp["xq"].shape, dtype=torch.int8, device=dev)
+        if xq_dev is None:
+            x16 = (inp["xq"].astype(np.float32) * np.float32(inp["s_x"])).astype(np.float16)
+            self.x16 = t(x16)
+        else:
+            self.x16 = (xq_dev.float() * float(np.float32(inp["s_x"]))).half()
+        self.xq = torch.empty(tuple(self.x16.shape), dtype=torch.int8, device=dev)
         self.s_x = inp["s_x"]
+        self.yq = None
         if self.conv:
             self.T = s.Nb * s.Ho * s.Wo
             self.ws_bytes = aq.aq_conv2d_workspace_size(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
                                                         s.stride, 1, 8, M, B, path)
             self.y = torch.empty((s.Nb, s.Ho, s.Wo, N), dtype=torch.float16, device=dev)
         else:
-            self.T = inp["xq"].shape[0]
+            self.T = self.x16.shape[0]
             self.ws_bytes = aq.aq_linear_workspace_size(self.T, K, N, 8, M, B, path)
             self.y = torch.empty((self.T, N), dtype=torch.float16, device=dev)
         self.ws = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=dev)
@@ -271,6 +279,22 @@ class Dev:
             aq.aq_linear(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias, self.y,
                          aq.AQ_DTYPE_F16, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
                          self.ws_bytes, self.path, stream=st)
+
+    def layer_q8(self, st, s_out=0.02):
+        """The layer with the next layer's quantizer in its epilogue (int8 output)."""
+        aq, s = self.aq, self.spec
+        if self.yq is None:
+            self.yq = self.torch.empty(tuple(self.y.shape), dtype=self.torch.int8,
+                                       device=self.y.device)
+        if self.conv:
+            aq.aq_conv2d_nhwc_q8(self.xq, self.s_x, self.packed, self.books, self.scale,
+                                 self.bias, self.yq, s_out, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
+                                 s.stride, 1, 8, self.M, self.B, self.ws, self.ws_bytes,
+                                 self.path, stream=st)
+        else:
+            aq.aq_linear_q8(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias,
+                            self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
+                            self.ws_bytes, self.path, stream=st)
 
     def decode_only(self, st, wbuf):
         self.aq.aq_decode(self.packed, self.books, wbuf, self.N, self.K, 8, self.M, self.B,
@@ -301,30 +325,59 @@ def replay_ms(torch, stream, g, reps):
     return e0.elapsed_time(e1) / reps
 
 
-def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20):
-    """One UNet-shaped forward: every AQ layer of the LDM-4-like sweep, each preceded by
-    its activation quantization, captured as one graph.  Returns (ms, GFLOP, layers)."""
+def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False):
+    """One UNet-shaped forward: every AQ layer of the LDM-4-like sweep, captured as one
+    graph.  Each layer is preceded by its activation quantizer (aq_quant_act), or, with
+    fused_quant, writes int8 output through its _q8 epilogue instead (the chain of
+    layers then has no separate quantizer pass).  Above batch 2 the int8 activations
+    are drawn on the device (seeded torch generator) and the host arrays only supply
+    the weights.  Returns (ms, GFLOP, layers)."""
     from aq_synth import ConvSpec, LinearSpec, make_conv, make_linear, unet_sweep_layers
     layers = []
     seed = 4000 + 100 * M
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed + batch)
+    big = batch > 2
+
+    def acts(shape):
+        # round(N(0, 40)) clipped to +-127, as the host generator's "normal40"
+        v = torch.randn(shape, generator=gen, device=dev) * 40.0
+        return v.round().clamp_(-127, 127).to(torch.int8)
+
     for kind, res, cin, cout, stride, count in unet_sweep_layers():
         for _ in range(count):
             seed += 1
             if kind == "conv3":
                 spec = ConvSpec(Nb=batch, H=res * stride, W=res * stride, Cin=cin, Cout=cout,
                                 stride=stride, M=M, B=8, cb_std=0.03)
-                layers.append(Dev(aq, torch, make_conv(spec, seed), dev))
+                if big:
+                    wspec = ConvSpec(Nb=1, H=8, W=8, Cin=cin, Cout=cout, M=M, B=8, cb_std=0.03)
+                    inp = dict(make_conv(wspec, seed), spec=spec)
+                    xq = acts((batch, res * stride, res * stride, cin))
+                    layers.append(Dev(aq, torch, inp, dev, xq_dev=xq))
+                else:
+                    layers.append(Dev(aq, torch, make_conv(spec, seed), dev))
             else:
-                spec = LinearSpec(T=batch * res * res, K=cin, N=cout, M=M, B=8, cb_std=0.03,
-                                  act="normal40")
-                layers.append(Dev(aq, torch, make_linear(spec, seed), dev))
+                T = batch * res * res
+                spec = LinearSpec(T=T, K=cin, N=cout, M=M, B=8, cb_std=0.03, act="normal40")
+                if big:
+                    wspec = LinearSpec(T=16, K=cin, N=cout, M=M, B=8, cb_std=0.03, act="normal40")
+                    inp = dict(make_linear(wspec, seed), spec=spec)
+                    layers.append(Dev(aq, torch, inp, dev, xq_dev=acts((T, cin))))
+                else:
+                    layers.append(Dev(aq, torch, make_linear(spec, seed), dev))
     torch.cuda.synchronize()
 
     def fwd():
         for L in layers:
-            L.step(stream)
+            if fused_quant:
+                L.layer_q8(stream)
+            else:
+                L.step(stream)
 
     with torch.cuda.stream(stream):
+        for L in layers:
+            L.quant(stream)          # int8 inputs for the fused-quantizer chain
         for _ in range(2):
             fwd()
     stream.synchronize()
@@ -375,6 +428,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the other workloads and the UNet-shaped forward")
+    ap.add_argument("--unet-batches", default="2,16",
+                    help="batches of the UNet-shaped forward extras (comma separated)")
     ap.add_argument("--workload", default="qkv", choices=["qkv", "conv64", "conv8", "unet"],
                     help="qkv: the headline line (default); the others run only that workload "
                          "and print its timing (for profiling)")
@@ -521,9 +576,16 @@ def main():
             del gl, L
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
-            ms, gflop, nl = unet_forward(aq, torch, dev, stream, Mu)
-            unet[label] = {"ms_per_forward": ms, "gflop": gflop, "tflops": gflop / ms,
-                           "layers": nl, "batch": 2}
+            for batch in [int(b) for b in args.unet_batches.split(",") if b]:
+                for fq in (False, True):
+                    ms, gflop, nl = unet_forward(aq, torch, dev, stream, Mu, batch=batch,
+                                                 reps=20 if batch <= 2 else 5, fused_quant=fq)
+                    key = f"{label} batch {batch}" + (" quantizer in epilogue" if fq else "")
+                    unet[key] = {"ms_per_forward": ms, "gflop": gflop, "tflops": gflop / ms,
+                                 "layers": nl, "batch": batch,
+                                 "step": ("each layer writes the next layer's int8 activations"
+                                          if fq else "each layer preceded by aq_quant_act")}
+                    torch.cuda.empty_cache()
         assert aq.aq_device_error() == 0
 
     if rank == 0:

@@ -66,7 +66,8 @@ extern "C" {
 /* ---- enums --------------------------------------------------------------- */
 typedef enum aq_dtype {
   AQ_DTYPE_F16 = 0,   /* output fp16, round to nearest even */
-  AQ_DTYPE_F32 = 1    /* output fp32                        */
+  AQ_DTYPE_F32 = 1,   /* output fp32                        */
+  AQ_DTYPE_I8 = 2     /* output int8, quantized (the _q8 entry points only) */
 } aq_dtype;
 
 typedef enum aq_path {
@@ -161,6 +162,20 @@ AQ_API int aq_linear(const int8_t* xq, float s_x, const void* codes_packed,
               void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
               void* workspace, size_t workspace_bytes, int path, void* stream);
 
+/* ---- layer with the next layer's activation quantizer fused in ------------
+ * yq[t][n] = clip(round_half_even(fp32(y16[t][n]) / s_out), -127, 127), where
+ * y16 is the fp16 output aq_linear would write: the 8-bit activations of the
+ * next layer (Sec. 4.2.3), produced in the layer's epilogue instead of by a
+ * separate aq_quant_act pass over an fp16 tensor.  Bit-exact against
+ * aq_linear (fp16) followed by aq_quant_act with s_out on the same path.
+ *   yq int8 [T][N]; s_out finite and > 0; N % 16 == 0 (AQ_ERR_SHAPE).
+ *   Workspace: aq_linear_workspace_size() (the same plan as fp16 output).
+ * Other arguments, layouts and errors as for aq_linear.                     */
+AQ_API int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed,
+                        const void* codebooks, const void* scale, const void* bias,
+                        int8_t* yq, float s_out, int T, int K, int N, int g, int M, int B,
+                        void* workspace, size_t workspace_bytes, int path, void* stream);
+
 /* ---- linear layer without any device allocation --------------------------
  * The paper has no counterpart: this is a deployment convenience.  Some callers
  * cannot call cudaMalloc at all (code running under a fixed memory budget that
@@ -207,6 +222,15 @@ AQ_API int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed,
                    void* y, int out_dtype, int Nb, int H, int W, int Cin, int Cout,
                    int kh, int kw, int stride, int pad, int g, int M, int B,
                    void* workspace, size_t workspace_bytes, int path, void* stream);
+
+/* The convolution with the next layer's quantizer fused in (as aq_linear_q8):
+ * yq int8 [Nb][Ho][Wo][Cout], Cout % 16 == 0; workspace as for
+ * aq_conv2d_workspace_size().                                                */
+AQ_API int aq_conv2d_nhwc_q8(const int8_t* xq, float s_x, const void* codes_packed,
+                             const void* codebooks, const void* scale, const void* bias,
+                             int8_t* yq, float s_out, int Nb, int H, int W, int Cin, int Cout,
+                             int kh, int kw, int stride, int pad, int g, int M, int B,
+                             void* workspace, size_t workspace_bytes, int path, void* stream);
 
 #ifdef __cplusplus
 }

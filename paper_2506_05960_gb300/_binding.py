@@ -14,7 +14,7 @@ import os
 _PKG = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_PKG, "lib", "libaq_gb300.so")
 
-AQ_DTYPE_F16, AQ_DTYPE_F32 = 0, 1
+AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_DTYPE_I8 = 0, 1, 2
 AQ_PATH_AUTO, AQ_PATH_DENSE, AQ_PATH_FUSED, AQ_PATH_LUT = 0, 1, 2, 3
 
 _ERRORS = {
@@ -42,9 +42,13 @@ _SIGNATURES = {
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_linear_noalloc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                           + [_c_void_p]),
+    "aq_linear_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float] + [_c_int] * 6
+                     + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
     "aq_conv2d_nhwc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_conv2d_nhwc_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float]
+                          + [_c_int] * 12 + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
 }
 
 _lib = None
@@ -172,6 +176,15 @@ def aq_linear(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K,
         _stream(stream)), "aq_linear")
 
 
+def aq_linear_q8(xq, s_x, codes_packed, codebooks, scale, bias, yq, s_out, T, K, N, g=8, M=2,
+                 B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """aq_linear whose epilogue writes the next layer's int8 activations (scale s_out)."""
+    _check(load_library().aq_linear_q8(
+        _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(yq), float(s_out), T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
+        _stream(stream)), "aq_linear_q8")
+
+
 def aq_linear_noalloc(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N,
                       g=8, M=2, B=8, stream=None) -> None:
     """aq_linear with the library's fixed device scratch instead of a caller workspace."""
@@ -196,3 +209,14 @@ def aq_conv2d_nhwc(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 
         _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
         _ptr(y), out_dtype, Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, _ptr(workspace),
         int(workspace_bytes), path, _stream(stream)), "aq_conv2d_nhwc")
+
+
+def aq_conv2d_nhwc_q8(xq, s_x, codes_packed, codebooks, scale, bias, yq, s_out, Nb, H, W, Cin,
+                      Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8, workspace=None,
+                      workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """aq_conv2d_nhwc whose epilogue writes the next layer's int8 activations (scale s_out)."""
+    _check(load_library().aq_conv2d_nhwc_q8(
+        _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(yq), float(s_out), Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B,
+        _ptr(workspace), int(workspace_bytes), path, _stream(stream)), "aq_conv2d_nhwc_q8")
+

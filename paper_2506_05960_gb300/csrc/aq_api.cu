@@ -477,6 +477,12 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
     cuuint32_t box[3] = {32, 32, 1};
     r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, p.partial, dims, strides, box,
                CU_TENSOR_MAP_SWIZZLE_128B);
+  } else if (p.out_q8) {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(N)};
+    cuuint32_t box[2] = {32, 32};
+    r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, p.y, dims, strides, box,
+               CU_TENSOR_MAP_SWIZZLE_NONE);
   } else if (p.out_f32) {
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(N) * 4};
@@ -552,6 +558,30 @@ int encode_linear_a(CUtensorMap* mapA, const int8_t* xq, int T, int K) {
   return encode(mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, xq, dims, strides, box,
                 CU_TENSOR_MAP_SWIZZLE_64B);
 }
+
+// Output kinds of the layer entry points: AQ_DTYPE_F16 / AQ_DTYPE_F32 through
+// aq_linear / aq_conv2d_nhwc, AQ_DTYPE_I8 (quantized with s_out) through the _q8
+// variants.  int8 rows need N % 16 == 0 (16-byte TMA row stride).
+int check_output(int out_dtype, float s_out, int N) {
+  if (out_dtype == AQ_DTYPE_I8) {
+    if (!(s_out > 0.0f) || s_out == __builtin_inff())
+      return set_error(AQ_ERR_SHAPE, "s_out must be finite and > 0");
+    if (N % 16 != 0) return set_error(AQ_ERR_SHAPE, "int8 output needs N %% 16 == 0");
+    return AQ_OK;
+  }
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  return AQ_OK;
+}
+
+int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+                const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
+                int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
+                int path, void* stream);
+int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+              const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
+              int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
+              int B, void* workspace, size_t workspace_bytes, int path, void* stream);
 
 }  // namespace
 
@@ -678,12 +708,33 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
               const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
               int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
               void* stream) {
+  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  return linear_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, T, K, N,
+                     g, M, B, workspace, workspace_bytes, path, stream);
+}
+
+int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+                 const void* scale, const void* bias, int8_t* yq, float s_out, int T, int K,
+                 int N, int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
+                 void* stream) {
+  return linear_impl(xq, s_x, codes_packed, codebooks, scale, bias, yq, AQ_DTYPE_I8, s_out, T, K,
+                     N, g, M, B, workspace, workspace_bytes, path, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+                const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
+                int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
+                int path, void* stream) {
   int r = check_format(g, M, B);
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
-    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  r = check_output(out_dtype, s_out, N);
+  if (r) return r;
   if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite");
   const int rp = resolve_linear_path(path, T, B);
@@ -727,6 +778,8 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
     rpar.bias = static_cast<const __half*>(bias);
     rpar.y = y;
     rpar.out_f32 = out_dtype == AQ_DTYPE_F32;
+    rpar.out_q8 = out_dtype == AQ_DTYPE_I8;
+    rpar.s_out = s_out;
     rpar.partial = lpar.partial;
     {
       ProfScope ps(kProfSplitK, st);
@@ -756,8 +809,14 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  p.out_q8 = out_dtype == AQ_DTYPE_I8;
+  p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st);
 }
+
+}  // namespace
+
+extern "C" {
 
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
                              int pad, int g, int M, int B, int path, size_t* bytes) {
@@ -781,12 +840,37 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
                    const void* scale, const void* bias, void* y, int out_dtype, int Nb, int H,
                    int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
                    int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
+  if (out_dtype == AQ_DTYPE_I8)
+    return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_conv2d_nhwc_q8");
+  return conv_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, Nb, H, W,
+                   Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes, path,
+                   stream);
+}
+
+int aq_conv2d_nhwc_q8(const int8_t* xq, float s_x, const void* codes_packed,
+                      const void* codebooks, const void* scale, const void* bias, int8_t* yq,
+                      float s_out, int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
+                      int stride, int pad, int g, int M, int B, void* workspace,
+                      size_t workspace_bytes, int path, void* stream) {
+  return conv_impl(xq, s_x, codes_packed, codebooks, scale, bias, yq, AQ_DTYPE_I8, s_out, Nb, H,
+                   W, Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes, path,
+                   stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
+              const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
+              int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
+              int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
   int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
   if (r) return r;
-  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
-    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  r = check_output(out_dtype, s_out, Cout);
+  if (r) return r;
   if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite");
   ConvGeom cg;
@@ -838,11 +922,13 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  p.out_q8 = out_dtype == AQ_DTYPE_I8;
+  p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st,
                   g == kKaqGroup);
 }
 
-}  // extern "C"
+}  // namespace
 
 // Device address of g_noalloc_scratch on the current device, looked up once per
 // device (the host-side symbol is only a stand-in, never a device address).

@@ -9,26 +9,11 @@
 
 #include "aq_internal.h"
 #include "aq_ptx.cuh"
+#include "aq_quant.cuh"
 
 namespace aq {
 
-// ============================================================== quantizer
-// x / s in IEEE fp32, round half to even, NaN -> 0, clip to [-127, 127].
-// Fast path: q = x * fl(1/s) lies within 3 * 2^-24 * |x/s| of fl(x/s); for
-// |x/s| < 128 that is < 2.3e-5, so unless q is within 1e-4 of a half-integer
-// both round to the same integer (and for |x/s| >= 128 both clip to the same
-// end).  Near a tie, and for NaN/inf, the exact IEEE quotient decides.
-__device__ __forceinline__ int8_t quant_one(__half h, float s, float rs) {
-  const float x = __half2float(h);
-  float q = x * rs;
-  const float fr = q - floorf(q);
-  if (!(fabsf(fr - 0.5f) > 1e-4f)) q = __fdiv_rn(x, s);
-  q = rintf(q);
-  if (q != q) q = 0.0f;
-  q = fminf(fmaxf(q, -127.0f), 127.0f);
-  return static_cast<int8_t>(static_cast<int>(q));
-}
-
+// ============================================================== quantizer (rule in aq_quant.cuh)
 // Each thread: 16 elements (32 B in, 16 B out) per grid-stride step.
 __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
                                                         int8_t* __restrict__ xq,

@@ -18,7 +18,9 @@
 //   warps 2..5  converters: int8 rows -> fp16 exactly -> tcgen05.st into a
 //               TMEM A ring (no shared-memory round trip for the fp16 operand)
 //   warps 6..9  epilogue: TMEM accumulator -> scale/bias -> 32 x 32 boxes in
-//               shared memory -> TMA stores (ragged edges clipped by TMA)
+//               shared memory -> TMA stores (ragged edges clipped by TMA).  The
+//               output is fp16, fp32, or int8: the fp16 value quantized with the
+//               next layer's activation scale (the quantizer fused into the layer)
 // The fp32 accumulator is double-buffered in TMEM so the epilogue of one tile
 // runs under the mainloop of the next.  The issue loop carries no divisions:
 // ring index and phase advance by counters.  Every wait is bounded (about 2 s);
@@ -31,6 +33,7 @@
 
 #include "aq_internal.h"
 #include "aq_ptx.cuh"
+#include "aq_quant.cuh"
 
 namespace aq {
 
@@ -498,6 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* wbias = wscale + kMaxBN;
     uint8_t* wbuf = epi + ew * 2 * epi_buf;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    const float rs_out = p.out_q8 ? __frcp_rn(p.s_out) : 0.0f;
     uint32_t lt = 0, chunk = 0;
     for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
       const TileCoord tc = tile_coord(p, t);
@@ -550,6 +554,37 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             *reinterpret_cast<float4*>(dst + lane * 128 + ((j ^ (lane & 7)) << 4)) = o;
           }
+        } else if (p.out_q8) {
+          // fp16 value of the output (as a separate quantizer would read it), then
+          // the 8-bit activation rule with the next layer's scale: 32 bytes per row.
+          // The fast path covers all but values near a rounding tie (rare): those
+          // are redone with the exact quotient.
+          uint32_t wq[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
+            const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
+            __half hv[4];
+            hv[0] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 0]), sc.x, bi.x));
+            hv[1] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 1]), sc.y, bi.y));
+            hv[2] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 2]), sc.z, bi.z));
+            hv[3] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 3]), sc.w, bi.w));
+            int qv[4];
+            bool fast = true;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) fast &= quant_fast(hv[e], rs_out, qv[e]);
+            if (!fast) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) qv[e] = quant_one(hv[e], p.s_out, rs_out);
+            }
+            wq[j] = (static_cast<uint32_t>(qv[0]) & 0xFFu) |
+                    ((static_cast<uint32_t>(qv[1]) & 0xFFu) << 8) |
+                    ((static_cast<uint32_t>(qv[2]) & 0xFFu) << 16) |
+                    (static_cast<uint32_t>(qv[3]) << 24);
+          }
+          uint4* row = reinterpret_cast<uint4*>(dst + lane * 32);
+          row[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+          row[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
         } else {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
@@ -668,6 +703,14 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
     if (p.out_f32) {
       *reinterpret_cast<float4*>(static_cast<float*>(p.y) + t * p.N + n) =
           make_float4(o[0], o[1], o[2], o[3]);
+    } else if (p.out_q8) {
+      const float rs = __frcp_rn(p.s_out);
+      uint32_t b = 0;
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        b |= static_cast<uint32_t>(static_cast<uint8_t>(quant_one(__float2half_rn(o[e]), p.s_out, rs)))
+             << (8 * e);
+      *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(p.y) + t * p.N + n) = b;
     } else {
       __half2 a = __floats2half2_rn(o[0], o[1]);
       __half2 b = __floats2half2_rn(o[2], o[3]);

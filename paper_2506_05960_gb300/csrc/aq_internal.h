@@ -35,6 +35,8 @@ struct GemmParams {
   const __half* bias;           // may be null
   void* y;
   int out_f32;
+  int out_q8;                   // int8 output: the next layer's activations, quantized with s_out
+  float s_out;
   float* partial;               // split-K partial sums [splits][T][N] (null: fused epilogue)
   // fused decode (B stages written by decoder warps instead of TMA from a decoded W)
   int fused;
