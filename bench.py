@@ -574,6 +574,30 @@ def main():
                             "tensor_roofline_frac": L.flops / (peaks["bf16_tflops"] * 1e12) / (ms * 1e-3),
                             "step": "quantizer + layer (AUTO path), CUDA graph replay"}
             del gl, L
+        # backward of Eq. 4 (codebook gradient) on the headline layer: HBM-bound read of G
+        gsets = []
+        for i in range(NSETS):
+            gsets.append(torch.randn((N, K), dtype=torch.float32, device=dev,
+                                     generator=torch.Generator(device=dev).manual_seed(i)))
+        dC = torch.zeros((M, 1 << B, g), dtype=torch.float32, device=dev)
+        gb = bufs[0]
+
+        def cgrad():
+            for G in gsets:
+                aq.aq_codebook_grad(gb.packed, G, gb.scale, gb.s_x, dC, N, K, g, M, B,
+                                    stream=stream)
+        with torch.cuda.stream(stream):
+            cgrad()
+        stream.synchronize()
+        gc = capture(torch, stream, cgrad)
+        ms = replay_ms(torch, stream, gc, 20) / NSETS
+        cg_bytes = N * K * 4 + aq.aq_packed_size(N, K, g, M, B) + 2 * N + M * (1 << B) * g * 4
+        layers["codebook gradient of the qkv layer (fp32 G, 2x8)"] = {
+            "us_per_step": ms * 1e3, "gbs": cg_bytes / (ms * 1e-3) / 1e9,
+            "hbm_roofline_frac": cg_bytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "bytes_per_call": cg_bytes,
+            "step": "aq_codebook_grad, 8 rotating G buffers (> L2), CUDA graph replay"}
+        del gc, gsets
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
             for batch in [int(b) for b in args.unet_batches.split(",") if b]:

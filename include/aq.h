@@ -138,6 +138,22 @@ AQ_API int aq_pack(const void* codes_canon, void* codes_packed,
 AQ_API int aq_decode(const void* codes_packed, const void* codebooks, void* W_out,
               int N, int K, int g, int M, int B, void* stream);
 
+/* ---- codebook gradient (backward of Eq. 4; Sec. 3.2.1 continuous step) -----
+ * The decoded group is the sum of its M codewords, so the gradient of a loss L
+ * with respect to codeword row c of codebook m collects every group that uses
+ * it:  dC[m][c][e] += sum_{(n, i): b[n, i, m] = c}  s_x * scale[n] * G[n][i*g + e]
+ * where G[n][k] = dL/dW[n][k] for the unscaled decoded weight, i.e.
+ * sum_t dY[t][n] * xq[t][k] (a plain GEMM of the output gradient and the
+ * layer's int8 input, run by the caller).  g = 9: G is in the convolution's OHWI
+ * order (element e of the (n, c) filter at column e*Cin + c).
+ *   codes_packed  as for aq_decode;  G fp32 [N][K];  scale fp16 [N] or NULL (1);
+ *   dC fp32 [M][2^B][g], ACCUMULATED (clear it first for a plain gradient).
+ * Summation order is not fixed (atomic adds): results match the exact sum to
+ * fp32 accumulation error, not bit for bit.                                    */
+AQ_API int aq_codebook_grad(const void* codes_packed, const float* G, const void* scale,
+                            float s_x, float* dC, int N, int K, int g, int M, int B,
+                            void* stream);
+
 /* ---- 8-bit activation quantizer (Sec. 4.2.3; symmetric form of Eq. 3) ------
  * xq[i] = clip(round_half_even(x[i] / s_x), -127, 127), x fp16, division in
  * IEEE fp32, NaN -> 0.  s_x must be finite and > 0 (AQ_ERR_SHAPE otherwise).

@@ -30,7 +30,8 @@ import math
 import numpy as np
 
 __all__ = [
-    "decode_f64", "decode_rule_f16", "decode_kaq_f64", "kaq_ohwi", "pack_codes", "packed_nbytes",
+    "decode_f64", "decode_rule_f16", "decode_kaq_f64", "kaq_ohwi", "kaq_from_ohwi",
+    "codebook_grad_f64", "pack_codes", "packed_nbytes",
     "quant_act", "linear_f64", "conv2d_nhwc_f64", "lut_linear_f64",
     "lut_conv_kaq_counted", "direct_conv_counted", "eq_a7_flops", "eq_a2_flops",
     "paper_lut_breakeven", "eq_a7_breakeven", "bits_per_weight",
@@ -101,6 +102,35 @@ def kaq_ohwi(F: np.ndarray) -> np.ndarray:
     index k = t*Cin + c for tap t and input channel c."""
     Cout, Cin, taps = F.shape
     return np.ascontiguousarray(F.transpose(0, 2, 1)).reshape(Cout, taps * Cin)
+
+
+def kaq_from_ohwi(W: np.ndarray, taps: int = 9) -> np.ndarray:
+    """Layout only, the inverse of ``kaq_ohwi``: [Cout][taps*Cin] (k = t*Cin + c)
+    -> [Cout][Cin][taps]."""
+    Cout, K = W.shape
+    Cin = K // taps
+    return np.ascontiguousarray(W.reshape(Cout, taps, Cin).transpose(0, 2, 1))
+
+
+def codebook_grad_f64(codes: np.ndarray, G: np.ndarray, scale: np.ndarray | None, s_x: float,
+                      n_code: int) -> np.ndarray:
+    """Backward of Eq. 4 with respect to the codebooks (the continuous step of
+    Stage-2 fine-tuning, Sec. 3.2.1), float64.
+
+    codes [N][Gr][M]; G [N][Gr*g] = dL/dW for the unscaled decoded weight, group i
+    of row n at columns i*g .. i*g+g-1 (pass ``kaq_from_ohwi(G).reshape(N, -1)`` for
+    the kernel-aware grouping).  The layer multiplies row n by s_x*scale[n], so
+      dC[m][c][e] = sum over (n, i) with codes[n, i, m] == c of s_x*scale[n]*G[n][i*g+e].
+    Returns dC [M][n_code][g].
+    """
+    N, Gr, M = codes.shape
+    g = G.shape[1] // Gr
+    f = float(s_x) * (scale.astype(np.float64) if scale is not None else np.ones(N))
+    Gs = (G.astype(np.float64) * f[:, None]).reshape(N * Gr, g)
+    dC = np.zeros((M, n_code, g), dtype=np.float64)
+    for m in range(M):
+        np.add.at(dC[m], codes[:, :, m].reshape(-1).astype(np.int64), Gs)
+    return dC
 
 
 # --------------------------------------------------------------------------- packing

@@ -37,6 +37,8 @@ _SIGNATURES = {
     "aq_pack": (_c_int, [_c_void_p, _c_void_p] + [_c_int] * 5 + [_c_void_p]),
     "aq_decode": (_c_int, [_c_void_p] * 3 + [_c_int] * 5 + [_c_void_p]),
     "aq_quant_act": (_c_int, [_c_void_p, _c_void_p, _c_int64, _c_float, _c_void_p]),
+    "aq_codebook_grad": (_c_int, [_c_void_p] * 3 + [_c_float, _c_void_p] + [_c_int] * 5
+                         + [_c_void_p]),
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
@@ -159,6 +161,13 @@ def aq_decode(codes_packed, codebooks, W_out, N, K, g=8, M=2, B=8, stream=None) 
 def aq_quant_act(x, xq, numel, s_x, stream=None) -> None:
     _check(load_library().aq_quant_act(_ptr(x), _ptr(xq), int(numel), float(s_x),
                                        _stream(stream)), "aq_quant_act")
+
+
+def aq_codebook_grad(codes_packed, G, scale, s_x, dC, N, K, g=8, M=2, B=8, stream=None) -> None:
+    """dC += the codebook gradient of the groups' codewords (dC accumulates)."""
+    _check(load_library().aq_codebook_grad(
+        _ptr(codes_packed), _ptr(G), _ptr(scale), float(s_x), _ptr(dC), N, K, g, M, B,
+        _stream(stream)), "aq_codebook_grad")
 
 
 def aq_linear_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:

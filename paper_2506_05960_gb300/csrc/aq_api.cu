@@ -676,6 +676,22 @@ int aq_decode(const void* codes_packed, const void* codebooks, void* W_out, int 
                      "aq_decode launch");
 }
 
+int aq_codebook_grad(const void* codes_packed, const float* G, const void* scale, float s_x,
+                     float* dC, int N, int K, int g, int M, int B, void* stream) {
+  int r = check_format(g, M, B, true);
+  if (r) return r;
+  if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
+  if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite");
+  if (!codes_packed || !G || !dC) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(codes_packed) || !aligned16(G) || !aligned16(dC) || (scale && !aligned16(scale)))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return cuda_status(aq::launch_codebook_grad(codes_packed, G, static_cast<const __half*>(scale),
+                                              s_x, dC, N, K, g, M, B, st),
+                     "aq_codebook_grad launch");
+}
+
 int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stream) {
   if (numel < 0) return set_error(AQ_ERR_SHAPE, "numel < 0");
   if (!(s_x > 0.0f) || s_x == __builtin_inff())

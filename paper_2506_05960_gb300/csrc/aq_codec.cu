@@ -259,4 +259,134 @@ cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int
                     b, w, N, Cin, M);
 }
 
+// ============================================================== codebook gradient
+// Backward of Eq. 4 for the continuous (codebook) step of Stage-2 fine-tuning
+// (Sec. 3.2.1, PV-Tuning): the decoded group is sum_m C^(m)[b_m], so
+//   dL/dC^(m)[c][e] = sum over groups (n, i) with b[n][i][m] = c of
+//                     s_x * scale[n] * G[n][i*g + e],
+// where G[n][k] = sum_t dY[t][n] * xq[t][k] is the gradient with respect to the
+// unscaled weight (a plain GEMM the caller runs).  dC is accumulated (+=) in fp32:
+// 8-bit codebooks in shared memory per CTA, flushed with global atomics; 16-bit
+// codebooks with global atomics directly.  One thread per group; g = 8 reads the
+// packed layout, g = 9 (one group per 3x3 filter) the canonical [N][Cin][M] codes
+// with G in the convolution's OHWI order.
+template <int EB, bool kKaq>
+__global__ void __launch_bounds__(256) codebook_grad_kernel(
+    const uint8_t* __restrict__ codes, const float* __restrict__ G,
+    const __half* __restrict__ scale, float s_x, float* __restrict__ dC, int N, int K, int M,
+    int KB) {
+  constexpr int g = kKaq ? 9 : 8;
+  // 8-bit codes: the CTA's table in shared memory, element-major [g][M*256] so that
+  // the adds of a warp (random codewords, same element) spread over all banks
+  extern __shared__ float sdc[];
+  grid_dependency_wait();
+  allow_dependents();
+  if constexpr (EB == 1) {
+    for (int i = threadIdx.x; i < M * 256 * g; i += blockDim.x) sdc[i] = 0.0f;
+    __syncthreads();
+  }
+  const int Cin = K / 9;
+  const int64_t total = kKaq ? static_cast<int64_t>(N) * Cin : static_cast<int64_t>(KB) * N * 8;
+  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    int n, col0, colstep;
+    if constexpr (kKaq) {
+      n = static_cast<int>(idx / Cin);
+      const int c = static_cast<int>(idx - static_cast<int64_t>(n) * Cin);
+      col0 = c;
+      colstep = Cin;                                    // tap t at t*Cin + c
+    } else {
+      const int j = static_cast<int>(idx & 7);
+      const int64_t r = idx >> 3;
+      const int kb = static_cast<int>(r / N);
+      n = static_cast<int>(r - static_cast<int64_t>(kb) * N);
+      col0 = (kb * 8 + j) * 8;
+      colstep = 1;
+      if (col0 >= K) continue;                          // zero-padded K tail
+    }
+    const float f = s_x * (scale ? __half2float(scale[n]) : 1.0f);
+    const float* grow = G + static_cast<int64_t>(n) * K + col0;
+    float v[g];
+    if constexpr (kKaq) {
+#pragma unroll
+      for (int e = 0; e < g; ++e) v[e] = f * __ldg(grow + static_cast<int64_t>(e) * colstep);
+    } else {
+      // 8 consecutive floats of the row (32-byte aligned: K % 8 == 0, G 16-byte aligned)
+      const float4 a = __ldg(reinterpret_cast<const float4*>(grow));
+      const float4 b = __ldg(reinterpret_cast<const float4*>(grow) + 1);
+      v[0] = f * a.x; v[1] = f * a.y; v[2] = f * a.z; v[3] = f * a.w;
+      v[4] = f * b.x; v[5] = f * b.y; v[6] = f * b.z; v[7] = f * b.w;
+    }
+    for (int m = 0; m < M; ++m) {
+      const int c = EB == 1 ? codes[idx * M + m]
+                            : reinterpret_cast<const uint16_t*>(codes)[idx * M + m];
+      if constexpr (EB == 1) {
+        float* dst = sdc + m * 256 + c;
+#pragma unroll
+        for (int e = 0; e < g; ++e) atomicAdd(dst + e * (M * 256), v[e]);
+      } else {
+        float* dst = dC + ((static_cast<int64_t>(m) << 16) + c) * g;
+#pragma unroll
+        for (int e = 0; e < g; ++e) atomicAdd(dst + e, v[e]);
+      }
+    }
+  }
+  if constexpr (EB == 1) {
+    // flush: dC[m][c][e] += table[e][m*256 + c], 4 consecutive entries per vector atomic
+    // (M*256*g is a multiple of 4; dC is 16-byte aligned)
+    __syncthreads();
+    for (int i = threadIdx.x; i < M * 256 * g / 4; i += blockDim.x) {
+      float w[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int lin = 4 * i + u;                      // = (m*256 + c)*g + e
+        const int mc = lin / g;
+        w[u] = sdc[(lin - mc * g) * (M * 256) + mc];
+      }
+      if (w[0] != 0.0f || w[1] != 0.0f || w[2] != 0.0f || w[3] != 0.0f)
+        asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dC + 4 * i),
+                     "f"(w[0]), "f"(w[1]), "f"(w[2]), "f"(w[3])
+                     : "memory");
+    }
+  }
+}
+
+cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half* scale,
+                                 float s_x, float* dC, int N, int K, int g, int M, int B,
+                                 cudaStream_t st) {
+  const bool kaq = g == 9;
+  const int KB = (K + 63) / 64;
+  const int64_t total = kaq ? static_cast<int64_t>(N) * (K / 9) : static_cast<int64_t>(KB) * N * 8;
+  int64_t blocks = (total + 255) / 256;
+  // 8-bit: two blocks per SM, each flushes its table once (more threads per SM only
+  // add shared-memory atomic contention)
+  const int64_t cap = B == 8 ? 152 * 2 : 152 * 8;
+  const int threads = 256;
+  blocks = (total + threads - 1) / threads;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  const dim3 grid(static_cast<unsigned>(blocks)), block(static_cast<unsigned>(threads));
+  const uint8_t* c = static_cast<const uint8_t*>(codes);
+  const size_t smem = B == 8 ? static_cast<size_t>(M) * 256 * g * 4 : 0;
+  if (B == 8) {
+    if (kaq) {
+      if (smem > 48 * 1024)
+        cudaFuncSetAttribute(codebook_grad_kernel<1, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      return launch_pdl(codebook_grad_kernel<1, true>, grid, block, smem, st, c, G, scale, s_x, dC,
+                        N, K, M, KB);
+    }
+    if (smem > 48 * 1024)
+      cudaFuncSetAttribute(codebook_grad_kernel<1, false>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    return launch_pdl(codebook_grad_kernel<1, false>, grid, block, smem, st, c, G, scale, s_x, dC,
+                      N, K, M, KB);
+  }
+  if (kaq)
+    return launch_pdl(codebook_grad_kernel<2, true>, grid, block, 0, st, c, G, scale, s_x, dC, N,
+                      K, M, KB);
+  return launch_pdl(codebook_grad_kernel<2, false>, grid, block, 0, st, c, G, scale, s_x, dC, N,
+                    K, M, KB);
+}
+
 }  // namespace aq

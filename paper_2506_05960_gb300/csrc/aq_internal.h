@@ -83,6 +83,10 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
+// dC[m][c][e] += sum over groups with code c of s_x*scale[n]*G[n][group element e]
+cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half* scale,
+                                 float s_x, float* dC, int N, int K, int g, int M, int B,
+                                 cudaStream_t st);
 // Kernel-aware grouping (g = 9, 3x3 conv): codes [N][Cin][M], books [M][2^B][9] ->
 // W [N][9*Cin] in the convolution's OHWI K order.
 cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int N, int Cin, int M,

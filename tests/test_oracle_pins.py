@@ -429,3 +429,53 @@ def test_kaq_layer_equals_torch_conv_on_oihw_filters(stride):
     # and the layout itself: W[n][t*Cin + c] = F[n][c][t]
     Wm = O.kaq_ohwi(F.reshape(3, 5, 9))
     assert Wm[2, 7 * 5 + 4] == F.reshape(3, 5, 9)[2, 4, 7]
+
+
+# ----------------------------------------------------------------------------- codebook gradient
+def test_codebook_grad_brute_force():
+    """Backward of Eq. 4: every use of codeword c in codebook m adds its group's gradient."""
+    rng = np.random.default_rng(31)
+    N, Gr, M, n_code, g = 3, 4, 2, 5, 8
+    codes = rng.integers(0, n_code, size=(N, Gr, M), dtype=np.uint8)
+    G = rng.normal(size=(N, Gr * g))
+    scale = rng.uniform(0.5, 1.5, size=N).astype(np.float16)
+    dC = O.codebook_grad_f64(codes, G, scale, 0.25, n_code)
+    ref = np.zeros((M, n_code, g))
+    for n in range(N):
+        for i in range(Gr):
+            for m in range(M):
+                for e in range(g):
+                    ref[m, codes[n, i, m], e] += 0.25 * float(scale[n]) * G[n, i * g + e]
+    np.testing.assert_allclose(dC, ref, rtol=1e-14, atol=1e-14)
+
+
+@pytest.mark.parametrize("kaq", [False, True])
+def test_codebook_grad_is_the_derivative_of_the_decoded_layer(kaq):
+    """The layer's weight term L(C) = sum_{n,k} s_x*scale[n]*G[n][k]*W-hat[n][k] is
+    linear in the codebooks, so a unit step of codeword entry (m, c, e) changes L
+    by exactly dC[m][c][e] (small integers keep float64 exact)."""
+    rng = np.random.default_rng(32 + kaq)
+    N, M, n_code = 3, 2, 4
+    g, Gr = (9, 5) if kaq else (8, 3)
+    books = rng.integers(-3, 4, size=(M, n_code, g)).astype(np.float64)
+    codes = rng.integers(0, n_code, size=(N, Gr, M), dtype=np.uint8)
+    scale = np.array([1.0, 0.5, 2.0], dtype=np.float16)
+    s_x = 0.25
+    if kaq:
+        decode = lambda C: O.kaq_ohwi(O.decode_kaq_f64(codes, C))      # [N][9*Cin], OHWI
+    else:
+        decode = lambda C: O.decode_f64(codes, C)
+    G = rng.integers(-4, 5, size=(N, Gr * g)).astype(np.float64)      # in decode's column order
+    L = lambda C: float(np.sum(s_x * scale.astype(np.float64)[:, None] * G * decode(C)))
+    Gf = O.kaq_from_ohwi(G).reshape(N, -1) if kaq else G
+    dC = O.codebook_grad_f64(codes, Gf, scale, s_x, n_code)
+    base = L(books)
+    for m in range(M):
+        for c in range(n_code):
+            for e in range(g):
+                C1 = books.copy()
+                C1[m, c, e] += 1.0
+                assert L(C1) - base == dC[m, c, e]
+    assert np.array_equal(O.kaq_from_ohwi(O.kaq_ohwi(books[:, :, :9].reshape(2, 4, 9)
+                                                      if kaq else np.zeros((1, 1, 9)))),
+                          books[:, :, :9].reshape(2, 4, 9) if kaq else np.zeros((1, 1, 9)))
