@@ -598,6 +598,31 @@ def main():
             "bytes_per_call": cg_bytes,
             "step": "aq_codebook_grad, 8 rotating G buffers (> L2), CUDA graph replay"}
         del gc, gsets
+        # Stage-1 code search (one greedy step over both codebooks) on the qkv layer
+        from aq_synth import make_linear as _ml
+        inp1 = _ml(CONFIGS[1], seed=1)
+        Wt = torch.from_numpy(np.ascontiguousarray(
+            (inp1["codebooks"].astype(np.float32)[0][inp1["codes"][:, :, 0]]
+             + inp1["codebooks"].astype(np.float32)[1][inp1["codes"][:, :, 1]]).reshape(N, K)
+            + np.float32(0.01))).to(dev)
+        books_cs = torch.from_numpy(inp1["codebooks"]).to(dev)
+        codes_cs = torch.from_numpy(np.ascontiguousarray(inp1["codes"])).to(dev)
+        Hb = torch.eye(8, device=dev).expand(K // 8, 8, 8).contiguous()
+        for weighted in (False, True):
+            def cs():
+                aq.aq_code_update(Wt, books_cs, codes_cs, Hb if weighted else None, 0, M, N, K,
+                                  8, M, 8, stream=stream)
+            with torch.cuda.stream(stream):
+                cs()
+            stream.synchronize()
+            gcs = capture(torch, stream, cs)
+            ms = replay_ms(torch, stream, gcs, 10)
+            cand = N * (K // 8) * M * 256
+            layers["code search step of the qkv layer (2x8, " + ("H-weighted" if weighted
+                                                                 else "unweighted") + ")"] = {
+                "us_per_step": ms * 1e3, "candidates_per_s": cand / (ms * 1e-3),
+                "step": "aq_code_update over both codebooks, CUDA graph replay"}
+            del gcs
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
             for batch in [int(b) for b in args.unet_batches.split(",") if b]:

@@ -154,6 +154,23 @@ AQ_API int aq_codebook_grad(const void* codes_packed, const float* G, const void
                             float s_x, float* dC, int N, int K, int g, int M, int B,
                             void* stream);
 
+/* ---- code search step (Stage-1 calibration, Sec. 3.1) ---------------------
+ * One greedy step of the code optimisation (beam width 1): for every group and
+ * each codebook m in [m_first, m_first + m_count), in that order, b[m] becomes
+ * the codeword that minimises the group's error with the other codes fixed:
+ *   r = w - sum_{m' != m} C^(m')[b[m']] (ascending m'),  d = C^(m)[c] - r,
+ *   score(c) = d^T H_i d,  ties to the lowest c,
+ * where H_i is group column i's g x g block of A A^T for calibration inputs A
+ * (the block-diagonal part of ||W A - W-hat A||^2), or the identity when H is
+ * NULL.  Computed in fp32, every product and sum rounded separately, sums in
+ * ascending element order; the result is bit-exact against that rule.
+ *   W fp32 [N][K] target weight;  codebooks fp16 [M][256][8];
+ *   codes uint8 CANONICAL [N][K/8][M], read and updated in place;
+ *   H fp32 [K/8][8][8] or NULL.  g = 8 and B = 8 only.                     */
+AQ_API int aq_code_update(const float* W, const void* codebooks, void* codes, const float* H,
+                          int m_first, int m_count, int N, int K, int g, int M, int B,
+                          void* stream);
+
 /* ---- 8-bit activation quantizer (Sec. 4.2.3; symmetric form of Eq. 3) ------
  * xq[i] = clip(round_half_even(x[i] / s_x), -127, 127), x fp16, division in
  * IEEE fp32, NaN -> 0.  s_x must be finite and > 0 (AQ_ERR_SHAPE otherwise).

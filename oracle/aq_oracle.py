@@ -31,7 +31,7 @@ import numpy as np
 
 __all__ = [
     "decode_f64", "decode_rule_f16", "decode_kaq_f64", "kaq_ohwi", "kaq_from_ohwi",
-    "codebook_grad_f64", "pack_codes", "packed_nbytes",
+    "codebook_grad_f64", "code_update_f32", "pack_codes", "packed_nbytes",
     "quant_act", "linear_f64", "conv2d_nhwc_f64", "lut_linear_f64",
     "lut_conv_kaq_counted", "direct_conv_counted", "eq_a7_flops", "eq_a2_flops",
     "paper_lut_breakeven", "eq_a7_breakeven", "bits_per_weight",
@@ -131,6 +131,51 @@ def codebook_grad_f64(codes: np.ndarray, G: np.ndarray, scale: np.ndarray | None
     for m in range(M):
         np.add.at(dC[m], codes[:, :, m].reshape(-1).astype(np.int64), Gs)
     return dC
+
+
+def code_update_f32(W: np.ndarray, codebooks: np.ndarray, codes: np.ndarray,
+                    H: np.ndarray | None = None, ms=None) -> np.ndarray:
+    """One greedy code-search step (Stage-1 calibration, Sec. 3.1; the code
+    optimisation of AQLM with beam width 1): for every group and each codebook m in
+    ``ms`` in turn, replace code b[m] by the codeword that minimises the group's
+    error with the other codebooks' codewords held fixed,
+        r = w_group - sum_{m' != m} C^(m')[b[m']]          (ascending m')
+        score(c) = d^T H d,  d = C^(m)[c] - r               (H = I when None)
+    with H the group's g x g block of A A^T for calibration inputs A (the
+    block-diagonal part of ||W A - W-hat A||^2).  The decision is taken in float32
+    with a fixed operation order (each product and sum rounded separately,
+    sums in ascending element index), ties to the lowest c.
+    W [N][K] float32; codebooks [M][n_code][g]; codes [N][K/g][M] (a copy is
+    updated and returned); H [K/g][g][g] float32 or None.  Pure Python loops over
+    groups: small inputs only.
+    """
+    N, Gr, M = codes.shape
+    Mc, n_code, g = codebooks.shape
+    C = codebooks.astype(np.float32)
+    Wf = W.astype(np.float32).reshape(N, Gr, g)
+    out = codes.copy()
+    ms = range(M) if ms is None else ms
+    f32 = np.float32
+    for n in range(N):
+        for i in range(Gr):
+            for m in ms:
+                r = Wf[n, i].copy()
+                for m2 in range(M):
+                    if m2 != m:
+                        r = (r - C[m2, int(out[n, i, m2])]).astype(f32)
+                d = (C[m] - r[None, :]).astype(f32)               # [n_code][g]
+                if H is None:
+                    t = d
+                else:
+                    Hi = H[i].astype(f32)
+                    t = np.zeros_like(d)
+                    for e2 in range(g):
+                        t = (t + (Hi[:, e2][None, :] * d[:, e2][:, None]).astype(f32)).astype(f32)
+                score = np.zeros(n_code, dtype=f32)
+                for e in range(g):
+                    score = (score + (d[:, e] * t[:, e]).astype(f32)).astype(f32)
+                out[n, i, m] = int(np.argmin(score))           # first minimum = lowest c
+    return out
 
 
 # --------------------------------------------------------------------------- packing

@@ -39,6 +39,7 @@ _SIGNATURES = {
     "aq_quant_act": (_c_int, [_c_void_p, _c_void_p, _c_int64, _c_float, _c_void_p]),
     "aq_codebook_grad": (_c_int, [_c_void_p] * 3 + [_c_float, _c_void_p] + [_c_int] * 5
                          + [_c_void_p]),
+    "aq_code_update": (_c_int, [_c_void_p] * 4 + [_c_int] * 7 + [_c_void_p]),
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
@@ -168,6 +169,14 @@ def aq_codebook_grad(codes_packed, G, scale, s_x, dC, N, K, g=8, M=2, B=8, strea
     _check(load_library().aq_codebook_grad(
         _ptr(codes_packed), _ptr(G), _ptr(scale), float(s_x), _ptr(dC), N, K, g, M, B,
         _stream(stream)), "aq_codebook_grad")
+
+
+def aq_code_update(W, codebooks, codes, H, m_first, m_count, N, K, g=8, M=2, B=8,
+                   stream=None) -> None:
+    """One greedy code-search step over codebooks [m_first, m_first + m_count)."""
+    _check(load_library().aq_code_update(
+        _ptr(W), _ptr(codebooks), _ptr(codes), _ptr(H), m_first, m_count, N, K, g, M, B,
+        _stream(stream)), "aq_code_update")
 
 
 def aq_linear_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:

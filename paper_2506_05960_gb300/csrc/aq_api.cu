@@ -692,6 +692,24 @@ int aq_codebook_grad(const void* codes_packed, const float* G, const void* scale
                      "aq_codebook_grad launch");
 }
 
+int aq_code_update(const float* W, const void* codebooks, void* codes, const float* H,
+                   int m_first, int m_count, int N, int K, int g, int M, int B, void* stream) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (B != 8) return set_error(AQ_ERR_UNSUPPORTED, "code search supports 8-bit codes only");
+  if (N <= 0 || K <= 0 || K % g != 0) return set_error(AQ_ERR_SHAPE, "need N, K > 0 and K %% g == 0");
+  if (m_first < 0 || m_count < 0 || m_first + m_count > M)
+    return set_error(AQ_ERR_SHAPE, "codebook range [%d, %d) outside [0, %d)", m_first,
+                     m_first + m_count, M);
+  if (!W || !codebooks || !codes) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(W) || !aligned16(codebooks) || !aligned16(codes) || (H && !aligned16(H)))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  if (m_count == 0) return ok();
+  return cuda_status(aq::launch_code_update(W, codebooks, codes, H, m_first, m_count, N, K, M,
+                                            static_cast<cudaStream_t>(stream)),
+                     "aq_code_update launch");
+}
+
 int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stream) {
   if (numel < 0) return set_error(AQ_ERR_SHAPE, "numel < 0");
   if (!(s_x > 0.0f) || s_x == __builtin_inff())

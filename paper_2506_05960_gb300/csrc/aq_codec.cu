@@ -389,4 +389,100 @@ cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half
                     K, M, KB);
 }
 
+// ============================================================== code search step
+// Stage-1 calibration (Sec. 3.1; the code optimisation of AQLM, beam width 1): for
+// every group and each codebook m in [m_first, m_first + m_count) in turn, set
+// b[m] to the codeword minimising the group's error with the other codewords fixed:
+//   r = w - sum_{m' != m} C^(m')[b[m']] (ascending m'),  d = C^(m)[c] - r,
+//   score(c) = d^T H d  (H = the group's 8x8 block of A A^T, or I when H is NULL),
+// in fp32 with every product and sum rounded separately in ascending element order
+// (no fused multiply-add), ties to the lowest c -- the same decision as the
+// reference step.  8-bit codes (256 candidates, codebooks staged in shared memory
+// as fp16); one thread per group, consecutive threads on consecutive rows of the
+// same group column so that a warp shares H's block.
+template <bool kWeighted>
+__global__ void __launch_bounds__(256) code_update_kernel(const float* __restrict__ W,
+                                                          const __half* __restrict__ books,
+                                                          uint8_t* __restrict__ codes,
+                                                          const float* __restrict__ H,
+                                                          int m_first, int m_count, int N, int K,
+                                                          int M) {
+  extern __shared__ __half sb[];                          // [M][256][8]
+  grid_dependency_wait();
+  allow_dependents();
+  for (int i = threadIdx.x; i < M * 256 * 8; i += blockDim.x) sb[i] = books[i];
+  __syncthreads();
+  const int Gr = K / 8;
+  const int64_t total = static_cast<int64_t>(N) * Gr;
+  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int i = static_cast<int>(idx / N);
+    const int n = static_cast<int>(idx - static_cast<int64_t>(i) * N);
+    uint8_t* bc = codes + (static_cast<int64_t>(n) * Gr + i) * M;
+    float w[8];
+    const float4 w0 = __ldg(reinterpret_cast<const float4*>(W + static_cast<int64_t>(n) * K + i * 8));
+    const float4 w1 = __ldg(reinterpret_cast<const float4*>(W + static_cast<int64_t>(n) * K + i * 8) + 1);
+    w[0] = w0.x; w[1] = w0.y; w[2] = w0.z; w[3] = w0.w;
+    w[4] = w1.x; w[5] = w1.y; w[6] = w1.z; w[7] = w1.w;
+    float h[64];
+    if constexpr (kWeighted) {
+#pragma unroll
+      for (int e = 0; e < 64; ++e) h[e] = __ldg(H + i * 64 + e);
+    }
+    for (int m = m_first; m < m_first + m_count; ++m) {
+      float r[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) r[e] = w[e];
+      for (int m2 = 0; m2 < M; ++m2) {
+        if (m2 == m) continue;
+        const __half* cw = sb + (m2 * 256 + bc[m2]) * 8;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) r[e] = __fsub_rn(r[e], __half2float(cw[e]));
+      }
+      float best = 0.0f;
+      int best_c = 0;
+      for (int c = 0; c < 256; ++c) {
+        const __half* cw = sb + (m * 256 + c) * 8;
+        float d[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) d[e] = __fsub_rn(__half2float(cw[e]), r[e]);
+        float sc = 0.0f;
+        if constexpr (kWeighted) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            float t = 0.0f;
+#pragma unroll
+            for (int e2 = 0; e2 < 8; ++e2) t = __fadd_rn(t, __fmul_rn(h[e * 8 + e2], d[e2]));
+            sc = __fadd_rn(sc, __fmul_rn(d[e], t));
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) sc = __fadd_rn(sc, __fmul_rn(d[e], d[e]));
+        }
+        if (c == 0 || sc < best) {
+          best = sc;
+          best_c = c;
+        }
+      }
+      bc[m] = static_cast<uint8_t>(best_c);
+    }
+  }
+}
+
+cudaError_t launch_code_update(const float* W, const void* books, void* codes, const float* H,
+                               int m_first, int m_count, int N, int K, int M, cudaStream_t st) {
+  const int64_t total = static_cast<int64_t>(N) * (K / 8);
+  int64_t blocks = (total + 255) / 256;
+  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (blocks < 1) blocks = 1;
+  const size_t smem = static_cast<size_t>(M) * 256 * 8 * 2;
+  const __half* b = static_cast<const __half*>(books);
+  uint8_t* c = static_cast<uint8_t*>(codes);
+  if (H)
+    return launch_pdl(code_update_kernel<true>, dim3(static_cast<unsigned>(blocks)), dim3(256), smem,
+                      st, W, b, c, H, m_first, m_count, N, K, M);
+  return launch_pdl(code_update_kernel<false>, dim3(static_cast<unsigned>(blocks)), dim3(256), smem,
+                    st, W, b, c, H, m_first, m_count, N, K, M);
+}
+
 }  // namespace aq

@@ -87,6 +87,10 @@ cudaError_t launch_decode(const void* packed, const void* books, void* W, int N,
 cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half* scale,
                                  float s_x, float* dC, int N, int K, int g, int M, int B,
                                  cudaStream_t st);
+// One greedy code-search step over codebooks [m_first, m_first + m_count) (8-bit
+// codes, g = 8, canonical codes [N][K/8][M] updated in place).
+cudaError_t launch_code_update(const float* W, const void* books, void* codes, const float* H,
+                               int m_first, int m_count, int N, int K, int M, cudaStream_t st);
 // Kernel-aware grouping (g = 9, 3x3 conv): codes [N][Cin][M], books [M][2^B][9] ->
 // W [N][9*Cin] in the convolution's OHWI K order.
 cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int N, int Cin, int M,

@@ -479,3 +479,81 @@ def test_codebook_grad_is_the_derivative_of_the_decoded_layer(kaq):
     assert np.array_equal(O.kaq_from_ohwi(O.kaq_ohwi(books[:, :, :9].reshape(2, 4, 9)
                                                       if kaq else np.zeros((1, 1, 9)))),
                           books[:, :, :9].reshape(2, 4, 9) if kaq else np.zeros((1, 1, 9)))
+
+
+# ----------------------------------------------------------------------------- code search
+def _group_err64(W, books, codes, H=None):
+    """||w - w-hat||_H^2 per group in float64 (H = I when None): [N][Gr]."""
+    N, Gr, M = codes.shape
+    g = books.shape[2]
+    E = W.astype(np.float64).reshape(N, Gr, g) - O.decode_f64(codes, books).reshape(N, Gr, g)
+    if H is None:
+        return np.einsum("nie,nie->ni", E, E)
+    return np.einsum("nie,ief,nif->ni", E, H.astype(np.float64), E)
+
+
+@pytest.mark.parametrize("weighted", [False, True])
+def test_code_update_picks_the_best_codeword(weighted):
+    """Each updated code is the float64 minimiser of the group error with the other
+    codebooks fixed (up to float32 near-ties), and a step never raises the error."""
+    rng = np.random.default_rng(41 + weighted)
+    N, Gr, M, n_code, g = 4, 3, 2, 16, 8
+    books = rng.normal(0, 0.5, size=(M, n_code, g)).astype(np.float16)
+    W = rng.normal(0, 1, size=(N, Gr * g)).astype(np.float32)
+    codes = rng.integers(0, n_code, size=(N, Gr, M), dtype=np.uint8)
+    H = None
+    if weighted:
+        A = rng.normal(size=(Gr, g, 3 * g))
+        H = np.einsum("iek,ifk->ief", A, A).astype(np.float32)      # SPD blocks of A A^T
+    before = _group_err64(W, books, codes, H)
+    new = O.code_update_f32(W, books, codes, H, ms=[1])
+    assert np.array_equal(new[:, :, 0], codes[:, :, 0])              # only codebook 1 moves
+    after = _group_err64(W, books, new, H)
+    assert np.all(after <= before + 1e-9 * (1 + before))
+    for n in range(N):
+        for i in range(Gr):
+            trial = []
+            for c in range(n_code):
+                cc = new.copy()
+                cc[n, i, 1] = c
+                trial.append(_group_err64(W, books, cc, H)[n, i])
+            assert trial[new[n, i, 1]] <= min(trial) + 1e-5 * (1 + min(trial))
+
+
+def test_code_update_identity_weights_equal_unweighted():
+    """H = I given explicitly reproduces the unweighted step bit for bit (the
+    weighted path's sums add exact zeros and unit products)."""
+    rng = np.random.default_rng(43)
+    N, Gr, M, n_code, g = 3, 4, 3, 32, 8
+    books = rng.normal(0, 0.5, size=(M, n_code, g)).astype(np.float16)
+    W = rng.normal(0, 1, size=(N, Gr * g)).astype(np.float32)
+    codes = rng.integers(0, n_code, size=(N, Gr, M), dtype=np.uint8)
+    I = np.broadcast_to(np.eye(g, dtype=np.float32), (Gr, g, g)).copy()
+    assert np.array_equal(O.code_update_f32(W, books, codes), O.code_update_f32(W, books, codes, I))
+
+
+def test_code_update_converges_to_exhaustive_on_separable_books():
+    """With one codebook the step is the exhaustive search; repeated sweeps over two
+    codebooks never increase the error and reach a fixed point."""
+    rng = np.random.default_rng(44)
+    N, Gr, n_code, g = 2, 2, 8, 8
+    books1 = rng.normal(size=(1, n_code, g)).astype(np.float16)
+    W = rng.normal(size=(N, Gr * g)).astype(np.float32)
+    codes = np.zeros((N, Gr, 1), dtype=np.uint8)
+    best = O.code_update_f32(W, books1, codes)
+    for n in range(N):
+        for i in range(Gr):
+            errs = [np.sum((W.reshape(N, Gr, g)[n, i].astype(np.float64) - books1[0, c]) ** 2)
+                    for c in range(n_code)]
+            assert best[n, i, 0] == int(np.argmin(errs))
+    books2 = rng.normal(size=(2, n_code, g)).astype(np.float16)
+    codes = np.zeros((N, Gr, 2), dtype=np.uint8)
+    err = _group_err64(W, books2, codes).sum()
+    for _ in range(6):
+        new = O.code_update_f32(W, books2, codes)
+        e2 = _group_err64(W, books2, new).sum()
+        assert e2 <= err + 1e-9
+        if np.array_equal(new, codes):
+            break
+        codes, err = new, e2
+    assert np.array_equal(O.code_update_f32(W, books2, codes), codes)
