@@ -17,9 +17,9 @@ the GEMM (quantizer + decode only), replayed in the same timed region.
 `e2e` repeats the step through the C ABI with the input copied from pinned host
 memory and the output copied back every step.  `layers` times the other
 workloads (64x64 W4A8 conv, 8x8 conv with one 2^16-entry codebook) and
-`unet_forward` one UNet-shaped forward (97 AQ layers, W2A8 and W4A8, batches 2 and
-16), with each layer preceded by the quantizer, or writing the next layer's int8
-activations from its epilogue.
+`unet_forward` one UNet-shaped forward (97 AQ layers, W2A8 and W4A8, batches 2, 16
+and 64), with each layer preceded by the quantizer, or writing the next layer's
+int8 activations from its epilogue.  A small-T sweep (T = 1..64) times every path.
 
 --impl reference times the CPU oracle (numpy float64) on the headline workload.
 Multi-GPU: independent replicas, one per rank (the layer has no exchange step).
@@ -428,7 +428,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the other workloads and the UNet-shaped forward")
-    ap.add_argument("--unet-batches", default="2,16",
+    ap.add_argument("--unet-batches", default="2,16,64",
                     help="batches of the UNet-shaped forward extras (comma separated)")
     ap.add_argument("--workload", default="qkv", choices=["qkv", "conv64", "conv8", "unet"],
                     help="qkv: the headline line (default); the others run only that workload "
@@ -623,6 +623,31 @@ def main():
                 "us_per_step": ms * 1e3, "candidates_per_s": cand / (ms * 1e-3),
                 "step": "aq_code_update over both codebooks, CUDA graph replay"}
             del gcs
+        # small-T sweep on the qkv shape (2x8) and the 2^16-codebook shape (K = 8640, N = 960,
+        # 1x16): per path, to locate where the lookup-table, fused and dense orders cross
+        from aq_synth import LinearSpec, make_linear as _mlin
+        sweep = {}
+        for (Ks, Ns, Ms, Bs, paths) in ((960, 2880, 2, 8, (0, 1, 2, 3)), (8640, 960, 1, 16, (0, 1, 2))):
+            for Ts in (1, 2, 4, 8, 16, 32, 64):
+                inp_s = _mlin(LinearSpec(T=Ts, K=Ks, N=Ns, M=Ms, B=Bs), seed=Ts)
+                for pth in paths:
+                    if pth == 3 and Ts > 16:
+                        continue
+                    Ls = [Dev(aq, torch, inp_s, dev, path=pth) for _ in range(NSETS)]
+                    with torch.cuda.stream(stream):
+                        for L in Ls:
+                            L.step(stream)
+                    stream.synchronize()
+                    gs = capture(torch, stream, lambda: [L.step(stream) for L in Ls])
+                    ms = replay_ms(torch, stream, gs, 20) / NSETS
+                    wbytes = alg_bytes(Ts, Ks, Ns, Ms, Bs)
+                    key = f"K={Ks} N={Ns} {Ms}x{Bs} T={Ts} " + ["AUTO", "DENSE", "FUSED", "LUT"][pth]
+                    sweep[key] = {"us_per_step": ms * 1e3,
+                                  "tflops": Ls[0].flops / (ms * 1e-3) / 1e12,
+                                  "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
+                                  "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
+                    del gs, Ls
+        layers["small-T sweep (quantizer + layer per step, 8 rotating buffer sets)"] = sweep
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
             for batch in [int(b) for b in args.unet_batches.split(",") if b]:

@@ -76,9 +76,12 @@ typedef enum aq_path {
                          the ordinary layer op), then a TMA-fed tcgen05 tensor-core GEMM   */
   AQ_PATH_FUSED = 2,  /* decode inside the GEMM into shared memory (codebooks in shared
                          memory, or in L2 for 2^16-entry books); W-hat never touches HBM  */
-  AQ_PATH_LUT   = 3   /* lookup-table order of App. A.1 (Eq. A5-A6): per token and group,
+  AQ_PATH_LUT   = 3,  /* lookup-table order of App. A.1 (Eq. A5-A6): per token and group,
                          the dot product with every codeword, then a gather-sum by code;
                          for small token counts and B = 8                                  */
+  AQ_PATH_FEW_TOKENS = 4  /* linear layers with T <= 16: one kernel streams each row's codes
+                         once, decodes in registers and dots with every token on CUDA
+                         cores; no workspace                                              */
 } aq_path;
 
 /* ---- library information -------------------------------------------------- */

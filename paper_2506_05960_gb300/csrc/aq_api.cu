@@ -228,7 +228,6 @@ int resolve_conv_path(int path, int m_tiles, int g) {
 
 // ---- lookup-table path (linear layers, 8-bit codes, T <= 16)
 constexpr int kLutMaxT = 16;       // tokens per call the LUT kernel handles
-constexpr int kLutAutoMaxT = 8;    // AUTO takes the LUT path up to this many tokens
 
 struct LutPlan {
   int J, Tp, chunks, rows_per_cta;
@@ -249,13 +248,21 @@ LutPlan plan_lut(int T, int K, int N, int M) {
   return lp;
 }
 
+// Few-token path: linear layers up to this many tokens; AUTO takes it up to
+// kFewTokensAutoMaxT (measured on GB300: faster than the table and fused paths at
+// T <= 4, equal at 8, slower at 16).
+constexpr int kFewTokensMaxT = 16;
+constexpr int kFewTokensAutoMaxT = 4;
+
 // AUTO / explicit path of a linear layer: -1 unknown path, -2 path cannot run this layer.
 int resolve_linear_path(int path, int T, int B) {
   const int m_tiles = (T + aq::kBM - 1) / aq::kBM;
   switch (path) {
     case AQ_PATH_AUTO:
-      if (B == 8 && T <= kLutAutoMaxT) return AQ_PATH_LUT;
+      if (T <= kFewTokensAutoMaxT) return AQ_PATH_FEW_TOKENS;
       return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
+    case AQ_PATH_FEW_TOKENS:
+      return T <= kFewTokensMaxT ? path : -2;
     case AQ_PATH_DENSE:
     case AQ_PATH_FUSED:
       return path;
@@ -730,6 +737,10 @@ int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
   const int rp = resolve_linear_path(path, T, B);
   if (rp < 0) return path_error(rp, path);
+  if (rp == AQ_PATH_FEW_TOKENS) {
+    *bytes = 0;
+    return ok();
+  }
   if (rp == AQ_PATH_LUT) {
     *bytes = plan_lut(T, K, N, M).ws_bytes;
     return ok();
@@ -778,6 +789,27 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  if (rp == AQ_PATH_FEW_TOKENS) {
+    aq::SkinnyParams sp{};
+    sp.xq = xq;
+    sp.codes = codes_packed;
+    sp.books = codebooks;
+    sp.scale = static_cast<const __half*>(scale);
+    sp.bias = static_cast<const __half*>(bias);
+    sp.y = y;
+    sp.out_f32 = out_dtype == AQ_DTYPE_F32;
+    sp.out_q8 = out_dtype == AQ_DTYPE_I8;
+    sp.s_x = s_x;
+    sp.s_out = s_out;
+    sp.T = T;
+    sp.K = K;
+    sp.N = N;
+    sp.M = M;
+    sp.B = B;
+    ProfScope ps(kProfLutGather, static_cast<cudaStream_t>(stream));
+    return cuda_status(aq::launch_skinny(sp, static_cast<cudaStream_t>(stream)),
+                       "few-token launch");
+  }
   if (rp == AQ_PATH_LUT) {
     const LutPlan lp = plan_lut(T, K, N, M);
     if (!workspace || workspace_bytes < lp.ws_bytes || !aligned16(workspace))

@@ -59,6 +59,20 @@ struct LutParams {
   int chunks, rows_per_cta;
 };
 
+// Parameters of the few-token kernel (linear layer, T <= 16, one pass, no workspace).
+struct SkinnyParams {
+  const int8_t* xq;             // [T][K]
+  const void* codes;            // packed codes [K/64][N][8][M]
+  const void* books;            // [M][2^B][8] fp16
+  const __half* scale;
+  const __half* bias;           // may be null
+  void* y;                      // [T][N]
+  int out_f32, out_q8;
+  float s_x, s_out;
+  int T, K, N, M, B;
+  int quads;                    // row quads per CTA (set by the launcher)
+};
+
 // Launch with programmatic stream serialization (the kernel must call
 // grid_dependency_wait() before touching global memory).
 template <typename... KArgs, typename... Args>
@@ -104,6 +118,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
                         const GemmParams& p, int grid, cudaStream_t st);
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st);
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st);
+cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st);
 
 // Device error words of each translation unit (read and cleared, synchronising).
 cudaError_t read_clear_gemm_error(unsigned* out);

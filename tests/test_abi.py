@@ -103,8 +103,8 @@ def test_null_and_alignment_errors_do_not_launch(lib):
     r = lib.aq_linear(8 + 1, 0.02, 16, 16, 16, None, 16, 0, 4, 64, 64, 8, 2, 8, 16, 1 << 20,
                       0, None)
     assert r == -4
-    # workspace too small
-    r = lib.aq_linear(16, 0.02, 16, 16, 16, None, 16, 0, 4, 64, 64, 8, 2, 8, 16, 8, 0, None)
+    # workspace too small (dense path: the decoded weights need N*K*2 bytes)
+    r = lib.aq_linear(16, 0.02, 16, 16, 16, None, 16, 0, 256, 64, 64, 8, 2, 8, 16, 8, 1, None)
     assert r == -5
     # T == 0 is a no-op even with NULL buffers
     assert lib.aq_linear(None, 0.02, None, None, None, None, None, 0, 0, 64, 64, 8, 2, 8, None,

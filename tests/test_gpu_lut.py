@@ -55,9 +55,10 @@ def test_lut_matches_oracle_lut_order():
 
 def test_lut_path_selection():
     import paper_2506_05960_gb300 as aq
-    # AUTO uses the table path for a handful of tokens, the tensor-core path beyond
-    assert aq.aq_linear_workspace_size(8, 960, 2880, 8, 2, 8, 0) == \
-        aq.aq_linear_workspace_size(8, 960, 2880, 8, 2, 8, LUT)
+    # AUTO takes the few-token path (no workspace) up to 4 tokens, the tensor-core path
+    # beyond; the table path is taken on request
+    assert aq.aq_linear_workspace_size(4, 960, 2880, 8, 2, 8, 0) == 0
+    assert aq.aq_linear_workspace_size(8, 960, 2880, 8, 2, 8, LUT) > 0
     assert aq.aq_linear_workspace_size(256, 960, 2880, 8, 2, 8, 0) == \
         aq.aq_linear_workspace_size(256, 960, 2880, 8, 2, 8, 1)
     with pytest.raises(aq.AQError) as e:
