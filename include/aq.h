@@ -193,6 +193,23 @@ AQ_API int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, voi
  *   path: AQ_PATH_* (AUTO recommended).                                       */
 AQ_API int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
                              size_t* bytes);
+/* Diagnostics: restrict the tensor-core plan of later calls made by this host
+ * thread (workspace-size queries included) to N tile BN (0 = any), K splits
+ * (0 = any) and in-cluster split sum (1), split-K through the workspace (0) or
+ * either (-1).  A call whose shapes admit no such plan runs the cost-model plan.
+ * aq_set_plan_override(0, 0, -1) restores the default.  AQ_ERR_SHAPE for a BN
+ * that is not a multiple of 32 in [0, 192] or other out-of-range values.     */
+AQ_API int aq_set_plan_override(int BN, int splits, int cluster);
+
+/* Plan that aq_linear (fp16 or int8 output) runs for these shapes, for
+ * diagnostics: info[0] = resolved AQ_PATH_*; for the tensor-core paths info[1] =
+ * N tile, info[2] = K splits, info[3] = 1 when the splits of a tile are summed
+ * inside one thread-block cluster (no partials in the workspace, no reduce
+ * kernel), info[4] = pipeline stages, info[5] = (tile, split) work items; 0 for
+ * the other paths.  Writes min(n_info, 6) entries (zero past 6).  No device
+ * access.                                                                      */
+AQ_API int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
+                          int n_info);
 AQ_API int aq_linear(const int8_t* xq, float s_x, const void* codes_packed,
               const void* codebooks, const void* scale, const void* bias,
               void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
@@ -253,6 +270,9 @@ AQ_API int aq_linear_noalloc(const int8_t* xq, float s_x, const void* codes_pack
 AQ_API int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
                              int stride, int pad, int g, int M, int B, int path,
                              size_t* bytes);
+/* Plan of aq_conv2d_nhwc for these shapes; info as for aq_linear_plan.          */
+AQ_API int aq_conv2d_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
+                          int pad, int g, int M, int B, int path, int* info, int n_info);
 AQ_API int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed,
                    const void* codebooks, const void* scale, const void* bias,
                    void* y, int out_dtype, int Nb, int H, int W, int Cin, int Cout,

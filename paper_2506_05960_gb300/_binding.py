@@ -41,6 +41,8 @@ _SIGNATURES = {
                          + [_c_void_p]),
     "aq_code_update": (_c_int, [_c_void_p] * 4 + [_c_int] * 7 + [_c_void_p]),
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
+    "aq_linear_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_set_plan_override": (_c_int, [_c_int] * 3),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_linear_noalloc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
@@ -48,6 +50,7 @@ _SIGNATURES = {
     "aq_linear_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float] + [_c_int] * 6
                      + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
+    "aq_conv2d_plan": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_int), _c_int]),
     "aq_conv2d_nhwc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_nhwc_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float]
@@ -186,6 +189,21 @@ def aq_linear_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:
     return out.value
 
 
+_PLAN_KEYS = ("path", "BN", "splits", "cluster", "stages", "work_items")
+
+
+def aq_set_plan_override(BN=0, splits=0, cluster=-1) -> None:
+    """Restrict this thread's later tensor-core plans (diagnostics); no arguments: default."""
+    _check(load_library().aq_set_plan_override(BN, splits, cluster), "aq_set_plan_override")
+
+
+def aq_linear_plan(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_linear runs for these shapes (diagnostics; no device access)."""
+    info = (_c_int * 6)()
+    _check(load_library().aq_linear_plan(T, K, N, g, M, B, path, info, 6), "aq_linear_plan")
+    return dict(zip(_PLAN_KEYS, list(info)))
+
+
 def aq_linear(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N, g=8, M=2,
               B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
     _check(load_library().aq_linear(
@@ -218,6 +236,15 @@ def aq_conv2d_workspace_size(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g
                                                    M, B, path, ctypes.byref(out)),
            "aq_conv2d_workspace_size")
     return out.value
+
+
+def aq_conv2d_plan(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8,
+                   path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_conv2d_nhwc runs for these shapes (diagnostics; no device access)."""
+    info = (_c_int * 6)()
+    _check(load_library().aq_conv2d_plan(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path,
+                                         info, 6), "aq_conv2d_plan")
+    return dict(zip(_PLAN_KEYS, list(info)))
 
 
 def aq_conv2d_nhwc(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, Nb, H, W, Cin,

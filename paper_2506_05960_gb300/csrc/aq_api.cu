@@ -110,9 +110,15 @@ int encode(CUtensorMap* map, CUtensorMapDataType dt, int rank, const void* base,
 constexpr int kPlanSMs = 152;            // GB300 SM count assumed by the cost model
 constexpr size_t kSmemOptin = 232448;    // max dynamic shared memory per CTA on sm_103
 
+// Clusters of S CTAs (one CTA per SM) resident at once, S = 0..8, as reported by
+// cudaOccupancyMaxActiveClusters on GB300 (152 SMs): the GPC layout leaves fewer
+// than 152 / S.  A plan whose clusters exceed this runs in two waves.
+constexpr int kPlanMaxClusters[aq::kMaxClusterSplits + 1] = {0, 152, 76, 46, 36, 28, 23, 15, 15};
+
 struct Plan {
   int BN, n_tiles, m_tiles, splits, kb_per_split, num_kb;
   int stages, a_stages, acc_stride, a_col, total_tiles;
+  int cluster;  // the splits of a tile form one cluster and are summed in shared memory
 };
 
 // Cycles of one pipeline stage (eight 128 x BN x 16 MMAs issued by one thread),
@@ -124,83 +130,127 @@ double stage_cycles(int BN) {
   return 8.0 * mma + exposed;
 }
 
-// Fused path: the four decoder warps rebuild BN x 16 groups per stage, each group
-// about 12 + 12*M instructions (twice that for 2^16-entry books gathered from L2).
+// Fused path: the decoder warps rebuild BN x 16 groups per stage.  With 8-bit codes
+// the stage is bound by shared-memory traffic: per group M codeword lookups of 16 B,
+// the 16-byte decoded store and the tensor core's 16-byte read, plus 32 KB of
+// activations (TMA write, converter read), at about 80 B per cycle (measured on
+// GB300), and by the lookup latency (about 1000 cycles) when there is little work.
+// 16-bit codes gather their codewords from L2: about (12 + 12*M) * 2 issue cycles
+// per group over 8 warps.
 double decode_stage_cycles(int BN, int M, int B) {
-  const double per_group = (12.0 + 12.0 * M) * (B == 16 ? 2.0 : 1.0);
-  return BN * 16.0 * per_group / 128.0;
+  if (B == 16) return BN * 16.0 * (12.0 + 12.0 * M) * 2.0 / 256.0;
+  const double bytes = BN * 16.0 * (16.0 * M + 32.0) + 32768.0;
+  return std::max(1000.0, bytes / 80.0);
 }
 
-int book_smem_bytes(bool fused, int M, int B) { return (fused && B == 8) ? M * 256 * 16 : 0; }
+int book_smem_bytes(bool fused, int M, int B) {
+  return (fused && B == 8) ? M * 256 * 16 * aq::fused_book_copies(M) : 0;
+}
 
 // Fused path: packed code bytes of one row for one 64-wide K block, staged per stage.
 int code_smem_bytes(bool fused, int M, int B) { return fused ? 8 * M * (B / 8) : 0; }
+
+// fp32 epilogue staging: fp32 output, or split-K partials stored to the workspace
+bool plan_f32_staging(const Plan& pl, bool f32_out) {
+  return f32_out || (pl.splits > 1 && !pl.cluster);
+}
 
 void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes) {
   pl.acc_stride = pl.BN;
   pl.a_col = 2 * pl.acc_stride;
   pl.a_stages = aq::gemm_a_stages(pl.BN);
-  pl.stages = aq::gemm_max_stages(pl.BN, f32_out || pl.splits > 1, book_bytes, code_bytes);
+  pl.stages = aq::gemm_max_stages(pl.BN, plan_f32_staging(pl, f32_out), book_bytes, code_bytes);
   pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
 }
 
 // Picks the N tile and the K split that minimise a model of the busiest SM's time:
-// waves x (stage cycles x stages per tile + a fixed tile overhead), plus the traffic
-// and launch of the split-K reduction when K is split.  Depends only on the shapes
-// (and, for the fused path, on the code format).
+// waves x (stage cycles x stages per tile + a fixed tile overhead), plus the cost of
+// the split-K reduction when K is split: either the partials' round trip through the
+// workspace and the reduce kernel (its launch waits for the GEMM to retire, about
+// 2 us), or, when all clusters of S <= 8 CTAs are resident at once, the in-cluster sum
+// through distributed shared memory (two cluster barriers and 128 x BN x 4 bytes per
+// CTA at about 64 B per cycle).  Depends only on the shapes (and, for the fused
+// path, on the code format).
+// Diagnostic plan override of this host thread (aq_set_plan_override): N tile, K
+// splits, in-cluster sum (-1: free).  Plans the shapes cannot take are skipped and the
+// cost-model plan runs instead.
+struct PlanOverride {
+  int BN = 0, splits = 0, cluster = -1;
+};
+thread_local PlanOverride g_plan_override;
+
 Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
                bool fused = false, int M = 1, int B = 8) {
   const int num_kb = (K + aq::kBK - 1) / aq::kBK;
   const int book_bytes = book_smem_bytes(fused, M, B);
   const int code_bytes = code_smem_bytes(fused, M, B);
+  const PlanOverride ov = g_plan_override;
   double best = 1e30;
   Plan bp{};
-  for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
-    if (BN == 224) continue;
-    if (aq::gemm_a_stages(BN) < 2) continue;
-    if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes) < 2) continue;
-    const int n_tiles = (N + BN - 1) / BN;
-    const int max_split = allow_split ? std::min(num_kb, 64) : 1;
-    double st_cyc = stage_cycles(BN);
-    if (fused) st_cyc = std::max(st_cyc, decode_stage_cycles(BN, M, B));
-    for (int sp = 1; sp <= max_split; ++sp) {
-      const int kbps = (num_kb + sp - 1) / sp;
-      const int s_eff = (num_kb + kbps - 1) / kbps;
-      if (s_eff != sp) continue;
-      const long tiles = static_cast<long>(m_tiles) * n_tiles * s_eff;
-      const long waves = (tiles + kPlanSMs - 1) / kPlanSMs;
-      const double tile_cycles = (kbps / 2) * st_cyc + (kbps & 1) * 0.5 * st_cyc + 800.0;
-      double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
-      if (s_eff > 1) {
-        // partials written and read back (mostly from L2) + the reduce launch
-        const double part_bytes = s_eff * 8.0 * T * static_cast<double>(N);
-        t += part_bytes / (part_bytes < 64e6 ? 15.0e12 : 6.0e12) + 2.0 * T * N / 6.0e12 + 1.0e-6;
-      }
-      if (t < best * 0.999) {
-        best = t;
-        bp = Plan{};
-        bp.BN = BN;
-        bp.n_tiles = n_tiles;
-        bp.m_tiles = m_tiles;
-        bp.splits = s_eff;
-        bp.kb_per_split = kbps;
-        bp.num_kb = num_kb;
+  // forced: only the override's choices (a cluster plan is then allowed beyond one wave of
+  // clusters, which still runs correctly, in waves)
+  auto search = [&](bool forced) {
+    for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
+      if (BN == 224) continue;
+      if (forced && ov.BN > 0 && BN != ov.BN) continue;
+      if (aq::gemm_a_stages(BN) < 2) continue;
+      if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes) < 2) continue;
+      const int n_tiles = (N + BN - 1) / BN;
+      const int max_split = allow_split ? std::min(num_kb, 64) : 1;
+      double st_cyc = stage_cycles(BN);
+      if (fused) st_cyc = std::max(st_cyc, decode_stage_cycles(BN, M, B));
+      for (int sp = 1; sp <= max_split; ++sp) {
+        const int kbps = (num_kb + sp - 1) / sp;
+        const int s_eff = (num_kb + kbps - 1) / kbps;
+        if (s_eff != sp) continue;
+        if (forced && ov.splits > 0 && s_eff != ov.splits) continue;
+        const long tiles = static_cast<long>(m_tiles) * n_tiles * s_eff;
+        const long waves = (tiles + kPlanSMs - 1) / kPlanSMs;
+        const double tile_cycles = (kbps / 2) * st_cyc + (kbps & 1) * 0.5 * st_cyc + 800.0;
+        for (int cl = 0; cl < 2; ++cl) {
+          if (forced && ov.cluster >= 0 && cl != ov.cluster) continue;
+          double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
+          if (cl) {
+            if (s_eff < 2 || s_eff > aq::kMaxClusterSplits) continue;
+            if (!forced && static_cast<long>(m_tiles) * n_tiles > kPlanMaxClusters[s_eff]) continue;
+            t = tile_cycles / 1.9e9 + (1000.0 + 128.0 * BN * 4.0 / 64.0) / 1.9e9;
+          } else if (s_eff > 1) {
+            // partials written and read back (mostly from L2) + the reduce kernel
+            const double part_bytes = s_eff * 8.0 * T * static_cast<double>(N);
+            t += part_bytes / (part_bytes < 64e6 ? 15.0e12 : 6.0e12) + 2.0 * T * N / 6.0e12 +
+                 2.0e-6;
+          }
+          if (t < best * 0.999) {
+            best = t;
+            bp = Plan{};
+            bp.BN = BN;
+            bp.n_tiles = n_tiles;
+            bp.m_tiles = m_tiles;
+            bp.splits = s_eff;
+            bp.kb_per_split = kbps;
+            bp.num_kb = num_kb;
+            bp.cluster = cl;
+          }
+        }
       }
     }
-  }
+  };
+  if (ov.BN > 0 || ov.splits > 0 || ov.cluster >= 0) search(true);
+  if (best > 1e29) search(false);
   finish_plan(bp, f32_out, book_bytes, code_bytes);
   return bp;
 }
 
 size_t dense_ws_bytes(int T, int N, int K, const Plan& pl) {
   size_t b = align_up(static_cast<size_t>(N) * K * 2, 1024);
-  if (pl.splits > 1) b += align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024);
+  if (pl.splits > 1 && !pl.cluster) b += align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024);
   return b;
 }
 
 // Fused path workspace: only the split-K partial sums (no decoded weights).
 size_t fused_ws_bytes(int T, int N, const Plan& pl) {
-  return pl.splits > 1 ? align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024) : 0;
+  return (pl.splits > 1 && !pl.cluster) ? align_up(static_cast<size_t>(pl.splits) * T * N * 4, 1024)
+                                        : 0;
 }
 
 // AUTO decodes inside the GEMM (fused path) when every weight tile is decoded by at
@@ -464,7 +514,8 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   p.a_stages = pl.a_stages;
   p.acc_stride = pl.acc_stride;
   p.a_col = pl.a_col;
-  p.partial = pl.splits > 1 ? partial : nullptr;
+  p.cluster = pl.cluster;
+  p.partial = (pl.splits > 1 && !pl.cluster) ? partial : nullptr;
   const int T = p.T, N = p.N, K = p.K;
   int r;
   CUtensorMap mapB, mapY;
@@ -513,10 +564,12 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   }
   {
     ProfScope ps(fused ? kProfFused : kProfGemm, st);
-    e = aq::launch_gemm(mapA, mapB, mapY, p, std::min(pl.total_tiles, sm_count()), st);
+    // in-cluster split-K runs one CTA per (tile, split); otherwise a persistent grid
+    const int grid = pl.cluster ? pl.total_tiles : std::min(pl.total_tiles, sm_count());
+    e = aq::launch_gemm(mapA, mapB, mapY, p, grid, st);
   }
   if (e != cudaSuccess) return cuda_status(e, "gemm launch");
-  if (pl.splits > 1) {
+  if (pl.splits > 1 && !pl.cluster) {
     ProfScope ps(kProfSplitK, st);
     e = aq::launch_splitk_reduce(p, pl.splits, st);
     if (e != cudaSuccess) return cuda_status(e, "split-K reduce launch");
@@ -749,6 +802,46 @@ int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path,
   return ok();
 }
 
+namespace {
+// info[0] = resolved path, then for the tensor-core paths [1] BN, [2] K splits,
+// [3] in-cluster split sum (0/1), [4] pipeline stages, [5] (tile, split) work items.
+int fill_plan_info(int rp, const Plan* pl, int* info, int n_info) {
+  if (!info || n_info < 1) return set_error(AQ_ERR_NULL, "info is NULL or n_info < 1");
+  int v[6] = {rp, 0, 0, 0, 0, 0};
+  if (pl) {
+    v[1] = pl->BN;
+    v[2] = pl->splits;
+    v[3] = pl->cluster;
+    v[4] = pl->stages;
+    v[5] = pl->total_tiles;
+  }
+  for (int i = 0; i < n_info; ++i) info[i] = i < 6 ? v[i] : 0;
+  return ok();
+}
+}  // namespace
+
+int aq_set_plan_override(int BN, int splits, int cluster) {
+  if (BN < 0 || BN > aq::kMaxBN || BN % 32 != 0 || splits < 0 || cluster < -1 || cluster > 1)
+    return set_error(AQ_ERR_SHAPE, "plan override: BN in {0, 32, ..., %d}, splits >= 0, "
+                     "cluster in {-1, 0, 1}", aq::kMaxBN);
+  g_plan_override.BN = BN;
+  g_plan_override.splits = splits;
+  g_plan_override.cluster = cluster;
+  return ok();
+}
+
+int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info, int n_info) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
+  const int rp = resolve_linear_path(path, T, B);
+  if (rp < 0) return path_error(rp, path);
+  if (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT) return fill_plan_info(rp, nullptr, info, n_info);
+  const Route rt = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B);
+  return fill_plan_info(rp, &rt.pl, info, n_info);
+}
+
 int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
               int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
@@ -900,6 +993,21 @@ int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, in
   const int T = Nb * cg.Ho * cg.Wo;
   *bytes = route_gemm(rp, T, Cout, K, cg.m_tiles, false, M, B).ws;
   return ok();
+}
+
+int aq_conv2d_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                   int g, int M, int B, int path, int* info, int n_info) {
+  int r = check_format(g, M, B, true);
+  if (r) return r;
+  r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
+  if (r) return r;
+  ConvGeom cg;
+  r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
+  if (r) return r;
+  const int rp = resolve_conv_path(path, cg.m_tiles, g);
+  if (rp < 0) return path_error(rp, path);
+  const Route rt = route_gemm(rp, Nb * cg.Ho * cg.Wo, Cout, kh * kw * Cin, cg.m_tiles, false, M, B);
+  return fill_plan_info(rp, &rt.pl, info, n_info);
 }
 
 int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,

@@ -7,7 +7,7 @@
 //
 // Persistent kernel, one CTA per SM, static round-robin over 128 x BN output
 // tiles (and K splits).  A pipeline stage covers 128 of K (two 64-wide TMA
-// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps:
+// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps (eighteen on the fused path):
 //   warp 0      TMA producer: int8 activation boxes (64-byte swizzle) and fp16
 //               weight boxes (128-byte swizzle) into an S-deep smem ring
 //   warp 1      TMEM owner (all 512 columns) and the single MMA-issuing thread:
@@ -21,6 +21,10 @@
 //               shared memory -> TMA stores (ragged edges clipped by TMA).  The
 //               output is fp16, fp32, or int8: the fp16 value quantized with the
 //               next layer's activation scale (the quantizer fused into the layer)
+//   warps 10..17 (fused path) decoders: rebuild each weight stage from the packed
+//               codes and the shared-memory codebooks (Eq. 4).  The lookups are
+//               bound by shared-memory bandwidth, hence eight warps and the
+//               bank-spread codebook copies (fused_book_copies).
 // The fp32 accumulator is double-buffered in TMEM so the epilogue of one tile
 // runs under the mainloop of the next.  The issue loop carries no divisions:
 // ring index and phase advance by counters.  Every wait is bounded (about 2 s);
@@ -39,8 +43,8 @@ namespace aq {
 
 __device__ unsigned g_gemm_err = 0;
 
-constexpr int kThreads = 448;                   // 14 warps (warps 10..13 decode on the fused path)
-constexpr int kDecodeThreads = 128;
+constexpr int kDecodeThreads = 256;             // warps 10..17 decode on the fused path
+constexpr int kThreads = 320 + kDecodeThreads;
 constexpr int kA8Half = kBM * 64;               // one 64-wide int8 box: 128 rows x 64 B
 constexpr int kA8Stage = kStageBlocks * kA8Half;
 constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A slot
@@ -95,9 +99,16 @@ struct TileCoord {
 
 __device__ __forceinline__ TileCoord tile_coord(const GemmParams& p, int t) {
   TileCoord c;
-  const int tiles_mn = p.m_tiles * p.n_tiles;
-  c.split = t / tiles_mn;
-  const int r = t - c.split * tiles_mn;
+  int r;
+  if (p.cluster) {
+    // the splits of one tile are consecutive CTAs: one cluster
+    r = t / p.splits;
+    c.split = t - r * p.splits;
+  } else {
+    const int tiles_mn = p.m_tiles * p.n_tiles;
+    c.split = t / tiles_mn;
+    r = t - c.split * tiles_mn;
+  }
   c.n_tile = r / p.m_tiles;
   c.m_tile = r - c.n_tile * p.m_tiles;
   c.kb_begin = c.split * p.kb_per_split;
@@ -161,12 +172,14 @@ __device__ __forceinline__ uint4 sum_codewords(const uint4* word) {
 // Fused path: decode the 8 groups of one output row in one 64-wide K block into the
 // row's 128-byte line of the swizzled B stage.  Codes: 8*M*EB contiguous bytes in
 // shared memory (EB = bytes per code), read as 32-bit words and unpacked with
-// constant shifts.  8-bit codes index the codebooks staged in shared memory;
-// 16-bit codes gather from L2, all 8*M reads issued before the first sum.
+// constant shifts.  8-bit codes index the codebooks staged in shared memory (this
+// lane's copy `copy` of fused_book_copies(M)); 16-bit codes gather from L2, all 8*M
+// reads issued before the first sum.
 template <int M, int EB>
 __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* sbook,
                                             const uint4* gbooks, uint8_t* rowp, int n,
-                                            int gvalid) {
+                                            int gvalid, int copy) {
+  constexpr int R = fused_book_copies(M);
   constexpr int kWords = 2 * M * EB;
   uint32_t w[kWords];
   if constexpr (kWords % 4 == 0) {
@@ -197,44 +210,87 @@ __device__ __forceinline__ void decode_unit(const uint8_t* codes, const uint4* s
                                           : make_uint4(0u, 0u, 0u, 0u);
     }
   }
+  if constexpr (EB == 1) {
+    // the codewords of J groups are loaded before any of them is stored: loads and
+    // stores share no ordering the compiler can prove, so a per-group loop would
+    // serialise every lookup behind the previous store (codes past gvalid are zero
+    // bytes in the packed layout, so their lookups stay inside the table)
+    constexpr int J = M <= 2 ? 4 : (M <= 4 ? 2 : 1);
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    uint4 out = make_uint4(0u, 0u, 0u, 0u);
-    if (j < gvalid) {
-      uint4 word[M];
+    for (int j0 = 0; j0 < 8; j0 += J) {
+      uint4 word[J * M];
 #pragma unroll
-      for (int m = 0; m < M; ++m) {
-        const int idx = j * M + m;
-        if (EB == 1)
-          word[m] = sbook[m * 256 + ((w[idx >> 2] >> (8 * (idx & 3))) & 0xFFu)];
-        else
-          word[m] = cw[idx % kPre];
+      for (int i = 0; i < J * M; ++i) {
+        const int idx = j0 * M + i;
+        word[i] = sbook[((i % M) * 256 + ((w[idx >> 2] >> (8 * (idx & 3))) & 0xFFu)) * R + copy];
       }
-      out = sum_codewords<M>(word);
+#pragma unroll
+      for (int jj = 0; jj < J; ++jj) {
+        const int j = j0 + jj;
+        uint4 out = sum_codewords<M>(word + jj * M);
+        if (j >= gvalid) out = make_uint4(0u, 0u, 0u, 0u);
+        *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = out;
+      }
     }
-    *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = out;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint4 out = j < gvalid ? sum_codewords<M>(cw + j * M) : make_uint4(0u, 0u, 0u, 0u);
+      *reinterpret_cast<uint4*>(rowp + ((j ^ (n & 7)) << 4)) = out;
+    }
   }
 }
 
 __device__ __forceinline__ void decode_unit_dispatch(int M, int EB, const uint8_t* codes,
                                                      const uint4* sbook, const uint4* gbooks,
-                                                     uint8_t* rowp, int n, int gvalid) {
+                                                     uint8_t* rowp, int n, int gvalid,
+                                                     int copy) {
   if (EB == 1) {
     switch (M) {
-      case 1: decode_unit<1, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 2: decode_unit<2, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 3: decode_unit<3, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 4: decode_unit<4, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 5: decode_unit<5, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 6: decode_unit<6, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      case 7: decode_unit<7, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
-      default: decode_unit<8, 1>(codes, sbook, gbooks, rowp, n, gvalid); break;
+      case 1: decode_unit<1, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 2: decode_unit<2, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 3: decode_unit<3, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 4: decode_unit<4, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 5: decode_unit<5, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 6: decode_unit<6, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      case 7: decode_unit<7, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
+      default: decode_unit<8, 1>(codes, sbook, gbooks, rowp, n, gvalid, copy); break;
     }
   } else {
     if (M == 1)
-      decode_unit<1, 2>(codes, sbook, gbooks, rowp, n, gvalid);
+      decode_unit<1, 2>(codes, sbook, gbooks, rowp, n, gvalid, copy);
     else
-      decode_unit<2, 2>(codes, sbook, gbooks, rowp, n, gvalid);
+      decode_unit<2, 2>(codes, sbook, gbooks, rowp, n, gvalid, copy);
+  }
+}
+
+// Epilogue of four summed split-K outputs y[t][n .. n+3]: acc * (s_x * scale) + bias in
+// fp32, then fp32, fp16 or the 8-bit activation rule (the same arithmetic as the
+// single-pass epilogue).
+__device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n, float4 acc) {
+  float o[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float sc = p.s_x * __half2float(p.scale[n + e]);
+    const float bi = p.bias ? __half2float(p.bias[n + e]) : 0.0f;
+    o[e] = fmaf(o[e], sc, bi);
+  }
+  if (p.out_f32) {
+    *reinterpret_cast<float4*>(static_cast<float*>(p.y) + t * p.N + n) =
+        make_float4(o[0], o[1], o[2], o[3]);
+  } else if (p.out_q8) {
+    const float rs = __frcp_rn(p.s_out);
+    uint32_t b = 0;
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      b |= static_cast<uint32_t>(static_cast<uint8_t>(quant_one(__float2half_rn(o[e]), p.s_out, rs)))
+           << (8 * e);
+    *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(p.y) + t * p.N + n) = b;
+  } else {
+    __half2 a = __floats2half2_rn(o[0], o[1]);
+    __half2 b = __floats2half2_rn(o[2], o[3]);
+    uint2 w = make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+    *reinterpret_cast<uint2*>(static_cast<__half*>(p.y) + t * p.N + n) = w;
   }
 }
 
@@ -268,14 +324,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // nothing in global memory is touched before the previous kernel in the stream is done
-  grid_dependency_wait();
-  allow_dependents();
-  if (p.fused && p.book_bytes > 0) {
-    // 8-bit codebooks of the fused path live in shared memory for the whole kernel
-    for (int i = threadIdx.x; i < p.book_bytes / 16; i += blockDim.x)
-      sbook[i] = reinterpret_cast<const uint4*>(p.books)[i];
-  }
+  // Barriers and tensor memory are set up while the previous kernel in the stream may
+  // still run (programmatic launch); nothing in global memory is touched before it is done.
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       // fused path: the producer's expect_tx arrival + one arrival per decoder warp
@@ -305,6 +355,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  grid_dependency_wait();
+  allow_dependents();
   const uint32_t tmem_base = bar->tmem_base;
 
   if (warp == 0) {
@@ -508,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int buf = static_cast<int>(lt & 1u);
       const int m0 = tc.m_tile * kBM;
       const int n0 = tc.n_tile * BN;
-      if (!raw) {
+      if (!raw && !p.cluster) {
         // this tile's scale/bias, loaded while the accumulator is still being computed
         for (int i = lane; i < BN; i += 32) {
           const int n = n0 + i;
@@ -532,6 +584,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar->acc_empty[buf]);
+        }
+        if (p.cluster) {
+          // this split's fp32 partial, row m of a [128][BN] tile in this CTA's shared
+          // memory (the ring is idle: one tile per CTA and its MMAs are complete);
+          // 16-byte chunks XOR-swizzled by the row so a warp's stores spread over banks
+          const int m = q * 32 + lane;
+          uint8_t* prow = smem + m * (BN * 4) + c0 * 4;
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(prow + ((j ^ (m & 7)) << 4)) =
+                make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                            __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+          continue;
         }
         uint8_t* dst = wbuf + (chunk & 1u) * epi_buf;
         if (lane == 0) bulk_wait_group_read<1>();   // the store issued from dst two chunks ago
@@ -622,6 +687,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     // shared memory.  Same arithmetic as the decode kernel: fp32 sum of the M
     // codewords in ascending m, one round to fp16.
     const int dt = threadIdx.x - 320;
+    const int copy = lane & (fused_book_copies(p.M) - 1);   // this lane's codebook copy
+    if (p.book_bytes > 0) {
+      // 8-bit codebooks live in shared memory for the whole kernel, R copies of each
+      // entry (staged by the decoders alone, while the producer's first loads are in
+      // flight); thread i writes copy (r + i) % R at step r, so the stores of a quarter
+      // warp land in distinct bank groups
+      const int R = fused_book_copies(p.M);
+      const uint4* gb = reinterpret_cast<const uint4*>(p.books);
+      for (int i = dt; i < p.M * 256; i += kDecodeThreads) {
+        const uint4 v = gb[i];
+        for (int r = 0; r < R; ++r) sbook[i * R + ((r + i) & (R - 1))] = v;
+      }
+      named_barrier_sync(1, kDecodeThreads);
+    }
     const int eb = p.B >> 3;                         // bytes per code
     const int G = p.K >> 3;
     Ring rg;
@@ -657,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const uint8_t* cp = c_src + u * code_bytes;
           decode_unit_dispatch(p.M, eb, cp, sbook, reinterpret_cast<const uint4*>(p.books), rowp,
-                               n, min(8, G - gk0));
+                               n, min(8, G - gk0), copy);
         }
         fence_proxy_async_smem();     // generic writes -> visible to the tensor core
         __syncwarp();
@@ -665,6 +744,52 @@ __global__ void __launch_bounds__(kThreads, 1)
         rg.next(S);
       }
     }
+  }
+
+  if (p.cluster) {
+    // In-cluster split-K reduction: CTA rank r of the cluster owns rows [r*rows, (r+1)*rows)
+    // of the tile and sums them over the splits' shared-memory partials in split order
+    // (the order of the split-K reduce kernel, so both give the same bits), then applies
+    // the epilogue.  Every thread of every CTA passes both cluster barriers, also after a
+    // failed wait above, so no CTA waits on a peer that left.
+    __syncwarp();
+    cluster_sync_all();  // every split's partial tile is in its CTA's shared memory
+    const TileCoord tc = tile_coord(p, blockIdx.x);
+    const int nsp = p.splits;
+    const int rows = (kBM + nsp - 1) / nsp;
+    const int r0 = tc.split * rows;
+    const int r1 = min(kBM, r0 + rows);
+    const int c4n = BN >> 2;
+    const int m0 = tc.m_tile * kBM;
+    const int n0 = tc.n_tile * BN;
+    const uint32_t pbase = smem_u32(smem);
+    const int items = r1 > r0 ? (r1 - r0) * c4n : 0;
+    for (int i = threadIdx.x; i < items; i += blockDim.x) {
+      const int mr = i / c4n;
+      const int c4 = i - mr * c4n;
+      const int m = r0 + mr;
+      const int t = m0 + m;
+      const int n = n0 + 4 * c4;
+      if (t >= p.T || n >= p.N) continue;
+      const uint32_t off =
+          static_cast<uint32_t>(m * (BN * 4) + (c4 >> 3) * 128 + (((c4 & 7) ^ (m & 7)) << 4));
+      float4 v[kMaxClusterSplits];
+#pragma unroll
+      for (int sp = 0; sp < kMaxClusterSplits; ++sp)
+        if (sp < nsp) v[sp] = ld_cluster_f4(cluster_map(pbase + off, static_cast<uint32_t>(sp)));
+      float4 acc = v[0];
+#pragma unroll
+      for (int sp = 1; sp < kMaxClusterSplits; ++sp) {
+        if (sp < nsp) {
+          acc.x += v[sp].x;
+          acc.y += v[sp].y;
+          acc.z += v[sp].z;
+          acc.w += v[sp].w;
+        }
+      }
+      store_out4(p, t, n, acc);
+    }
+    cluster_sync_all();  // no CTA leaves while a peer still reads its shared memory
   }
 
   tc_fence_before();
@@ -693,30 +818,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
       acc.z += v.z;
       acc.w += v.w;
     }
-    float o[4] = {acc.x, acc.y, acc.z, acc.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float sc = p.s_x * __half2float(p.scale[n + e]);
-      const float bi = p.bias ? __half2float(p.bias[n + e]) : 0.0f;
-      o[e] = fmaf(o[e], sc, bi);
-    }
-    if (p.out_f32) {
-      *reinterpret_cast<float4*>(static_cast<float*>(p.y) + t * p.N + n) =
-          make_float4(o[0], o[1], o[2], o[3]);
-    } else if (p.out_q8) {
-      const float rs = __frcp_rn(p.s_out);
-      uint32_t b = 0;
-#pragma unroll
-      for (int e = 0; e < 4; ++e)
-        b |= static_cast<uint32_t>(static_cast<uint8_t>(quant_one(__float2half_rn(o[e]), p.s_out, rs)))
-             << (8 * e);
-      *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(p.y) + t * p.N + n) = b;
-    } else {
-      __half2 a = __floats2half2_rn(o[0], o[1]);
-      __half2 b = __floats2half2_rn(o[2], o[3]);
-      uint2 w = make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
-      *reinterpret_cast<uint2*>(static_cast<__half*>(p.y) + t * p.N + n) = w;
-    }
+    store_out4(p, t, static_cast<int>(n), acc);
   }
 }
 
@@ -732,9 +834,29 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
     if (e != cudaSuccess) return e;
     configured_bytes = static_cast<int>(bytes);
   }
-  // the decoder warps (10..13) exist only on the fused path
+  // the decoder warps (10..17) exist only on the fused path
   const int threads = p.fused ? kThreads : kThreads - kDecodeThreads;
-  return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
+  if (!p.cluster)
+    return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
+  // in-cluster split-K: one CTA per (tile, split), the splits of a tile in one cluster
+  if (p.splits < 2 || p.splits > kMaxClusterSplits || grid != p.total_tiles ||
+      grid % p.splits != 0)
+    return cudaErrorInvalidConfiguration;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = bytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(p.splits);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, aq_gemm_kernel, mapA, mapB, mapY, p);
 }
 
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st) {

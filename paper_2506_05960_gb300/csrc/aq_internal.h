@@ -16,6 +16,16 @@ constexpr int kBK = 64;         // K per TMA box / swizzle row (128 bytes of fp1
 constexpr int kStageBlocks = 2; // 64-wide K blocks per pipeline stage (8 MMAs of K = 16)
 constexpr int kMaxBN = 192;     // widest N tile: 2 fp32 accumulators + >= 2 A stages in TMEM
 constexpr int kMaxStages = 8;   // pipeline ring depth bound
+constexpr int kMaxClusterSplits = 8;  // K splits summed inside one cluster (portable size)
+
+// Fused path, 8-bit codes: copies of the codebooks kept in shared memory.  A 16-byte
+// load is served one quarter warp (8 lanes) per shared-memory cycle, and random codes
+// make those lanes collide on banks.  Copy r stores entry e in 16-byte slot e * R + r
+// and lane l reads copy l % R, so with R = 8 the 8 lanes of a quarter warp always hit
+// 8 different bank groups.  Fewer copies for more codebooks keep the table <= 64 KB.
+__host__ __device__ constexpr int fused_book_copies(int M) {
+  return M <= 2 ? 8 : (M <= 4 ? 4 : 2);
+}
 
 // Parameters of one GEMM launch (passed by value).
 struct GemmParams {
@@ -38,6 +48,9 @@ struct GemmParams {
   int out_q8;                   // int8 output: the next layer's activations, quantized with s_out
   float s_out;
   float* partial;               // split-K partial sums [splits][T][N] (null: fused epilogue)
+  int cluster;                  // 1: the splits of a tile form one thread-block cluster (split =
+                                // cluster rank) and are summed through distributed shared
+                                // memory; grid = total_tiles, one tile per CTA
   // fused decode (B stages written by decoder warps instead of TMA from a decoded W)
   int fused;
   const void* codes;            // packed codes

@@ -141,3 +141,30 @@ def test_kernel_aware_grouping_g9(lib):
         assert _size(lib.aq_conv2d_workspace_size, 2, 16, 16, 64, 96, 3, 3, 1, 1, 9, 2, 8,
                      path)[0] == -3
 
+
+
+def test_plan_query_and_override(lib):
+    """Plan introspection and the diagnostic plan override (no device access)."""
+    import paper_2506_05960_gb300 as aq
+    try:
+        p = aq.aq_linear_plan(128, 960, 960)
+        # one row tile: fused path, K split over a cluster, nothing in the workspace
+        assert p["path"] == 2 and p["cluster"] == 1 and 2 <= p["splits"] <= 8
+        assert aq.aq_linear_workspace_size(128, 960, 960) == 0
+        assert aq.aq_linear_plan(4, 960, 960)["path"] == 4          # few tokens
+        aq.aq_set_plan_override(64, 5, 0)
+        p = aq.aq_linear_plan(128, 960, 960)
+        assert (p["BN"], p["splits"], p["cluster"]) == (64, 5, 0)
+        assert aq.aq_linear_workspace_size(128, 960, 960) == 5 * 128 * 960 * 4
+        aq.aq_set_plan_override(0, 7, -1)                 # 15 K blocks cannot split 7 ways
+        forced = aq.aq_linear_plan(128, 960, 960)
+        aq.aq_set_plan_override()
+        assert forced == aq.aq_linear_plan(128, 960, 960)  # the cost-model plan runs
+        for bad in [(48, 0, -1), (-32, 0, -1), (224 + 32, 0, -1), (0, -1, -1), (0, 0, 2)]:
+            with pytest.raises(aq.AQError) as e:
+                aq.aq_set_plan_override(*bad)
+            assert e.value.status == -2
+        p = aq.aq_conv2d_plan(2, 8, 8, 960, 960, M=2)
+        assert p["cluster"] == 1 and aq.aq_conv2d_workspace_size(2, 8, 8, 960, 960, M=2) == 0
+    finally:
+        aq.aq_set_plan_override()
