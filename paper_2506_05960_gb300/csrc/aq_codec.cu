@@ -27,18 +27,24 @@ __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict
     const float rs = __frcp_rn(s);
     uint4 a = __ldcs(src);
     uint4 b = __ldcs(src + 1);
-    const __half* ha = reinterpret_cast<const __half*>(&a);
-    const __half* hb = reinterpret_cast<const __half*>(&b);
+    __half2 h[8];
+    *reinterpret_cast<uint4*>(&h[0]) = a;
+    *reinterpret_cast<uint4*>(&h[4]) = b;
+    // all 16 values on the fast path (FMA/ALU pipes, straight-line); a value near a tie
+    // is redone alone with the exact rule
+    uint32_t qb[16];
+    uint32_t slow = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float2 xf = __half22float2(h[i]);
+      slow |= quant_fast_bits(xf.x, rs, qb[2 * i]) ? 0u : 1u << (2 * i);
+      slow |= quant_fast_bits(xf.y, rs, qb[2 * i + 1]) ? 0u : 1u << (2 * i + 1);
+    }
+    quant_fix16(slow, h, qb, s, rs);
     uint32_t w[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const __half* h = (i < 2) ? ha + 4 * i : hb + 4 * (i - 2);
-      uint32_t b0 = static_cast<uint8_t>(quant_one(h[0], s, rs));
-      uint32_t b1 = static_cast<uint8_t>(quant_one(h[1], s, rs));
-      uint32_t b2 = static_cast<uint8_t>(quant_one(h[2], s, rs));
-      uint32_t b3 = static_cast<uint8_t>(quant_one(h[3], s, rs));
-      w[i] = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
-    }
+    for (int i = 0; i < 4; ++i)
+      w[i] = pack_low_bytes(qb[4 * i], qb[4 * i + 1], qb[4 * i + 2], qb[4 * i + 3]);
     __stcs(reinterpret_cast<uint4*>(xq) + v, make_uint4(w[0], w[1], w[2], w[3]));
   }
   // scalar tail (numel % 16 elements), handled by the first threads of block 0

@@ -7,7 +7,7 @@
 //
 // Persistent kernel, one CTA per SM, static round-robin over 128 x BN output
 // tiles (and K splits).  A pipeline stage covers 128 of K (two 64-wide TMA
-// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps (eighteen on the fused path):
+// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps (sixteen on the fused path):
 //   warp 0      TMA producer: int8 activation boxes (64-byte swizzle) and fp16
 //               weight boxes (128-byte swizzle) into an S-deep smem ring
 //   warp 1      TMEM owner (all 512 columns) and the single MMA-issuing thread:
@@ -21,9 +21,9 @@
 //               shared memory -> TMA stores (ragged edges clipped by TMA).  The
 //               output is fp16, fp32, or int8: the fp16 value quantized with the
 //               next layer's activation scale (the quantizer fused into the layer)
-//   warps 10..17 (fused path) decoders: rebuild each weight stage from the packed
+//   warps 10..15 (fused path) decoders: rebuild each weight stage from the packed
 //               codes and the shared-memory codebooks (Eq. 4).  The lookups are
-//               bound by shared-memory bandwidth, hence eight warps and the
+//               bound by shared-memory bandwidth, hence six warps and the
 //               bank-spread codebook copies (fused_book_copies).
 // The fp32 accumulator is double-buffered in TMEM so the epilogue of one tile
 // runs under the mainloop of the next.  The issue loop carries no divisions:
@@ -43,7 +43,7 @@ namespace aq {
 
 __device__ unsigned g_gemm_err = 0;
 
-constexpr int kDecodeThreads = 256;             // warps 10..17 decode on the fused path
+constexpr int kDecodeThreads = 192;             // warps 10..15 decode on the fused path
 constexpr int kThreads = 320 + kDecodeThreads;
 constexpr int kA8Half = kBM * 64;               // one 64-wide int8 box: 128 rows x 64 B
 constexpr int kA8Stage = kStageBlocks * kA8Half;
@@ -624,28 +624,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the 8-bit activation rule with the next layer's scale: 32 bytes per row.
           // The fast path covers all but values near a rounding tie (rare): those
           // are redone with the exact quotient.
+          // 16 values at a time on the fast path (straight-line code the compiler can
+          // interleave); a value near a tie (exact ties are common when s has few
+          // significant bits) is redone alone with the exact quotient.
           uint32_t wq[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
-            const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
-            __half hv[4];
-            hv[0] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 0]), sc.x, bi.x));
-            hv[1] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 1]), sc.y, bi.y));
-            hv[2] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 2]), sc.z, bi.z));
-            hv[3] = __float2half_rn(fmaf(__uint_as_float(r[4 * j + 3]), sc.w, bi.w));
-            int qv[4];
-            bool fast = true;
+          for (int hf = 0; hf < 2; ++hf) {
+            __half2 h[8];
+            uint32_t qb[16];
+            uint32_t slow = 0;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) fast &= quant_fast(hv[e], rs_out, qv[e]);
-            if (!fast) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) qv[e] = quant_one(hv[e], p.s_out, rs_out);
+            for (int jj = 0; jj < 4; ++jj) {
+              const int j = 4 * hf + jj;
+              const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
+              const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
+              h[2 * jj] = __floats2half2_rn(fmaf(__uint_as_float(r[4 * j + 0]), sc.x, bi.x),
+                                            fmaf(__uint_as_float(r[4 * j + 1]), sc.y, bi.y));
+              h[2 * jj + 1] = __floats2half2_rn(fmaf(__uint_as_float(r[4 * j + 2]), sc.z, bi.z),
+                                                fmaf(__uint_as_float(r[4 * j + 3]), sc.w, bi.w));
+              const float2 x01 = __half22float2(h[2 * jj]);
+              const float2 x23 = __half22float2(h[2 * jj + 1]);
+              slow |= quant_fast_bits(x01.x, rs_out, qb[4 * jj + 0]) ? 0u : 1u << (4 * jj + 0);
+              slow |= quant_fast_bits(x01.y, rs_out, qb[4 * jj + 1]) ? 0u : 1u << (4 * jj + 1);
+              slow |= quant_fast_bits(x23.x, rs_out, qb[4 * jj + 2]) ? 0u : 1u << (4 * jj + 2);
+              slow |= quant_fast_bits(x23.y, rs_out, qb[4 * jj + 3]) ? 0u : 1u << (4 * jj + 3);
             }
-            wq[j] = (static_cast<uint32_t>(qv[0]) & 0xFFu) |
-                    ((static_cast<uint32_t>(qv[1]) & 0xFFu) << 8) |
-                    ((static_cast<uint32_t>(qv[2]) & 0xFFu) << 16) |
-                    (static_cast<uint32_t>(qv[3]) << 24);
+            quant_fix16(slow, h, qb, p.s_out, rs_out);
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj)
+              wq[4 * hf + jj] = pack_low_bytes(qb[4 * jj], qb[4 * jj + 1], qb[4 * jj + 2], qb[4 * jj + 3]);
           }
           uint4* row = reinterpret_cast<uint4*>(dst + lane * 32);
           row[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
@@ -834,7 +841,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
     if (e != cudaSuccess) return e;
     configured_bytes = static_cast<int>(bytes);
   }
-  // the decoder warps (10..17) exist only on the fused path
+  // the decoder warps (10..15) exist only on the fused path
   const int threads = p.fused ? kThreads : kThreads - kDecodeThreads;
   if (!p.cluster)
     return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);

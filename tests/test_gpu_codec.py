@@ -42,6 +42,20 @@ def test_quant_act_special_values():
     assert np.array_equal(xq.cpu().numpy(), O.quant_act(x, 0.5))
 
 
+@pytest.mark.parametrize("s_x", [0.05, 0.02, 0.1, 0.125, 1.0, 0.0473, 0.0387, 7.3e-3,
+                                 1.1920929e-07, 300.0])
+def test_quant_act_every_f16_value(s_x):
+    """All 65536 fp16 bit patterns (ties of x / s are exact for scales with few
+    significant bits, e.g. 0.05 at x = 0.875), bit-exact against the rule."""
+    import torch
+    import paper_2506_05960_gb300 as aq
+    x = np.arange(65536, dtype=np.uint16).view(np.float16)
+    x = np.concatenate([x, x[::-1]])          # each value in several lanes / positions
+    xq = torch.empty(x.size, dtype=torch.int8, device="cuda")
+    aq.aq_quant_act(dev(x), xq, x.size, float(np.float32(s_x)))
+    assert np.array_equal(xq.cpu().numpy(), O.quant_act(x, float(np.float32(s_x))))
+
+
 @pytest.mark.parametrize("N,K,M,B", [(256, 256, 2, 8), (37, 200, 3, 8), (8, 64, 8, 8),
                                      (960, 8640, 1, 16), (24, 72, 2, 16), (5, 8, 1, 8)])
 def test_pack_bit_exact(N, K, M, B):

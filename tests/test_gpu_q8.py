@@ -34,7 +34,7 @@ def _check(q, q_chain, y64, s_out):
     assert np.abs(q.astype(np.int32) - ref.astype(np.int32)).max() <= 1
 
 
-def _linear_pair(inp, path):
+def _linear_pair(inp, path, s_out=None):
     import torch
     import paper_2506_05960_gb300 as aq
     xq = inp["xq"]
@@ -48,7 +48,8 @@ def _linear_pair(inp, path):
     y16 = torch.empty((T, N), dtype=torch.float16, device="cuda")
     aq.aq_linear(*args, y16, aq.AQ_DTYPE_F16, T, K, N, 8, M, B, ws, ws_bytes, path)
     y64 = O.layer_f64(inp)
-    s_out = _s_out(y64)
+    if s_out is None:
+        s_out = _s_out(y64)
     q_chain = torch.empty((T, N), dtype=torch.int8, device="cuda")
     aq.aq_quant_act(y16, q_chain, T * N, s_out)
     q = torch.full((T, N), 99, dtype=torch.int8, device="cuda")
@@ -69,6 +70,18 @@ def test_linear_q8_equals_chain(T, K, N, M, B, path):
     inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=B, cb_std=0.05 / M ** 0.5),
                       seed=T + K + N + M + path)
     _check(*_linear_pair(inp, path))
+
+
+@pytest.mark.parametrize("s_out", [0.05, 0.125, 0.02, 0.0473])
+@pytest.mark.parametrize("path", [DENSE, FUSED])
+def test_linear_q8_scales_with_exact_ties(s_out, path):
+    """Scales with few significant bits make x / s_out an exact half-integer for many
+    fp16 outputs (0.05 at x = 0.875): the epilogue's exact tie handling must still give
+    the chain's bits."""
+    inp = make_linear(LinearSpec(T=512, K=512, N=1024, M=2, B=8, cb_std=0.05 / 2 ** 0.5),
+                      seed=int(s_out * 1e4) + path)
+    q, q_chain, y64, s = _linear_pair(inp, path, s_out=float(np.float32(s_out)))
+    assert np.array_equal(q, q_chain)
 
 
 @pytest.mark.parametrize("cfg,path", [(2, AUTO), (3, AUTO)])
