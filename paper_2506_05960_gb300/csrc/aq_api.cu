@@ -118,7 +118,8 @@ constexpr int kPlanMaxClusters[aq::kMaxClusterSplits + 1] = {0, 152, 76, 46, 36,
 struct Plan {
   int BN, n_tiles, m_tiles, splits, kb_per_split, num_kb;
   int stages, a_stages, acc_stride, a_col, total_tiles;
-  int cluster;  // the splits of a tile form one cluster and are summed in shared memory
+  int cluster;    // the splits of a tile form one cluster and are summed in shared memory
+  int epi_warps;  // 4, or 8 on the dense path with fp16/int8 staging and BN >= 64
 };
 
 // Cycles of one pipeline stage (eight 128 x BN x 16 MMAs issued by one thread),
@@ -155,11 +156,15 @@ bool plan_f32_staging(const Plan& pl, bool f32_out) {
   return f32_out || (pl.splits > 1 && !pl.cluster);
 }
 
-void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes) {
+void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes, bool fused) {
   pl.acc_stride = pl.BN;
   pl.a_col = 2 * pl.acc_stride;
   pl.a_stages = aq::gemm_a_stages(pl.BN);
-  pl.stages = aq::gemm_max_stages(pl.BN, plan_f32_staging(pl, f32_out), book_bytes, code_bytes);
+  const bool f32_staging = plan_f32_staging(pl, f32_out);
+  // the dense path has no decoder warps: 8 epilogue warps double the epilogue's rate,
+  // which bounds tiles with small K; fp32 staging would cost a pipeline stage
+  pl.epi_warps = (!fused && !f32_staging && pl.BN >= 64) ? 8 : 4;
+  pl.stages = aq::gemm_max_stages(pl.BN, f32_staging, book_bytes, code_bytes, pl.epi_warps);
   pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
 }
 
@@ -194,7 +199,7 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
       if (BN == 224) continue;
       if (forced && ov.BN > 0 && BN != ov.BN) continue;
       if (aq::gemm_a_stages(BN) < 2) continue;
-      if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes) < 2) continue;
+      if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes, 4) < 2) continue;
       const int n_tiles = (N + BN - 1) / BN;
       const int max_split = allow_split ? std::min(num_kb, 64) : 1;
       double st_cyc = stage_cycles(BN);
@@ -237,7 +242,7 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
   };
   if (ov.BN > 0 || ov.splits > 0 || ov.cluster >= 0) search(true);
   if (best > 1e29) search(false);
-  finish_plan(bp, f32_out, book_bytes, code_bytes);
+  finish_plan(bp, f32_out, book_bytes, code_bytes, fused);
   return bp;
 }
 
@@ -515,6 +520,7 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   p.acc_stride = pl.acc_stride;
   p.a_col = pl.a_col;
   p.cluster = pl.cluster;
+  p.epi_warps = pl.epi_warps;
   p.partial = (pl.splits > 1 && !pl.cluster) ? partial : nullptr;
   const int T = p.T, N = p.N, K = p.K;
   int r;

@@ -33,14 +33,14 @@ __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict
     // all 16 values on the fast path (FMA/ALU pipes, straight-line); a value near a tie
     // is redone alone with the exact rule
     uint32_t qb[16];
-    uint32_t slow = 0;
+    bool fast = true;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const float2 xf = __half22float2(h[i]);
-      slow |= quant_fast_bits(xf.x, rs, qb[2 * i]) ? 0u : 1u << (2 * i);
-      slow |= quant_fast_bits(xf.y, rs, qb[2 * i + 1]) ? 0u : 1u << (2 * i + 1);
+      fast &= quant_fast_bits(xf.x, rs, qb[2 * i]);
+      fast &= quant_fast_bits(xf.y, rs, qb[2 * i + 1]);
     }
-    quant_fix16(slow, h, qb, s, rs);
+    if (!fast) quant_fix16(h, qb, s, rs);
     uint32_t w[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i)

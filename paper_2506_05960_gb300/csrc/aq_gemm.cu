@@ -7,7 +7,8 @@
 //
 // Persistent kernel, one CTA per SM, static round-robin over 128 x BN output
 // tiles (and K splits).  A pipeline stage covers 128 of K (two 64-wide TMA
-// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps (sixteen on the fused path):
+// boxes per operand, eight 128 x BN x 16 MMAs).  Ten warps, fourteen on the dense path
+// with 8 epilogue warps, sixteen on the fused path:
 //   warp 0      TMA producer: int8 activation boxes (64-byte swizzle) and fp16
 //               weight boxes (128-byte swizzle) into an S-deep smem ring
 //   warp 1      TMEM owner (all 512 columns) and the single MMA-issuing thread:
@@ -18,9 +19,12 @@
 //   warps 2..5  converters: int8 rows -> fp16 exactly -> tcgen05.st into a
 //               TMEM A ring (no shared-memory round trip for the fp16 operand)
 //   warps 6..9  epilogue: TMEM accumulator -> scale/bias -> 32 x 32 boxes in
-//               shared memory -> TMA stores (ragged edges clipped by TMA).  The
+//   (6..13)     shared memory -> TMA stores (ragged edges clipped by TMA).  The
 //               output is fp16, fp32, or int8: the fp16 value quantized with the
-//               next layer's activation scale (the quantizer fused into the layer)
+//               next layer's activation scale (the quantizer fused into the layer).
+//               A warp reads only its TMEM lane quarter (warp % 4), so 8 epilogue
+//               warps pair up per quarter and take alternate 32-column chunks: with
+//               small K the epilogue, not the mainloop, bounds a tile.
 //   warps 10..15 (fused path) decoders: rebuild each weight stage from the packed
 //               codes and the shared-memory codebooks (Eq. 4).  The lookups are
 //               bound by shared-memory bandwidth, hence six warps and the
@@ -50,7 +54,11 @@ constexpr int kA8Stage = kStageBlocks * kA8Half;
 constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A slot
 constexpr int kEpiBuf32 = 4096;                 // one 32 x 32 fp32 output box (128-byte rows)
 constexpr int kEpiBuf16 = 2048;                 // one 32 x 32 fp16 output box (64-byte rows)
-constexpr int kScaleBytes = 4 * 2 * kMaxBN * 4; // per epilogue warp: scale and bias of a tile
+// Epilogue staging per warp: 4 warps keep two output boxes and the scale/bias of all BN
+// columns each; 8 warps (two per lane quarter, alternate 32-column chunks) keep one box
+// and the scale/bias of their own columns, so both take the same shared memory.
+__host__ __device__ constexpr int epi_out_bufs(int epi_warps) { return epi_warps == 8 ? 1 : 2; }
+__host__ __device__ constexpr int epi_scale_cols(int epi_warps) { return kMaxBN / (epi_warps / 4); }
 constexpr int kTmemCols = 512;
 
 struct alignas(8) GemmBarriers {
@@ -59,7 +67,7 @@ struct alignas(8) GemmBarriers {
   uint32_t a_ready[kMaxStages];  // fp16 A slot written: +1 per converter warp (4 per use)
   uint64_t a_empty[kMaxStages];  // MMAs reading the TMEM slot done (commit)
   uint64_t acc_full[2];          // accumulator buffer complete (commit)
-  uint64_t acc_empty[2];         // accumulator buffer drained (4 epilogue warps)
+  uint64_t acc_empty[2];         // accumulator buffer drained (one arrival per epilogue warp)
   uint64_t drain;                // all MMAs of this CTA complete (teardown)
   uint64_t codes_full[kMaxStages];  // fused path: a stage's packed codes landed in smem
   uint32_t tmem_base;
@@ -68,16 +76,18 @@ struct alignas(8) GemmBarriers {
 
 // code_bytes: packed code bytes of one row for one 64-wide K block on the fused path
 // (8 * M * bytes per code), 0 on the dense path.
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes) {
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes,
+                       int epi_warps) {
   return 1024 +
          static_cast<size_t>(stages) *
              (kStageBlocks * BN * 128 + kA8Stage + kStageBlocks * BN * code_bytes) +
-         4 * 2 * (f32_out ? kEpiBuf32 : kEpiBuf16) + kScaleBytes + book_bytes +
-         sizeof(GemmBarriers);
+         static_cast<size_t>(epi_warps) * (epi_out_bufs(epi_warps) * (f32_out ? kEpiBuf32 : kEpiBuf16) +
+                                           2 * epi_scale_cols(epi_warps) * 4) +
+         book_bytes + sizeof(GemmBarriers);
 }
 
-int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes) {
-  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes, code_bytes);
+int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes, int epi_warps) {
+  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes, code_bytes, epi_warps);
   const size_t per = static_cast<size_t>(kStageBlocks) * BN * (128 + code_bytes) + kA8Stage;
   const int s = static_cast<int>((232448 - fixed) / per);
   return s < kMaxStages ? s : kMaxStages;
@@ -312,8 +322,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* bring = smem;
   uint8_t* aring = bring + S * b_stage;
   uint8_t* epi = aring + S * kA8Stage;
-  float* sscale = reinterpret_cast<float*>(epi + 4 * 2 * epi_buf);
-  uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) + kScaleBytes);
+  const int EW = p.epi_warps;                  // 4, or 8 (two per TMEM lane quarter)
+  float* sscale = reinterpret_cast<float*>(epi + EW * epi_out_bufs(EW) * epi_buf);
+  uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) +
+                                          EW * 2 * epi_scale_cols(EW) * 4);
   // fused path: each stage's packed codes, [h][BN rows][code_bytes] (16-byte aligned)
   const int code_bytes = p.fused ? 8 * p.M * (p.B >> 3) : 0;
   const int code_stage = kStageBlocks * BN * code_bytes;
@@ -338,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar->acc_full[b], 1);
-      mbar_init(&bar->acc_empty[b], 4);
+      mbar_init(&bar->acc_empty[b], EW);
     }
     mbar_init(&bar->drain, 1);
     for (int s = 0; s < S; ++s) mbar_init(&bar->codes_full[s], 1);
@@ -545,13 +557,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         ra.next(SA);
       }
     }
-  } else if (warp < 10) {
+  } else if (warp < 6 + EW) {
     // ================================================================ epilogue
     const int q = warp & 3;
     const int ew = warp - 6;
-    float* wscale = sscale + ew * 2 * kMaxBN;
-    float* wbias = wscale + kMaxBN;
-    uint8_t* wbuf = epi + ew * 2 * epi_buf;
+    // with 8 epilogue warps the two warps of a lane quarter take alternate 32-column chunks
+    const int c_first = 32 * (ew >> 2);
+    const int c_step = 32 * (EW >> 2);
+    const int wcols = epi_scale_cols(EW);    // this warp's chunks' columns, compacted
+    const int nbuf = epi_out_bufs(EW);
+    float* wscale = sscale + ew * 2 * wcols;
+    float* wbias = wscale + wcols;
+    uint8_t* wbuf = epi + ew * nbuf * epi_buf;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
     const float rs_out = p.out_q8 ? __frcp_rn(p.s_out) : 0.0f;
     uint32_t lt = 0, chunk = 0;
@@ -562,10 +579,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int n0 = tc.n_tile * BN;
       if (!raw && !p.cluster) {
         // this tile's scale/bias, loaded while the accumulator is still being computed
-        for (int i = lane; i < BN; i += 32) {
-          const int n = n0 + i;
-          wscale[i] = (n < p.N) ? p.s_x * __half2float(p.scale[n]) : 0.0f;
-          wbias[i] = (n < p.N && p.bias != nullptr) ? __half2float(p.bias[n]) : 0.0f;
+        for (int i = lane; i < wcols; i += 32) {
+          const int col = c_first + (i >> 5) * c_step + (i & 31);
+          const int n = n0 + col;
+          const bool in = col < BN && n < p.N;
+          wscale[i] = in ? p.s_x * __half2float(p.scale[n]) : 0.0f;
+          wbias[i] = (in && p.bias != nullptr) ? __half2float(p.bias[n]) : 0.0f;
         }
       }
       if (!mbar_wait(&bar->acc_full[buf], (lt >> 1) & 1u, abort_flag)) {
@@ -575,11 +594,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       __syncwarp();
       const uint32_t tacc = t_row + static_cast<uint32_t>(buf * p.acc_stride);
-      for (int c0 = 0; c0 < BN; c0 += 32, ++chunk) {
+      int kc = 0;   // chunk index of this warp within the tile
+      for (int c0 = c_first; c0 < BN; c0 += c_step, ++chunk, ++kc) {
+        const float* csc = wscale + kc * 32;
+        const float* cbi = wbias + kc * 32;
         uint32_t r[32];
         tmem_ld_32x32b_x32(tacc + static_cast<uint32_t>(c0), r);
         tmem_wait_ld();
-        if (c0 + 32 >= BN) {
+        if (c0 + c_step >= BN) {
           // last read of this accumulator buffer: hand it back to the MMA warp
           tc_fence_before();
           __syncwarp();
@@ -598,8 +620,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                             __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
           continue;
         }
-        uint8_t* dst = wbuf + (chunk & 1u) * epi_buf;
-        if (lane == 0) bulk_wait_group_read<1>();   // the store issued from dst two chunks ago
+        uint8_t* dst = wbuf + (nbuf == 2 ? (chunk & 1u) * epi_buf : 0u);
+        if (lane == 0) {
+          // the store that last read dst: two chunks ago (two buffers) or the previous one
+          if (nbuf == 2)
+            bulk_wait_group_read<1>();
+          else
+            bulk_wait_group_read<0>();
+        }
         __syncwarp();
         if (f32) {
 #pragma unroll
@@ -610,8 +638,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             o.z = __uint_as_float(r[4 * j + 2]);
             o.w = __uint_as_float(r[4 * j + 3]);
             if (!raw) {
-              const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
-              const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
+              const float4 sc = *reinterpret_cast<const float4*>(csc + 4 * j);
+              const float4 bi = *reinterpret_cast<const float4*>(cbi + 4 * j);
               o.x = fmaf(o.x, sc.x, bi.x);
               o.y = fmaf(o.y, sc.y, bi.y);
               o.z = fmaf(o.z, sc.z, bi.z);
@@ -632,24 +660,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int hf = 0; hf < 2; ++hf) {
             __half2 h[8];
             uint32_t qb[16];
-            uint32_t slow = 0;
+            bool fast = true;
 #pragma unroll
             for (int jj = 0; jj < 4; ++jj) {
               const int j = 4 * hf + jj;
-              const float4 sc = *reinterpret_cast<const float4*>(wscale + c0 + 4 * j);
-              const float4 bi = *reinterpret_cast<const float4*>(wbias + c0 + 4 * j);
+              const float4 sc = *reinterpret_cast<const float4*>(csc + 4 * j);
+              const float4 bi = *reinterpret_cast<const float4*>(cbi + 4 * j);
               h[2 * jj] = __floats2half2_rn(fmaf(__uint_as_float(r[4 * j + 0]), sc.x, bi.x),
                                             fmaf(__uint_as_float(r[4 * j + 1]), sc.y, bi.y));
               h[2 * jj + 1] = __floats2half2_rn(fmaf(__uint_as_float(r[4 * j + 2]), sc.z, bi.z),
                                                 fmaf(__uint_as_float(r[4 * j + 3]), sc.w, bi.w));
               const float2 x01 = __half22float2(h[2 * jj]);
               const float2 x23 = __half22float2(h[2 * jj + 1]);
-              slow |= quant_fast_bits(x01.x, rs_out, qb[4 * jj + 0]) ? 0u : 1u << (4 * jj + 0);
-              slow |= quant_fast_bits(x01.y, rs_out, qb[4 * jj + 1]) ? 0u : 1u << (4 * jj + 1);
-              slow |= quant_fast_bits(x23.x, rs_out, qb[4 * jj + 2]) ? 0u : 1u << (4 * jj + 2);
-              slow |= quant_fast_bits(x23.y, rs_out, qb[4 * jj + 3]) ? 0u : 1u << (4 * jj + 3);
+              fast &= quant_fast_bits(x01.x, rs_out, qb[4 * jj + 0]);
+              fast &= quant_fast_bits(x01.y, rs_out, qb[4 * jj + 1]);
+              fast &= quant_fast_bits(x23.x, rs_out, qb[4 * jj + 2]);
+              fast &= quant_fast_bits(x23.y, rs_out, qb[4 * jj + 3]);
             }
-            quant_fix16(slow, h, qb, p.s_out, rs_out);
+            if (!fast) quant_fix16(h, qb, p.s_out, rs_out);
 #pragma unroll
             for (int jj = 0; jj < 4; ++jj)
               wq[4 * hf + jj] = pack_low_bytes(qb[4 * jj], qb[4 * jj + 1], qb[4 * jj + 2], qb[4 * jj + 3]);
@@ -660,10 +688,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            const float4 sc0 = *reinterpret_cast<const float4*>(wscale + c0 + 8 * j);
-            const float4 sc1 = *reinterpret_cast<const float4*>(wscale + c0 + 8 * j + 4);
-            const float4 bi0 = *reinterpret_cast<const float4*>(wbias + c0 + 8 * j);
-            const float4 bi1 = *reinterpret_cast<const float4*>(wbias + c0 + 8 * j + 4);
+            const float4 sc0 = *reinterpret_cast<const float4*>(csc + 8 * j);
+            const float4 sc1 = *reinterpret_cast<const float4*>(csc + 8 * j + 4);
+            const float4 bi0 = *reinterpret_cast<const float4*>(cbi + 8 * j);
+            const float4 bi1 = *reinterpret_cast<const float4*>(cbi + 8 * j + 4);
             const float* rr = reinterpret_cast<const float*>(r) + 8 * j;
             __half2 h0 = __floats2half2_rn(fmaf(rr[0], sc0.x, bi0.x), fmaf(rr[1], sc0.y, bi0.y));
             __half2 h1 = __floats2half2_rn(fmaf(rr[2], sc0.z, bi0.z), fmaf(rr[3], sc0.w, bi0.w));
@@ -834,7 +862,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
   static int configured_bytes = 0;
   const size_t bytes =
       gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes,
-                      p.fused ? 8 * p.M * (p.B >> 3) : 0);
+                      p.fused ? 8 * p.M * (p.B >> 3) : 0, p.epi_warps);
   if (static_cast<int>(bytes) > configured_bytes) {
     cudaError_t e = cudaFuncSetAttribute(aq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(bytes));
@@ -842,7 +870,9 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
     configured_bytes = static_cast<int>(bytes);
   }
   // the decoder warps (10..15) exist only on the fused path
-  const int threads = p.fused ? kThreads : kThreads - kDecodeThreads;
+  if (p.epi_warps != 4 && !(p.epi_warps == 8 && !p.fused && p.BN >= 64))
+    return cudaErrorInvalidConfiguration;
+  const int threads = p.fused ? kThreads : 32 * (6 + p.epi_warps);
   if (!p.cluster)
     return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
   // in-cluster split-K: one CTA per (tile, split), the splits of a tile in one cluster

@@ -48,6 +48,7 @@ struct GemmParams {
   int out_q8;                   // int8 output: the next layer's activations, quantized with s_out
   float s_out;
   float* partial;               // split-K partial sums [splits][T][N] (null: fused epilogue)
+  int epi_warps;                // epilogue warps: 4, or 8 on the dense path (BN >= 64)
   int cluster;                  // 1: the splits of a tile form one thread-block cluster (split =
                                 // cluster rank) and are summed through distributed shared
                                 // memory; grid = total_tiles, one tile per CTA
@@ -124,8 +125,10 @@ cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int
                               int B, cudaStream_t st);
 // code_bytes: packed code bytes per row and 64-wide K block staged per stage on
 // the fused path (8 * M * bytes per code), 0 on the dense path.
-size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes);
-int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes);  // ring depth that fits
+size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes,
+                       int epi_warps);
+int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes,
+                    int epi_warps);              // ring depth that fits
 int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-column accumulators
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st);

@@ -23,36 +23,50 @@ __device__ __forceinline__ int8_t quant_one(__half h, float s, float rs) {
   return static_cast<int8_t>(static_cast<int>(q));
 }
 
-// The fast path on the FMA/ALU pipes only (no conversion-unit instructions), for an
-// fp16 value already widened to fp32: q = x * fl(1/s) is clipped to [-127, 127] first
-// (for that range clip-then-round equals round-then-clip) and rounded half to even by
-// adding 1.5 * 2^23, which leaves the integer in the low bits of the sum: the low byte
-// of `bits` is the int8 code.
-// When is rint(q) the rule's rint(fl(x / s))?  With u = 2^-24, fl(1/s) and the product
-// each add a relative error of at most u, and fl(x / s) one more, so
-// |q - fl(x / s)| <= |q| * (3u + u^2) / (1 - 2u - u^2) < 4u |q|.  If q is farther than
-// that from every half-integer, both round to the same integer.  The test
-// |q - rint(q)| < 1/2 - 4u |q| is evaluated with an exact subtraction and a threshold
-// whose rounding (<= 2^-26) stays below the margin u |q| for |q| >= 1/4; below 1/4 the
-// nearest half-integer is more than 1/4 away and the answer is 0 either way.  Returns
-// false for a NaN or a value that fails the test: the caller applies quant_one.
-__device__ __forceinline__ bool quant_fast_bits(float x, float rs, uint32_t& bits) {
-  constexpr float kRound = 12582912.0f;        // 1.5 * 2^23
-  constexpr float kFourU = 2.384185791015625e-7f;  // 2^-22
-  const float q = x * rs;
-  const float qc = fminf(fmaxf(q, -127.0f), 127.0f);
-  const float t = __fadd_rn(qc, kRound);
-  bits = __float_as_uint(t);
-  const float thr = __fmaf_rn(-fabsf(qc), kFourU, 0.5f);
-  return fabsf(__fsub_rn(qc, __fsub_rn(t, kRound))) < thr && q == q;
+// Clip to [-127, 127] keeping NaN (min/max with .NaN propagate it).
+__device__ __forceinline__ float clip127_keep_nan(float q) {
+  float r;
+  asm("max.NaN.f32 %0, %1, 0fC2FE0000;\n\tmin.NaN.f32 %0, %0, 0f42FE0000;" : "=f"(r) : "f"(q));
+  return r;
 }
 
-// Redoes the values of a group of 16 that quant_fast_bits rejected (bit i of `slow`:
-// value i, the half (i & 1) of h[i >> 1]) with the exact rule, one value per lane per
-// round: the warp runs as many rounds as its busiest lane has rejected values (the
-// selects keep h and qb in registers).
-__device__ __forceinline__ void quant_fix16(uint32_t slow, const __half2 (&h)[8],
-                                            uint32_t (&qb)[16], float s, float rs) {
+// The fast path on the FMA/ALU pipes only (no conversion-unit instructions), for an
+// fp16 value already widened to fp32.
+// Error bound: with u = 2^-24, fl(1/s) and the product x * fl(1/s) each add a relative
+// error of at most u, and fl(x / s) one more, so q = x * fl(1/s) satisfies
+// |q - fl(x / s)| <= |q| * (3u + u^2) / (1 - 2u - u^2) < 4u |q| = 2^-22 |q|.
+// Test: q is clipped to [-127, 127] (for that range clip-then-round equals
+// round-then-clip), and qc * (1 - 2^-22) and qc * (1 + 2^-22), which bracket fl(x / s),
+// are rounded half to even with one FMA each by adding 1.5 * 2^23 (exact products, one
+// rounding at integer spacing).  Rounding is monotonic, so if both ends give the same
+// integer, so does fl(x / s): that integer is the code, in the low byte of `bits`.  The
+// ends differ near a half-integer (the caller then applies quant_one), and a NaN fails
+// the equality.
+__device__ __forceinline__ bool quant_fast_bits(float x, float rs, uint32_t& bits) {
+  constexpr float kRound = 12582912.0f;             // 1.5 * 2^23
+  constexpr float kUp = 1.0000002384185791015625f;   // 1 + 2^-22
+  constexpr float kDown = 0.999999761581420898437f;  // 1 - 2^-22
+  const float qc = clip127_keep_nan(x * rs);
+  const float hi = __fmaf_rn(qc, kUp, kRound);
+  const float lo = __fmaf_rn(qc, kDown, kRound);
+  bits = __float_as_uint(hi);
+  return hi == lo;
+}
+
+// Redoes, with the exact rule, the values of a group of 16 (value i: the half (i & 1) of
+// h[i >> 1]) that quant_fast_bits rejects, one value per lane per round: the warp runs
+// as many rounds as its busiest lane has rejected values (the selects keep h and qb in
+// registers).
+__device__ __forceinline__ void quant_fix16(const __half2 (&h)[8], uint32_t (&qb)[16], float s,
+                                            float rs) {
+  uint32_t slow = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float2 xf = __half22float2(h[i]);
+    uint32_t unused;
+    slow |= quant_fast_bits(xf.x, rs, unused) ? 0u : 1u << (2 * i);
+    slow |= quant_fast_bits(xf.y, rs, unused) ? 0u : 1u << (2 * i + 1);
+  }
   while (slow) {
     const int i = __ffs(slow) - 1;
     slow &= slow - 1;
