@@ -43,8 +43,11 @@ _SIGNATURES = {
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
     "aq_set_plan_override": (_c_int, [_c_int] * 3),
+    "aq_linear_f16_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_linear_f16": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
+                      + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_linear_noalloc": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                           + [_c_void_p]),
     "aq_linear_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float] + [_c_int] * 6
@@ -210,6 +213,22 @@ def aq_linear(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K,
         _ptr(xq), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
         _ptr(y), out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
         _stream(stream)), "aq_linear")
+
+
+def aq_linear_f16_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_linear_f16_workspace_size(T, K, N, g, M, B, path, ctypes.byref(out)),
+           "aq_linear_f16_workspace_size")
+    return out.value
+
+
+def aq_linear_f16(x, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N, g=8, M=2,
+                  B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """aq_quant_act + aq_linear in one call from fp16 activations x (int8 kept in workspace)."""
+    _check(load_library().aq_linear_f16(
+        _ptr(x), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(y), out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
+        _stream(stream)), "aq_linear_f16")
 
 
 def aq_linear_q8(xq, s_x, codes_packed, codebooks, scale, bias, yq, s_out, T, K, N, g=8, M=2,

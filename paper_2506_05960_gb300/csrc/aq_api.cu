@@ -498,9 +498,12 @@ int sm_count() {
 // workspace (Wdec), then the GEMM streams it with TMA.  Fused (Wdec == nullptr): the
 // GEMM's decoder warps rebuild each weight tile in shared memory from the codes.
 // kaq: the codes use the kernel-aware grouping (g = 9, dense path only).
+// x16 != nullptr: the layer's fp16 activations, quantized here into the GEMM's int8
+// operand xq (the memory mapA points at) with the rule of aq_quant_act and scale p.s_x;
+// on the dense path in the same launch as the decode.
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
-             bool kaq = false) {
+             bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr) {
   const bool fused = Wdec == nullptr;
   p.fused = fused ? 1 : 0;
   p.codes = codes_packed;
@@ -562,10 +565,21 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   }
   if (r) return r;
   cudaError_t e;
+  const int64_t x_elems = static_cast<int64_t>(T) * K;
+  if (x16 && (fused || kaq)) {
+    ProfScope ps(kProfQuant, st);
+    e = aq::launch_quant_act(x16, xq, x_elems, p.s_x, st);
+    if (e != cudaSuccess) return cuda_status(e, "quantizer launch");
+  }
   if (!fused) {
     ProfScope ps(kProfDecode, st);
-    e = kaq ? aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st)
-            : aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+    if (kaq)
+      e = aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st);
+    else if (x16)
+      e = aq::launch_quant_decode(x16, xq, x_elems, p.s_x, codes_packed, codebooks, Wdec, N, K,
+                                  M, B, st);
+    else
+      e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
     if (e != cudaSuccess) return cuda_status(e, "decode launch");
   }
   {
@@ -643,7 +657,7 @@ int check_output(int out_dtype, float s_out, int N) {
 int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
                 const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
                 int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
-                int path, void* stream);
+                int path, void* stream, const void* x16 = nullptr);
 int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
@@ -865,14 +879,51 @@ int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed, const vo
                      N, g, M, B, workspace, workspace_bytes, path, stream);
 }
 
+// aq_linear from fp16 activations: the workspace starts with the int8 activations
+// (T*K bytes, 1 KB-aligned), then what aq_linear needs.
+static size_t f16_act_bytes(int T, int K) { return align_up(static_cast<size_t>(T) * K, 1024); }
+
+int aq_linear_f16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
+                                 size_t* bytes) {
+  size_t rest = 0;
+  const int r = aq_linear_workspace_size(T, K, N, g, M, B, path, &rest);
+  if (r) return r;
+  *bytes = f16_act_bytes(T, K) + rest;
+  return ok();
+}
+
+int aq_linear_f16(const void* x, float s_x, const void* codes_packed, const void* codebooks,
+                  const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
+                  int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
+                  void* stream) {
+  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  if (!(s_x > 0.0f) || s_x == __builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite and > 0");
+  if (T < 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and K > 0");
+  if (T == 0)  // argument checks only, as aq_linear
+    return linear_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, 0,
+                       K, N, g, M, B, workspace, workspace_bytes, path, stream);
+  if (!x) return set_error(AQ_ERR_NULL, "x is NULL");
+  if (!aligned16(x)) return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  const size_t xq_bytes = f16_act_bytes(T, K);
+  if (!workspace || workspace_bytes < xq_bytes || !aligned16(workspace))
+    return set_error(AQ_ERR_WORKSPACE, "workspace needs at least %zu bytes (got %zu)", xq_bytes,
+                     workspace_bytes);
+  int8_t* xq = static_cast<int8_t*>(workspace);
+  void* rest = static_cast<uint8_t*>(workspace) + xq_bytes;
+  return linear_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, T, K, N,
+                     g, M, B, rest, workspace_bytes - xq_bytes, path, stream, x);
+}
+
 }  // extern "C"
 
 namespace {
 
+// x16 != nullptr (aq_linear_f16): the fp16 activations, quantized into xq by this call.
 int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
                 const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
                 int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
-                int path, void* stream) {
+                int path, void* stream, const void* x16) {
   int r = check_format(g, M, B);
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
@@ -888,6 +939,13 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  if (x16 && (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT)) {
+    ProfScope ps(kProfQuant, static_cast<cudaStream_t>(stream));
+    const cudaError_t e = aq::launch_quant_act(x16, const_cast<int8_t*>(xq),
+                                               static_cast<int64_t>(T) * K, s_x,
+                                               static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_status(e, "quantizer launch");
+  }
   if (rp == AQ_PATH_FEW_TOKENS) {
     aq::SkinnyParams sp{};
     sp.xq = xq;
@@ -976,7 +1034,8 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
   p.out_q8 = out_dtype == AQ_DTYPE_I8;
   p.s_out = s_out;
-  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st);
+  return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st, false, x16,
+                  const_cast<int8_t*>(xq));
 }
 
 }  // namespace

@@ -3,6 +3,7 @@
 //   * code packing into the 64-wide-K-block layout
 //   * AQ decode (Sec. 2.4 Eq. 4): W-hat = sum of the selected codewords, fp32
 //     sum in ascending codebook order, one round to fp16.
+#include <algorithm>
 #include <cstdint>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -14,17 +15,15 @@
 namespace aq {
 
 // ============================================================== quantizer (rule in aq_quant.cuh)
-// Each thread: 16 elements (32 B in, 16 B out) per grid-stride step.
-__global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
-                                                        int8_t* __restrict__ xq,
-                                                        int64_t nvec, int64_t numel, float s) {
-  grid_dependency_wait();
-  allow_dependents();
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec;
-       v += stride) {
+// Each thread: 16 elements (32 B in, 16 B out) per grid-stride step over `nblocks` blocks
+// (block index `bid`); the first block also takes the scalar tail (numel % 16 elements).
+__device__ __forceinline__ void quant_range(const __half* __restrict__ x, int8_t* __restrict__ xq,
+                                            int64_t nvec, int64_t numel, float s, int bid,
+                                            int nblocks) {
+  const float rs = __frcp_rn(s);
+  const int64_t stride = static_cast<int64_t>(nblocks) * blockDim.x;
+  for (int64_t v = static_cast<int64_t>(bid) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
     const uint4* src = reinterpret_cast<const uint4*>(x) + 2 * v;
-    const float rs = __frcp_rn(s);
     uint4 a = __ldcs(src);
     uint4 b = __ldcs(src + 1);
     __half2 h[8];
@@ -47,11 +46,18 @@ __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict
       w[i] = pack_low_bytes(qb[4 * i], qb[4 * i + 1], qb[4 * i + 2], qb[4 * i + 3]);
     __stcs(reinterpret_cast<uint4*>(xq) + v, make_uint4(w[0], w[1], w[2], w[3]));
   }
-  // scalar tail (numel % 16 elements), handled by the first threads of block 0
-  if (blockIdx.x == 0) {
+  if (bid == 0) {
     for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x)
-      xq[i] = quant_one(x[i], s, __frcp_rn(s));
+      xq[i] = quant_one(x[i], s, rs);
   }
+}
+
+__global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
+                                                        int8_t* __restrict__ xq,
+                                                        int64_t nvec, int64_t numel, float s) {
+  grid_dependency_wait();
+  allow_dependents();
+  quant_range(x, xq, nvec, numel, s, blockIdx.x, gridDim.x);
 }
 
 cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s,
@@ -129,23 +135,18 @@ __device__ __forceinline__ uint4 narrow(const F8& acc) {
   return r;
 }
 
-// 8-bit codes: all M codebooks (M x 256 x 16 B <= 32 KB) staged in shared memory.
-// One thread per group: packed index idx = (kb*N + n)*8 + j is also the thread's
-// linear index, so code loads are contiguous across the warp and each group of 8
-// threads writes 128 contiguous bytes of W.
-__global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restrict__ packed,
-                                                        const uint4* __restrict__ books,
-                                                        __half* __restrict__ W, int N, int K,
-                                                        int M, int KB) {
-  extern __shared__ uint4 sbook[];                       // [M][256]
-  grid_dependency_wait();
-  allow_dependents();
-  for (int i = threadIdx.x; i < M * 256; i += blockDim.x) sbook[i] = books[i];
-  __syncthreads();
+// 8-bit codes: all M codebooks (M x 256 x 16 B <= 32 KB) staged in shared memory by the
+// caller.  One thread per group: packed index idx = (kb*N + n)*8 + j is also the
+// thread's linear index, so code loads are contiguous across the warp and each group of
+// 8 threads writes 128 contiguous bytes of W.
+__device__ __forceinline__ void decode_b8_range(const uint8_t* __restrict__ packed,
+                                                const uint4* sbook, __half* __restrict__ W,
+                                                int N, int K, int M, int KB, int bid,
+                                                int nblocks) {
   const int G = K / 8;
   const int64_t total = static_cast<int64_t>(KB) * N * 8;
-  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
-       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  for (int64_t idx = static_cast<int64_t>(bid) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(nblocks) * blockDim.x) {
     const int j = static_cast<int>(idx & 7);
     const int64_t rem = idx >> 3;
     const int kb = static_cast<int>(rem / N);
@@ -160,16 +161,14 @@ __global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restric
 }
 
 // 16-bit codes: codebooks (M x 65536 x 16 B) stay in global memory / L2.
-__global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restrict__ packed,
-                                                         const uint4* __restrict__ books,
-                                                         __half* __restrict__ W, int N, int K,
-                                                         int M, int KB) {
-  grid_dependency_wait();
-  allow_dependents();
+__device__ __forceinline__ void decode_b16_range(const uint16_t* __restrict__ packed,
+                                                 const uint4* __restrict__ books,
+                                                 __half* __restrict__ W, int N, int K, int M,
+                                                 int KB, int bid, int nblocks) {
   const int G = K / 8;
   const int64_t total = static_cast<int64_t>(KB) * N * 8;
-  for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
-       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  for (int64_t idx = static_cast<int64_t>(bid) * blockDim.x + threadIdx.x; idx < total;
+       idx += static_cast<int64_t>(nblocks) * blockDim.x) {
     const int j = static_cast<int>(idx & 7);
     const int64_t rem = idx >> 3;
     const int kb = static_cast<int>(rem / N);
@@ -182,6 +181,81 @@ __global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restr
       widen_add(acc, __ldg(books + (static_cast<int64_t>(m) << 16) + c[m]), m == 0);
     *reinterpret_cast<uint4*>(W + static_cast<int64_t>(n) * K + grp * 8) = narrow(acc);
   }
+}
+
+__device__ __forceinline__ void stage_books8(const uint4* __restrict__ books, uint4* sbook, int M) {
+  for (int i = threadIdx.x; i < M * 256; i += blockDim.x) sbook[i] = books[i];
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restrict__ packed,
+                                                        const uint4* __restrict__ books,
+                                                        __half* __restrict__ W, int N, int K,
+                                                        int M, int KB) {
+  extern __shared__ uint4 sbook[];                       // [M][256]
+  grid_dependency_wait();
+  allow_dependents();
+  stage_books8(books, sbook, M);
+  decode_b8_range(packed, sbook, W, N, K, M, KB, blockIdx.x, gridDim.x);
+}
+
+__global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restrict__ packed,
+                                                         const uint4* __restrict__ books,
+                                                         __half* __restrict__ W, int N, int K,
+                                                         int M, int KB) {
+  grid_dependency_wait();
+  allow_dependents();
+  decode_b16_range(packed, books, W, N, K, M, KB, blockIdx.x, gridDim.x);
+}
+
+// The activation quantizer and the weight decode of one dense-path layer call in one
+// launch: they share no data, so blocks [0, qblocks) quantize and the rest decode, and
+// neither waits for the other.
+__global__ void __launch_bounds__(256) quant_decode_kernel(
+    const __half* __restrict__ x, int8_t* __restrict__ xq, int64_t nvec, int64_t numel, float s,
+    const void* __restrict__ packed, const uint4* __restrict__ books, __half* __restrict__ W,
+    int N, int K, int M, int B, int KB, int qblocks) {
+  extern __shared__ uint4 sbook[];                       // [M][256] for 8-bit codes
+  grid_dependency_wait();
+  allow_dependents();
+  if (static_cast<int>(blockIdx.x) < qblocks) {
+    quant_range(x, xq, nvec, numel, s, blockIdx.x, qblocks);
+    return;
+  }
+  const int bid = blockIdx.x - qblocks;
+  const int nb = gridDim.x - qblocks;
+  if (B == 8) {
+    stage_books8(books, sbook, M);
+    decode_b8_range(static_cast<const uint8_t*>(packed), sbook, W, N, K, M, KB, bid, nb);
+  } else {
+    decode_b16_range(static_cast<const uint16_t*>(packed), books, W, N, K, M, KB, bid, nb);
+  }
+}
+
+cudaError_t launch_quant_decode(const void* x, int8_t* xq, int64_t numel, float s,
+                                const void* packed, const void* books, void* W, int N, int K,
+                                int M, int B, cudaStream_t st) {
+  const int KB = (K + 63) / 64;
+  const int64_t nvec = numel / 16;
+  const int64_t groups = static_cast<int64_t>(KB) * N * 8;
+  // blocks in proportion to each side's bytes (48 per 16 activations, 18 per group),
+  // at most one resident wave of 256-thread blocks
+  int64_t qb = (nvec + 255) / 256;
+  int64_t db = (groups + 255) / 256;
+  const int64_t cap = 152 * 8;
+  if (qb + db > cap) {
+    const double qw = 48.0 * static_cast<double>(nvec);
+    const double dw = 18.0 * static_cast<double>(groups);
+    qb = std::min(qb, std::max<int64_t>(1, static_cast<int64_t>(cap * qw / (qw + dw))));
+    db = std::min(db, std::max<int64_t>(1, cap - qb));
+  }
+  if (qb < 1) qb = 1;
+  if (db < 1) db = 1;
+  const size_t smem = B == 8 ? static_cast<size_t>(M) * 256 * 16 : 0;
+  return launch_pdl(quant_decode_kernel, dim3(static_cast<unsigned>(qb + db)), dim3(256), smem, st,
+                    static_cast<const __half*>(x), xq, nvec, numel, s, packed,
+                    static_cast<const uint4*>(books), static_cast<__half*>(W), N, K, M, B, KB,
+                    static_cast<int>(qb));
 }
 
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
