@@ -193,6 +193,17 @@ __global__ void __launch_bounds__(512) decode_b8_kernel(const uint8_t* __restric
                                                         __half* __restrict__ W, int N, int K,
                                                         int M, int KB) {
   extern __shared__ uint4 sbook[];                       // [M][256]
+  if (threadIdx.x == 0) {
+    // the codes and books do not come from the previous kernel: this block's first codes
+    // start moving into L2 while it still runs (a hint, no effect on memory values)
+    const int64_t total = static_cast<int64_t>(KB) * N * 8 * M;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * blockDim.x * M;
+    const int64_t left = total - first;
+    const int64_t span = left < static_cast<int64_t>(blockDim.x) * M ? left : blockDim.x * M;
+    const uint32_t bytes = static_cast<uint32_t>(span > 0 ? span : 0) & ~15u;
+    if (bytes > 0) bulk_prefetch_l2(packed + first, bytes);
+    if (blockIdx.x == 0) bulk_prefetch_l2(books, static_cast<uint32_t>(M * 256 * 16));
+  }
   grid_dependency_wait();
   allow_dependents();
   stage_books8(books, sbook, M);

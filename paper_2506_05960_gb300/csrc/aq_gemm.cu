@@ -359,6 +359,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&mapA);
     if (!p.fused) tma_prefetch_desc(&mapB);
     tma_prefetch_desc(&mapY);
+    if (p.fused && blockIdx.x < p.total_tiles) {
+      // the weights do not come from the previous kernel: their first stages (and the
+      // 8-bit codebooks) start moving into L2 while it still runs
+      const TileCoord tc = tile_coord(p, blockIdx.x);
+      const int n0 = tc.n_tile * BN;
+      const int rows = min(BN, p.N - n0);
+      const int cb = 8 * p.M * (p.B >> 3);
+      const int kb_last = min(tc.kb_end, tc.kb_begin + kStageBlocks * S);
+      for (int kb = tc.kb_begin; kb < kb_last; ++kb)
+        bulk_prefetch_l2(static_cast<const uint8_t*>(p.codes) +
+                             (static_cast<int64_t>(kb) * p.N + n0) * cb,
+                         static_cast<uint32_t>(rows * cb));
+      if (p.book_bytes > 0) bulk_prefetch_l2(p.books, static_cast<uint32_t>(p.M * 256 * 16));
+    }
   }
   if (warp == 1) {
     tmem_alloc(&bar->tmem_base, kTmemCols);

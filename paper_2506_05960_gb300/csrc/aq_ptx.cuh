@@ -168,6 +168,12 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
 
 // Plain bulk copy global -> shared (both 16-byte aligned, size a multiple of 16),
 // completing bytes on an mbarrier.
+// Hint: bring [src, src + bytes) into L2 (16-byte aligned, bytes a multiple of 16).  No
+// effect on memory values, so it may be issued before the programmatic-launch wait.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
                                           uint64_t* bar) {
   asm volatile(
