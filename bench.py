@@ -401,6 +401,64 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False)
     return ms, gflop, len(layers)
 
 
+KERNEL_WORKLOADS = {
+    "quant": "aq_quant_act on the qkv input (4096 x 960 fp16)",
+    "decode": "aq_decode of the qkv weight (2880 x 960, 2x8)",
+    "quant_decode": "aq_linear_f16 on the qkv layer (quantizer + decode launch, then the GEMM)",
+    "fused128": "aq_linear, T=128 K=960 N=2880 2x8 (fused decode, K split in cluster)",
+    "few4": "aq_linear, T=4 K=960 N=2880 2x8 (few-token kernel)",
+    "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
+    "grad": "aq_codebook_grad of the qkv layer (fp32 G)",
+    "search": "aq_code_update of the qkv layer, both codebooks, unweighted",
+}
+
+
+def run_kernel_workload(args, aq, torch, dev, stream):
+    """One kernel's call on the seeded qkv-shaped layer, --warmup + --steps plain launches
+    (no graph), for ncu captures; returns the mean time per call (CUDA events)."""
+    from aq_synth import CONFIGS, LinearSpec, make_linear
+    w = args.workload
+    if w in ("fused128", "few4", "lut8"):
+        T = {"fused128": 128, "few4": 4, "lut8": 8}[w]
+        spec = LinearSpec(T=T, K=960, N=2880, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02)
+        L = Dev(aq, torch, make_linear(spec, seed=7), dev, path=3 if w == "lut8" else 0)
+        call = lambda: L.layer(stream)
+    else:
+        L = Dev(aq, torch, make_linear(CONFIGS[1], seed=1), dev)
+        N, K = L.N, L.K
+        if w == "quant":
+            call = lambda: L.quant(stream)
+        elif w == "decode":
+            wdec = torch.empty((N, K), dtype=torch.float16, device=dev)
+            call = lambda: L.decode_only(stream, wdec)
+        elif w == "quant_decode":
+            call = lambda: L.step_f16(stream)
+        elif w == "grad":
+            G = torch.randn((N, K), dtype=torch.float32, device=dev,
+                            generator=torch.Generator(device=dev).manual_seed(0))
+            dC = torch.zeros((2, 256, 8), dtype=torch.float32, device=dev)
+            call = lambda: aq.aq_codebook_grad(L.packed, G, L.scale, L.s_x, dC, N, K, 8, 2, 8,
+                                               stream=stream)
+        else:
+            Wt = torch.randn((N, K), dtype=torch.float32, device=dev,
+                             generator=torch.Generator(device=dev).manual_seed(0)) * 0.05
+            codes = torch.randint(0, 256, (N, K // 8, 2), dtype=torch.uint8, device=dev,
+                                  generator=torch.Generator(device=dev).manual_seed(1))
+            call = lambda: aq.aq_code_update(Wt, L.books, codes, None, 0, 2, N, K, 8, 2, 8,
+                                             stream=stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            call()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            call()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / max(1, args.steps)
+
+
 def run_single(args):
     """One non-headline workload on one GPU (profiling aid): prints its timing."""
     import torch
@@ -409,7 +467,11 @@ def run_single(args):
     dev = torch.device("cuda", 0)
     aq.load_library()
     stream = torch.cuda.Stream(device=dev)
-    if args.workload == "unet":
+    if args.workload in KERNEL_WORKLOADS:
+        ms = run_kernel_workload(args, aq, torch, dev, stream)
+        out = {"workload": KERNEL_WORKLOADS[args.workload], "us_per_call": ms * 1e3,
+               "timing": "plain launches, CUDA events (no graph)"}
+    elif args.workload == "unet":
         ms, gflop, nl = unet_forward(aq, torch, dev, stream, 2, reps=max(1, args.steps // 100))
         out = {"workload": "UNet-shaped forward W2A8 batch 2", "ms_per_forward": ms,
                "gflop": gflop, "layers": nl}
@@ -443,7 +505,8 @@ def main():
                     help="skip the other workloads and the UNet-shaped forward")
     ap.add_argument("--unet-batches", default="2,16,64",
                     help="batches of the UNet-shaped forward extras (comma separated)")
-    ap.add_argument("--workload", default="qkv", choices=["qkv", "conv64", "conv8", "unet"],
+    ap.add_argument("--workload", default="qkv",
+                    choices=["qkv", "conv64", "conv8", "unet"] + list(KERNEL_WORKLOADS),
                     help="qkv: the headline line (default); the others run only that workload "
                          "and print its timing (for profiling)")
     args = ap.parse_args()
