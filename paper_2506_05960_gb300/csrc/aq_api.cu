@@ -173,8 +173,7 @@ void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes, bool fu
 // the split-K reduction when K is split: either the partials' round trip through the
 // workspace and the reduce kernel (its launch waits for the GEMM to retire, about
 // 2 us), or, when all clusters of S <= 8 CTAs are resident at once, the in-cluster sum
-// through distributed shared memory (two cluster barriers and 128 x BN x 4 bytes per
-// CTA at about 64 B per cycle).  Depends only on the shapes (and, for the fused
+// through distributed shared memory.  Depends only on the shapes (and, for the fused
 // path, on the code format).
 // Diagnostic plan override of this host thread (aq_set_plan_override): N tile, K
 // splits, in-cluster sum (-1: free).  Plans the shapes cannot take are skipped and the
@@ -214,11 +213,22 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
         const double tile_cycles = (kbps / 2) * st_cyc + (kbps & 1) * 0.5 * st_cyc + 800.0;
         for (int cl = 0; cl < 2; ++cl) {
           if (forced && ov.cluster >= 0 && cl != ov.cluster) continue;
-          double t = static_cast<double>(waves) * tile_cycles / 1.9e9;
+          // Epilogue: about 900 cycles per 32-column chunk and epilogue warp group (4 warps;
+          // 8 on the dense path without fp32 staging).  It overlaps the next tile's
+          // mainloop (double-buffered accumulators), so a tile takes the longer of the two,
+          // and the last tile's epilogue adds to the end.  The same estimate for every output
+          // type keeps the plan, and so the workspace, independent of it.
+          const bool partials = s_eff > 1 && !cl;
+          const int ew = (!fused && !partials && BN >= 64) ? 8 : 4;
+          const double epi = (BN / 32.0) * 900.0 / (ew / 4);
+          double t = (static_cast<double>(waves) * std::max(tile_cycles, epi) + epi) / 1.9e9;
           if (cl) {
             if (s_eff < 2 || s_eff > aq::kMaxClusterSplits) continue;
             if (!forced && static_cast<long>(m_tiles) * n_tiles > kPlanMaxClusters[s_eff]) continue;
-            t = tile_cycles / 1.9e9 + (1000.0 + 128.0 * BN * 4.0 / 64.0) / 1.9e9;
+            // one tile per CTA; then the partial's shared-memory write, two cluster
+            // barriers and the 128 x BN x 4 bytes each CTA reads over distributed shared
+            // memory (about 3000 + 8 BN cycles measured on GB300 layers)
+            t = (tile_cycles + 3000.0 + 8.0 * BN) / 1.9e9;
           } else if (s_eff > 1) {
             // partials written and read back (mostly from L2) + the reduce kernel
             const double part_bytes = s_eff * 8.0 * T * static_cast<double>(N);
