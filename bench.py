@@ -283,9 +283,10 @@ class Dev:
                          aq.AQ_DTYPE_F16, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
                          self.ws_bytes, self.path, stream=st)
 
-    def layer_q8(self, st, s_out=0.02):
+    def layer_q8(self, st, s_out=0.02, path=None):
         """The layer with the next layer's quantizer in its epilogue (int8 output)."""
         aq, s = self.aq, self.spec
+        path = self.path if path is None else path
         if self.yq is None:
             self.yq = self.torch.empty(tuple(self.y.shape), dtype=self.torch.int8,
                                        device=self.y.device)
@@ -293,11 +294,11 @@ class Dev:
             aq.aq_conv2d_nhwc_q8(self.xq, self.s_x, self.packed, self.books, self.scale,
                                  self.bias, self.yq, s_out, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
                                  s.stride, 1, 8, self.M, self.B, self.ws, self.ws_bytes,
-                                 self.path, stream=st)
+                                 path, stream=st)
         else:
             aq.aq_linear_q8(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias,
                             self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
-                            self.ws_bytes, self.path, stream=st)
+                            self.ws_bytes, path, stream=st)
 
     def decode_only(self, st, wbuf):
         self.aq.aq_decode(self.packed, self.books, wbuf, self.N, self.K, 8, self.M, self.B,
@@ -338,7 +339,8 @@ def replay_ms(torch, stream, g, reps):
     return e0.elapsed_time(e1) / reps
 
 
-def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False):
+def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
+                 decode_ahead=False):
     """One UNet-shaped forward: every AQ layer of the LDM-4-like sweep, captured as one
     graph.  Each layer is preceded by its activation quantizer (aq_quant_act), or, with
     fused_quant, writes int8 output through its _q8 epilogue instead (the chain of
@@ -381,7 +383,40 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False)
                     layers.append(Dev(aq, torch, make_linear(spec, seed), dev))
     torch.cuda.synchronize()
 
+    # decode_ahead (with fused_quant): the dense-path layers take AQ_PATH_PREDECODED and a
+    # second stream decodes every such layer's weights (aq_decode into its workspace)
+    # ahead of the layer chain; each layer waits only for its own decode.  Every weight
+    # is still decoded once per forward; each dense layer then needs its decoded weights
+    # resident until it runs (here: one workspace per layer).
+    side = torch.cuda.Stream(device=dev) if decode_ahead else None
+    for L in layers:
+        L.dense = False
+        if decode_ahead:
+            s = L.spec
+            plan = (aq.aq_conv2d_plan(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3, s.stride, 1, 8, L.M,
+                                      L.B, L.path) if L.conv
+                    else aq.aq_linear_plan(L.T, L.K, L.N, 8, L.M, L.B, L.path))
+            L.dense = plan["path"] == aq.AQ_PATH_DENSE
+
     def fwd():
+        if decode_ahead:
+            start = torch.cuda.Event()
+            start.record(stream)
+            side.wait_event(start)
+            ready = []
+            for L in layers:
+                if L.dense:
+                    aq.aq_decode(L.packed, L.books, L.ws, L.N, L.K, 8, L.M, L.B, stream=side)
+                    e = torch.cuda.Event()
+                    e.record(side)
+                    ready.append(e)
+                else:
+                    ready.append(None)
+            for L, e in zip(layers, ready):
+                if e is not None:
+                    stream.wait_event(e)
+                L.layer_q8(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None)
+            return
         for L in layers:
             if fused_quant:
                 L.layer_q8(stream)
@@ -736,14 +771,19 @@ def main():
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
             for batch in [int(b) for b in args.unet_batches.split(",") if b]:
-                for fq in (False, True):
+                for fq, ahead in ((False, False), (True, False), (True, True)):
                     ms, gflop, nl = unet_forward(aq, torch, dev, stream, Mu, batch=batch,
-                                                 reps=20 if batch <= 2 else 5, fused_quant=fq)
-                    key = f"{label} batch {batch}" + (" quantizer in epilogue" if fq else "")
+                                                 reps=20 if batch <= 2 else 5, fused_quant=fq,
+                                                 decode_ahead=ahead)
+                    key = (f"{label} batch {batch}" + (" quantizer in epilogue" if fq else "")
+                           + (", decode ahead" if ahead else ""))
                     unet[key] = {"ms_per_forward": ms, "gflop": gflop, "tflops": gflop / ms,
                                  "layers": nl, "batch": batch,
                                  "step": ("each layer writes the next layer's int8 activations"
-                                          if fq else "each layer preceded by aq_quant_act")}
+                                          if fq else "each layer preceded by aq_quant_act")
+                                         + ("; dense-path layers decoded on a second stream "
+                                            "ahead of the chain (AQ_PATH_PREDECODED)"
+                                            if ahead else "")}
                     torch.cuda.empty_cache()
         assert aq.aq_device_error() == 0
 

@@ -79,9 +79,14 @@ typedef enum aq_path {
   AQ_PATH_LUT   = 3,  /* lookup-table order of App. A.1 (Eq. A5-A6): per token and group,
                          the dot product with every codeword, then a gather-sum by code;
                          for small token counts and B = 8                                  */
-  AQ_PATH_FEW_TOKENS = 4  /* linear layers with T <= 16: one kernel streams each row's codes
+  AQ_PATH_FEW_TOKENS = 4, /* linear layers with T <= 16: one kernel streams each row's codes
                          once, decodes in registers and dots with every token on CUDA
                          cores; no workspace                                              */
+  AQ_PATH_PREDECODED = 5  /* the dense path without its decode: the workspace's first
+                         N*K fp16 values already hold W-hat, written by aq_decode with the
+                         same codes and codebooks (e.g. on another stream, ahead of the
+                         layer, while the previous layer runs); same workspace size and
+                         plan as AQ_PATH_DENSE, same results                              */
 } aq_path;
 
 /* ---- library information -------------------------------------------------- */

@@ -16,6 +16,7 @@ _LIB_PATH = os.path.join(_PKG, "lib", "libaq_gb300.so")
 
 AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_DTYPE_I8 = 0, 1, 2
 AQ_PATH_AUTO, AQ_PATH_DENSE, AQ_PATH_FUSED, AQ_PATH_LUT, AQ_PATH_FEW_TOKENS = 0, 1, 2, 3, 4
+AQ_PATH_PREDECODED = 5
 
 _ERRORS = {
     -1: "AQ_ERR_NULL", -2: "AQ_ERR_SHAPE", -3: "AQ_ERR_UNSUPPORTED", -4: "AQ_ERR_ALIGN",

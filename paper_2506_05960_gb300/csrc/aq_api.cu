@@ -137,9 +137,9 @@ double stage_cycles(int BN) {
 // activations (TMA write, converter read), at about 80 B per cycle (measured on
 // GB300), and by the lookup latency (about 1000 cycles) when there is little work.
 // 16-bit codes gather their codewords from L2: about (12 + 12*M) * 2 issue cycles
-// per group over 8 warps.
+// per group over the 6 decoder warps (192 threads).
 double decode_stage_cycles(int BN, int M, int B) {
-  if (B == 16) return BN * 16.0 * (12.0 + 12.0 * M) * 2.0 / 256.0;
+  if (B == 16) return BN * 16.0 * (12.0 + 12.0 * M) * 2.0 / 192.0;
   const double bytes = BN * 16.0 * (16.0 * M + 32.0) + 32768.0;
   return std::max(1000.0, bytes / 80.0);
 }
@@ -281,6 +281,7 @@ int resolve_conv_path(int path, int m_tiles, int g) {
     case AQ_PATH_AUTO:
       return (m_tiles <= kFusedAutoMaxMTiles && !kaq) ? AQ_PATH_FUSED : AQ_PATH_DENSE;
     case AQ_PATH_DENSE:
+    case AQ_PATH_PREDECODED:
       return path;
     case AQ_PATH_FUSED:
       return kaq ? -2 : path;
@@ -330,6 +331,7 @@ int resolve_linear_path(int path, int T, int B) {
       return T <= kFewTokensMaxT ? path : -2;
     case AQ_PATH_DENSE:
     case AQ_PATH_FUSED:
+    case AQ_PATH_PREDECODED:
       return path;
     case AQ_PATH_LUT:
       return (B == 8 && T <= kLutMaxT) ? AQ_PATH_LUT : -2;
@@ -513,7 +515,8 @@ int sm_count() {
 // on the dense path in the same launch as the decode.
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
-             bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr) {
+             bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr,
+             bool predecoded = false) {
   const bool fused = Wdec == nullptr;
   p.fused = fused ? 1 : 0;
   p.codes = codes_packed;
@@ -576,12 +579,12 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   if (r) return r;
   cudaError_t e;
   const int64_t x_elems = static_cast<int64_t>(T) * K;
-  if (x16 && (fused || kaq)) {
+  if (x16 && (fused || kaq || predecoded)) {
     ProfScope ps(kProfQuant, st);
     e = aq::launch_quant_act(x16, xq, x_elems, p.s_x, st);
     if (e != cudaSuccess) return cuda_status(e, "quantizer launch");
   }
-  if (!fused) {
+  if (!fused && !predecoded) {
     ProfScope ps(kProfDecode, st);
     if (kaq)
       e = aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st);
@@ -610,6 +613,7 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
 // Plan and workspace layout of a tensor-core call on the dense or the fused path.
 struct Route {
   bool fused;
+  bool predecoded;  // the workspace already holds W-hat: the GEMM only
   Plan pl;
   size_t ws;
 };
@@ -617,6 +621,7 @@ struct Route {
 Route route_gemm(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, int B) {
   Route rt;
   rt.fused = rp == AQ_PATH_FUSED;
+  rt.predecoded = rp == AQ_PATH_PREDECODED;
   rt.pl = plan_gemm(T, N, K, m_tiles, true, f32_out, rt.fused, M, B);
   rt.ws = rt.fused ? fused_ws_bytes(T, N, rt.pl) : dense_ws_bytes(T, N, K, rt.pl);
   return rt;
@@ -1045,7 +1050,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   p.out_q8 = out_dtype == AQ_DTYPE_I8;
   p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st, false, x16,
-                  const_cast<int8_t*>(xq));
+                  const_cast<int8_t*>(xq), rt.predecoded);
 }
 
 }  // namespace
@@ -1174,7 +1179,7 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
   p.out_q8 = out_dtype == AQ_DTYPE_I8;
   p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st,
-                  g == kKaqGroup);
+                  g == kKaqGroup, nullptr, nullptr, rt.predecoded);
 }
 
 }  // namespace

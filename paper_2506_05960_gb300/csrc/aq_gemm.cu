@@ -873,16 +873,12 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
 
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st) {
-  static int configured_bytes = 0;
+  static std::atomic<int> configured[64] = {};
   const size_t bytes =
       gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes,
                       p.fused ? 8 * p.M * (p.B >> 3) : 0, p.epi_warps);
-  if (static_cast<int>(bytes) > configured_bytes) {
-    cudaError_t e = cudaFuncSetAttribute(aq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(bytes));
-    if (e != cudaSuccess) return e;
-    configured_bytes = static_cast<int>(bytes);
-  }
+  const cudaError_t se = ensure_dynamic_smem(aq_gemm_kernel, bytes, configured);
+  if (se != cudaSuccess) return se;
   // the decoder warps (10..15) exist only on the fused path
   if (p.epi_warps != 4 && !(p.epi_warps == 8 && !p.fused && p.BN >= 64))
     return cudaErrorInvalidConfiguration;

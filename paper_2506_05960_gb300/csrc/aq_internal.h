@@ -1,6 +1,7 @@
 // aq_internal.h -- host-side declarations shared by the library's translation units.
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <cuda.h>
@@ -103,6 +104,28 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) applies to the current device: the
+// size set so far is kept per device (0..63; others are set on every call) and raised
+// only when a launch needs more.
+template <typename Kernel>
+cudaError_t ensure_dynamic_smem(Kernel kernel, size_t bytes, std::atomic<int> (&configured)[64]) {
+  if (bytes <= 48 * 1024) return cudaSuccess;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const bool tracked = dev >= 0 && dev < 64;
+  if (tracked && configured[dev].load() >= static_cast<int>(bytes)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(bytes));
+  if (e == cudaSuccess && tracked) {
+    int cur = configured[dev].load();
+    while (cur < static_cast<int>(bytes) &&
+           !configured[dev].compare_exchange_weak(cur, static_cast<int>(bytes))) {
+    }
+  }
+  return e;
 }
 
 // Launchers (return the launch status; they never synchronise).

@@ -118,14 +118,10 @@ size_t lut_smem_bytes(int J, int M, int Tp, int T) {
 }
 
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
-  static size_t configured = 0;
+  static std::atomic<int> configured[64] = {};
   const size_t bytes = lut_smem_bytes(p.J, p.M, p.Tp, p.T);
-  if (bytes > 48 * 1024 && bytes > configured) {
-    cudaError_t e = cudaFuncSetAttribute(lut_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(bytes));
-    if (e != cudaSuccess) return e;
-    configured = bytes;
-  }
+  const cudaError_t se = ensure_dynamic_smem(lut_kernel, bytes, configured);
+  if (se != cudaSuccess) return se;
   const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
   dim3 grid(p.chunks, n_slices);
   return launch_pdl(lut_kernel, grid, dim3(256), bytes, st, p);
