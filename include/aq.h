@@ -237,8 +237,7 @@ AQ_API int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed,
 /* ---- layer from fp16 activations -------------------------------------------
  * aq_quant_act(x, xq, T*K, s_x) followed by aq_linear(xq, s_x, ...) in one call, the
  * int8 activations xq kept at the start of the workspace: the same bits as the two
- * calls.  On the dense path the quantizer and the weight decode (they share no data)
- * run in one kernel launch.
+ * calls.
  *   x fp16 [T][K]; s_x finite and > 0 (AQ_ERR_SHAPE); out_dtype F16 or F32.
  *   Workspace: aq_linear_f16_workspace_size() bytes = T*K rounded up to 1 KB plus
  *   aq_linear_workspace_size().                                                */

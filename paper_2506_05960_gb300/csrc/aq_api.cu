@@ -511,8 +511,7 @@ int sm_count() {
 // GEMM's decoder warps rebuild each weight tile in shared memory from the codes.
 // kaq: the codes use the kernel-aware grouping (g = 9, dense path only).
 // x16 != nullptr: the layer's fp16 activations, quantized here into the GEMM's int8
-// operand xq (the memory mapA points at) with the rule of aq_quant_act and scale p.s_x;
-// on the dense path in the same launch as the decode.
+// operand xq (the memory mapA points at) with the rule of aq_quant_act and scale p.s_x.
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
              bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr,
@@ -579,20 +578,15 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   if (r) return r;
   cudaError_t e;
   const int64_t x_elems = static_cast<int64_t>(T) * K;
-  if (x16 && (fused || kaq || predecoded)) {
+  if (x16) {
     ProfScope ps(kProfQuant, st);
     e = aq::launch_quant_act(x16, xq, x_elems, p.s_x, st);
     if (e != cudaSuccess) return cuda_status(e, "quantizer launch");
   }
   if (!fused && !predecoded) {
     ProfScope ps(kProfDecode, st);
-    if (kaq)
-      e = aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st);
-    else if (x16)
-      e = aq::launch_quant_decode(x16, xq, x_elems, p.s_x, codes_packed, codebooks, Wdec, N, K,
-                                  M, B, st);
-    else
-      e = aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
+    e = kaq ? aq::launch_decode_kaq(codes_packed, codebooks, Wdec, N, K / kKaqGroup, M, B, st)
+            : aq::launch_decode(codes_packed, codebooks, Wdec, N, K, M, B, st);
     if (e != cudaSuccess) return cuda_status(e, "decode launch");
   }
   {

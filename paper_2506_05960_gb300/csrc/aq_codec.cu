@@ -3,7 +3,6 @@
 //   * code packing into the 64-wide-K-block layout
 //   * AQ decode (Sec. 2.4 Eq. 4): W-hat = sum of the selected codewords, fp32
 //     sum in ascending codebook order, one round to fp16.
-#include <algorithm>
 #include <cstdint>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -217,56 +216,6 @@ __global__ void __launch_bounds__(512) decode_b16_kernel(const uint16_t* __restr
   grid_dependency_wait();
   allow_dependents();
   decode_b16_range(packed, books, W, N, K, M, KB, blockIdx.x, gridDim.x);
-}
-
-// The activation quantizer and the weight decode of one dense-path layer call in one
-// launch: they share no data, so blocks [0, qblocks) quantize and the rest decode, and
-// neither waits for the other.
-__global__ void __launch_bounds__(256) quant_decode_kernel(
-    const __half* __restrict__ x, int8_t* __restrict__ xq, int64_t nvec, int64_t numel, float s,
-    const void* __restrict__ packed, const uint4* __restrict__ books, __half* __restrict__ W,
-    int N, int K, int M, int B, int KB, int qblocks) {
-  extern __shared__ uint4 sbook[];                       // [M][256] for 8-bit codes
-  grid_dependency_wait();
-  allow_dependents();
-  if (static_cast<int>(blockIdx.x) < qblocks) {
-    quant_range(x, xq, nvec, numel, s, blockIdx.x, qblocks);
-    return;
-  }
-  const int bid = blockIdx.x - qblocks;
-  const int nb = gridDim.x - qblocks;
-  if (B == 8) {
-    stage_books8(books, sbook, M);
-    decode_b8_range(static_cast<const uint8_t*>(packed), sbook, W, N, K, M, KB, bid, nb);
-  } else {
-    decode_b16_range(static_cast<const uint16_t*>(packed), books, W, N, K, M, KB, bid, nb);
-  }
-}
-
-cudaError_t launch_quant_decode(const void* x, int8_t* xq, int64_t numel, float s,
-                                const void* packed, const void* books, void* W, int N, int K,
-                                int M, int B, cudaStream_t st) {
-  const int KB = (K + 63) / 64;
-  const int64_t nvec = numel / 16;
-  const int64_t groups = static_cast<int64_t>(KB) * N * 8;
-  // blocks in proportion to each side's bytes (48 per 16 activations, 18 per group),
-  // at most one resident wave of 256-thread blocks
-  int64_t qb = (nvec + 255) / 256;
-  int64_t db = (groups + 255) / 256;
-  const int64_t cap = 152 * 8;
-  if (qb + db > cap) {
-    const double qw = 48.0 * static_cast<double>(nvec);
-    const double dw = 18.0 * static_cast<double>(groups);
-    qb = std::min(qb, std::max<int64_t>(1, static_cast<int64_t>(cap * qw / (qw + dw))));
-    db = std::min(db, std::max<int64_t>(1, cap - qb));
-  }
-  if (qb < 1) qb = 1;
-  if (db < 1) db = 1;
-  const size_t smem = B == 8 ? static_cast<size_t>(M) * 256 * 16 : 0;
-  return launch_pdl(quant_decode_kernel, dim3(static_cast<unsigned>(qb + db)), dim3(256), smem, st,
-                    static_cast<const __half*>(x), xq, nvec, numel, s, packed,
-                    static_cast<const uint4*>(books), static_cast<__half*>(W), N, K, M, B, KB,
-                    static_cast<int>(qb));
 }
 
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,

@@ -134,10 +134,6 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
-// aq_quant_act of x into xq and the decode of W in one launch (independent block ranges).
-cudaError_t launch_quant_decode(const void* x, int8_t* xq, int64_t numel, float s,
-                                const void* packed, const void* books, void* W, int N, int K,
-                                int M, int B, cudaStream_t st);
 // dC[m][c][e] += sum over groups with code c of s_x*scale[n]*G[n][group element e]
 cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half* scale,
                                  float s_x, float* dC, int N, int K, int g, int M, int B,
