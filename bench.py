@@ -15,8 +15,12 @@ both sides, max over ranks.  The dominant kernel (the tensor-core GEMM) is
 timed live as the difference between the graph of the layer on int8 inputs
 (decode + GEMM) and the graph of the decode alone, replayed in the same timed
 region.
-`e2e` repeats the step through the C ABI with the input copied from pinned host
-memory and the output copied back every step.  `layers` times the other
+`e2e` repeats the step through the C ABI with every step's fp16 input copied from
+pinned host memory and its fp16 output copied back: copy-in, compute and
+copy-out on three streams, so one step's compute overlaps the neighbouring
+steps' copies (the serial single-stream figure is reported beside it).  A
+cuBLAS fp16 GEMM of the same shapes is timed as context for the GEMM's
+roofline fraction.  `layers` times the other
 workloads (64x64 W4A8 conv, 8x8 conv with one 2^16-entry codebook) and
 `unet_forward` one UNet-shaped forward (97 AQ layers, W2A8 and W4A8, batches 2, 16
 and 64), with each layer preceded by the quantizer, or writing the next layer's
@@ -649,36 +653,126 @@ def main():
     traffic = TRAFFIC["bytes"] if TRAFFIC.get("sources_sha") == sources_sha() else None
     launches_per_step = 3    # quantizer, decode, GEMM (the headline plan does not split K)
 
-    # e2e through the public API: pinned host input -> device, step, device -> pinned host
+    # e2e through the public API: every step copies its fp16 input from pinned host memory,
+    # runs aq_linear_f16 and copies its fp16 output back to pinned host memory.
+    #  - serial: copy in, step, copy out on one stream (each step waits for its copies);
+    #  - pipelined (the reported e2e): the serving pattern -- copy-in, compute and copy-out
+    #    streams with two buffer slots, so step i's compute overlaps the input copy of step
+    #    i+1 and the output copy of step i-1 on the two copy engines.  Every step still
+    #    moves all of its bytes between host and device inside the timed region.
     h_x = [b.x16.cpu().pin_memory() for b in bufs[:2]]
-    h_y = torch.empty((T, N), dtype=torch.float16).pin_memory()
+    h_y = [torch.empty((T, N), dtype=torch.float16).pin_memory() for _ in range(2)]
     e2e_steps = max(1, args.e2e_steps)
-    with torch.cuda.stream(stream):
-        for i in range(3):
+
+    def e2e_serial(n):
+        for i in range(n):
             b = bufs[i % 2]
             b.x16.copy_(h_x[i % 2], non_blocking=True)
             b.step_f16(stream)
-            h_y.copy_(b.y, non_blocking=True)
-        stream.synchronize()
+            h_y[i % 2].copy_(b.y, non_blocking=True)
+
+    s_in = torch.cuda.Stream(device=dev)
+    s_out = torch.cuda.Stream(device=dev)
+
+    def e2e_pipelined(n):
+        ev_in = [torch.cuda.Event() for _ in range(2)]     # input slot filled
+        ev_cmp = [torch.cuda.Event() for _ in range(2)]    # step done (input read, y written)
+        ev_out = [torch.cuda.Event() for _ in range(2)]    # output slot copied out
+        for i in range(n):
+            k = i % 2
+            b = bufs[k]
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(ev_cmp[k])              # the step that read x16[k] is done
+                b.x16.copy_(h_x[k], non_blocking=True)
+                ev_in[k].record(s_in)
+            stream.wait_event(ev_in[k])
+            if i >= 2:
+                stream.wait_event(ev_out[k])                # y[k] of step i-2 copied out
+            with torch.cuda.stream(stream):
+                b.step_f16(stream)
+                ev_cmp[k].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_cmp[k])
+                h_y[k].copy_(b.y, non_blocking=True)
+                ev_out[k].record(s_out)
+
+    def time_e2e(fn):
+        # the compute stream is torch's current stream here, so copies that name no stream
+        # (the serial variant) are ordered with the steps on it
+        with torch.cuda.stream(stream):
+            fn(4)
+        torch.cuda.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for i in range(e2e_steps):
-            b = bufs[i % 2]
-            b.x16.copy_(h_x[i % 2], non_blocking=True)
-            b.step_f16(stream)
-            h_y.copy_(b.y, non_blocking=True)
-        e1.record(stream)
-    stream.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    if pg:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            s_in.wait_stream(stream)
+            s_out.wait_stream(stream)
+            fn(e2e_steps)
+            stream.wait_stream(s_in)
+            stream.wait_stream(s_out)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / e2e_steps
+        if pg:
+            t = torch.tensor([ms], dtype=torch.float64, device=dev)
+            pg.all_reduce(t, op=pg.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms
+
+    def copies_only(n):
+        # the same host <-> device copies with no compute: the floor of the pipelined loop
+        for i in range(n):
+            k = i % 2
+            with torch.cuda.stream(s_in):
+                bufs[k].x16.copy_(h_x[k], non_blocking=True)
+            with torch.cuda.stream(s_out):
+                h_y[k].copy_(bufs[k].y, non_blocking=True)
+
+    e2e_serial_ms = time_e2e(e2e_serial)
+    e2e_ms = time_e2e(e2e_pipelined)
+    # every step's output reached the host: the last two slots hold the last two steps
+    y_last = bufs[(e2e_steps - 1) % 2].y.cpu()
+    assert torch.equal(h_y[(e2e_steps - 1) % 2], y_last)
+    copy_ms = time_e2e(copies_only)
 
     # the other workloads (per layer, graph replay) and the UNet-shaped forward
     layers, unet = {}, None
     if not args.no_extras and rank == 0:
+        # context, not the product path: a library fp16 GEMM (cuBLAS through torch.mm) of the
+        # same contraction shapes on fp16 operands already in HBM -- no int8 operand, no
+        # weight decode, no scale/bias epilogue -- 8 rotating buffer sets, CUDA graph replay
+        lib = {}
+        for name, (Tm, Km, Nm) in (("qkv T=4096 K=960 N=2880", (T, K, N)),
+                                   ("conv 16x64x64x192->192 as a GEMM T=65536 K=1728 N=192",
+                                    (65536, 1728, 192))):
+            gen = torch.Generator(device=dev).manual_seed(7)
+            As = [torch.randn((Tm, Km), dtype=torch.float16, device=dev, generator=gen)
+                  for _ in range(NSETS)]
+            Ws = [torch.randn((Nm, Km), dtype=torch.float16, device=dev, generator=gen)
+                  for _ in range(NSETS)]
+            Ys = [torch.empty((Tm, Nm), dtype=torch.float16, device=dev) for _ in range(NSETS)]
+
+            def mm():
+                for a, w, y in zip(As, Ws, Ys):
+                    torch.mm(a, w.t(), out=y)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    mm()
+            stream.synchronize()
+            gm = capture(torch, stream, mm)
+            ms = replay_ms(torch, stream, gm, 20) / NSETS
+            tf = linear_flops(Tm, Nm, Km) / (ms * 1e-3) / 1e12
+            lib[name] = {"us_per_gemm": ms * 1e3, "tflops": tf,
+                         "tensor_roofline_frac": tf / peaks["bf16_tflops"]}
+            del gm, As, Ws, Ys
+        lib["what"] = ("cuBLAS fp16 GEMM (torch.mm, fp32 accumulate) of the same shape on fp16 "
+                       "operands, no decode/int8 conversion/epilogue; context for the GEMM's "
+                       "roofline fraction at this shape")
+        lib["aq_gemm_over_cublas_qkv"] = achieved / lib["qkv T=4096 K=960 N=2880"]["tflops"]
+        layers["library GEMM of the same shapes (context)"] = lib
+        torch.cuda.empty_cache()
         from aq_synth import CONFIGS, make_conv
         for name, cfg in (("conv3x3 16x64x64x192->192 W4A8 (4x8)", 2),
                           ("conv3x3 2x8x8x960->960 one 2^16 codebook (1x16)", 3)):
@@ -815,7 +909,15 @@ def main():
             "cpu_baseline": cpu,
             "e2e": {"value": world * fl / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                     "ms_per_step": e2e_ms, "h2d_bytes_per_step": T * K * 2,
-                    "d2h_bytes_per_step": T * N * 2},
+                    "d2h_bytes_per_step": T * N * 2,
+                    "how": ("aq_linear_f16 from pinned host input to pinned host output, copy-in / "
+                            "compute / copy-out streams overlapped across consecutive steps"),
+                    "copy_floor_ms_per_step": copy_ms,
+                    "copy_floor_how": ("the step's input and output copies alone, on the "
+                                       "copy-in and copy-out streams (no compute)"),
+                    "serial": {"value": world * fl / (e2e_serial_ms * 1e-3) / 1e12,
+                               "ms_per_step": e2e_serial_ms,
+                               "how": "copy in, step, copy out on one stream"}},
             "gpu_launches": launches_per_step * steps + 3 * NSETS * reps_nogemm,
             "clocks": clocks,
         }
