@@ -29,7 +29,7 @@ import numpy as np
 
 __all__ = [
     "LinearSpec", "ConvSpec", "make_linear", "make_conv", "make_f16_activations",
-    "CONFIGS", "unet_sweep_layers",
+    "WORKLOADS", "SEEDS", "unet_sweep_layers",
 ]
 
 
@@ -140,19 +140,20 @@ def make_f16_activations(shape, seed: int, std: float = 1.0) -> np.ndarray:
     return rng.normal(0.0, std, size=shape).astype(np.float16)
 
 
-# Workloads.  Index = seed.
-CONFIGS = {
+# Workloads by name, each drawn from its own seed (SEEDS).
+WORKLOADS = {
     # tiny AQ linear, 2x8 codebooks (about 2 bits per weight)
-    0: LinearSpec(T=64, K=256, N=256, g=8, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02),
+    "tiny_linear": LinearSpec(T=64, K=256, N=256, g=8, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02),
     # fused qkv projection at the 8x8 level, 32 images x CFG pair: 64*64 tokens
-    1: LinearSpec(T=4096, K=960, N=2880, g=8, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02),
+    "qkv": LinearSpec(T=4096, K=960, N=2880, g=8, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02),
     # 3x3 conv, 16 x 64x64 x 192 -> 192, 4x8 codebooks
-    2: ConvSpec(Nb=16, H=64, W=64, Cin=192, Cout=192, stride=1, pad=1, g=8, M=4, B=8,
+    "conv64": ConvSpec(Nb=16, H=64, W=64, Cin=192, Cout=192, stride=1, pad=1, g=8, M=4, B=8,
                 cb_std=0.03, act="normal40", s_x=0.02),
     # 3x3 conv, 2 x 8x8 x 960 -> 960, one 2^16-entry codebook
-    3: ConvSpec(Nb=2, H=8, W=8, Cin=960, Cout=960, stride=1, pad=1, g=8, M=1, B=16,
-                cb_std=0.05, act="uniform", s_x=0.02),
+    "conv8_book16": ConvSpec(Nb=2, H=8, W=8, Cin=960, Cout=960, stride=1, pad=1, g=8, M=1,
+                             B=16, cb_std=0.05, act="uniform", s_x=0.02),
 }
+SEEDS = {"tiny_linear": 0, "qkv": 1, "conv64": 2, "conv8_book16": 3}
 
 
 def unet_sweep_layers():

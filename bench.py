@@ -143,8 +143,8 @@ class ClockSampler:
 
 # ----------------------------------------------------------------------------- workload
 def headline_sets(nsets: int):
-    from aq_synth import CONFIGS, make_linear
-    spec = CONFIGS[1]
+    from aq_synth import WORKLOADS, make_linear
+    spec = WORKLOADS["qkv"]
     return spec, [make_linear(spec, seed=1000 + i) for i in range(nsets)]
 
 
@@ -455,7 +455,7 @@ KERNEL_WORKLOADS = {
 def run_kernel_workload(args, aq, torch, dev, stream):
     """One kernel's call on the seeded qkv-shaped layer, --warmup + --steps plain launches
     (no graph), for ncu captures; returns the mean time per call (CUDA events)."""
-    from aq_synth import CONFIGS, LinearSpec, make_linear
+    from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_linear
     w = args.workload
     if w in ("fused128", "few4", "lut8"):
         T = {"fused128": 128, "few4": 4, "lut8": 8}[w]
@@ -463,7 +463,7 @@ def run_kernel_workload(args, aq, torch, dev, stream):
         L = Dev(aq, torch, make_linear(spec, seed=7), dev, path=3 if w == "lut8" else 0)
         call = lambda: L.layer(stream)
     else:
-        L = Dev(aq, torch, make_linear(CONFIGS[1], seed=1), dev)
+        L = Dev(aq, torch, make_linear(WORKLOADS["qkv"], seed=SEEDS["qkv"]), dev)
         N, K = L.N, L.K
         if w == "quant":
             call = lambda: L.quant(stream)
@@ -502,7 +502,7 @@ def run_single(args):
     """One non-headline workload on one GPU (profiling aid): prints its timing."""
     import torch
     import paper_2506_05960_gb300 as aq
-    from aq_synth import CONFIGS, make_conv
+    from aq_synth import SEEDS, WORKLOADS, make_conv
     dev = torch.device("cuda", 0)
     aq.load_library()
     stream = torch.cuda.Stream(device=dev)
@@ -515,8 +515,8 @@ def run_single(args):
         out = {"workload": "UNet-shaped forward W2A8 batch 2", "ms_per_forward": ms,
                "gflop": gflop, "layers": nl}
     else:
-        cfg = 2 if args.workload == "conv64" else 3
-        L = Dev(aq, torch, make_conv(CONFIGS[cfg], seed=cfg), dev)
+        name = "conv64" if args.workload == "conv64" else "conv8_book16"
+        L = Dev(aq, torch, make_conv(WORKLOADS[name], seed=SEEDS[name]), dev)
         with torch.cuda.stream(stream):
             for _ in range(args.warmup):
                 L.step(stream)
@@ -773,10 +773,10 @@ def main():
         lib["aq_gemm_over_cublas_qkv"] = achieved / lib["qkv T=4096 K=960 N=2880"]["tflops"]
         layers["library GEMM of the same shapes (context)"] = lib
         torch.cuda.empty_cache()
-        from aq_synth import CONFIGS, make_conv
-        for name, cfg in (("conv3x3 16x64x64x192->192 W4A8 (4x8)", 2),
-                          ("conv3x3 2x8x8x960->960 one 2^16 codebook (1x16)", 3)):
-            L = Dev(aq, torch, make_conv(CONFIGS[cfg], seed=cfg), dev)
+        from aq_synth import SEEDS, WORKLOADS, make_conv
+        for name, wl in (("conv3x3 16x64x64x192->192 W4A8 (4x8)", "conv64"),
+                         ("conv3x3 2x8x8x960->960 one 2^16 codebook (1x16)", "conv8_book16")):
+            L = Dev(aq, torch, make_conv(WORKLOADS[wl], seed=SEEDS[wl]), dev)
             with torch.cuda.stream(stream):
                 for _ in range(3):
                     L.step(stream)
@@ -814,7 +814,7 @@ def main():
         del gc, gsets
         # Stage-1 code search (one greedy step over both codebooks) on the qkv layer
         from aq_synth import make_linear as _ml
-        inp1 = _ml(CONFIGS[1], seed=1)
+        inp1 = _ml(WORKLOADS["qkv"], seed=SEEDS["qkv"])
         Wt = torch.from_numpy(np.ascontiguousarray(
             (inp1["codebooks"].astype(np.float32)[0][inp1["codes"][:, :, 0]]
              + inp1["codebooks"].astype(np.float32)[1][inp1["codes"][:, :, 1]]).reshape(N, K)

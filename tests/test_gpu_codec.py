@@ -4,7 +4,7 @@ activation quantizer, code packing, and the AQ decode rule."""
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, make_f16_activations, make_conv, make_linear
+from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_f16_activations, make_conv, make_linear
 from oracle import aq_oracle as O
 
 from gpu_util import dev, pack
@@ -75,10 +75,11 @@ def _decode_gpu(codes, books, N, K, M, B):
     return W.cpu().numpy()
 
 
-@pytest.mark.parametrize("cfg", [0, 1, 2, 3])
-def test_decode_bit_exact_configs(cfg):
-    spec = CONFIGS[cfg]
-    inp = make_linear(spec, seed=cfg) if cfg < 2 else make_conv(spec, seed=cfg)
+@pytest.mark.parametrize("wl", ["tiny_linear", "qkv", "conv64", "conv8_book16"])
+def test_decode_bit_exact_workloads(wl):
+    spec = WORKLOADS[wl]
+    make = make_linear if isinstance(spec, LinearSpec) else make_conv
+    inp = make(spec, seed=SEEDS[wl])
     N, G, M = inp["codes"].shape
     B = spec.B
     W = _decode_gpu(inp["codes"], inp["codebooks"], N, G * 8, M, B)

@@ -3,7 +3,7 @@ oracle's direct convolution."""
 
 import pytest
 
-from aq_synth import CONFIGS, ConvSpec, make_conv
+from aq_synth import SEEDS, WORKLOADS, ConvSpec, make_conv
 from oracle import aq_oracle as O
 
 from gpu_util import assert_close, run_conv
@@ -57,13 +57,13 @@ def test_conv_fp32_no_bias():
 
 def test_conv_64x64_w4a8_full():
     """16 x 64x64 x 192 -> 192, 4x8 codebooks: every output pixel and channel."""
-    inp = make_conv(CONFIGS[2], seed=2)
+    inp = make_conv(WORKLOADS["conv64"], seed=SEEDS["conv64"])
     y = run_conv(inp)
     assert_close(y, O.layer_f64(inp), "conv 64x64")
 
 
 def test_conv_8x8_large_codebook_full():
     """2 x 8x8 x 960 -> 960, one 2^16-entry codebook (split-K plan)."""
-    inp = make_conv(CONFIGS[3], seed=3)
+    inp = make_conv(WORKLOADS["conv8_book16"], seed=SEEDS["conv8_book16"])
     y = run_conv(inp)
     assert_close(y, O.layer_f64(inp), "conv 8x8 1x16")

@@ -5,7 +5,7 @@ oracle, for linear and convolution layers and both code widths."""
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, ConvSpec, LinearSpec, make_conv, make_linear
+from aq_synth import SEEDS, WORKLOADS, ConvSpec, LinearSpec, make_conv, make_linear
 from oracle import aq_oracle as O
 
 from gpu_util import assert_close, run_conv, run_linear
@@ -49,7 +49,7 @@ def test_fused_linear_fp32_matches_dense():
 
 def test_fused_conv_large_codebook_full():
     """2 x 8x8 x 960 -> 960, one 2^16-entry codebook: the fused path with split K."""
-    inp = make_conv(CONFIGS[3], seed=3)
+    inp = make_conv(WORKLOADS["conv8_book16"], seed=SEEDS["conv8_book16"])
     y = run_conv(inp, path=FUSED)
     assert_close(y, O.layer_f64(inp), "conv 8x8 1x16 fused")
 

@@ -5,7 +5,7 @@ codebook formats, output dtypes and the split-K plan."""
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, LinearSpec, make_linear
+from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_linear
 from oracle import aq_oracle as O
 
 from gpu_util import assert_close, run_linear
@@ -21,8 +21,8 @@ def _lib():
 
 @pytest.mark.parametrize("out_f32", [False, True])
 @pytest.mark.parametrize("with_bias", [True, False])
-def test_tiny_config(out_f32, with_bias):
-    inp = make_linear(CONFIGS[0], seed=0)
+def test_tiny_linear_workload(out_f32, with_bias):
+    inp = make_linear(WORKLOADS["tiny_linear"], seed=SEEDS["tiny_linear"])
     y = run_linear(inp, out_f32=out_f32, with_bias=with_bias)
     W = O.decode_f64(inp["codes"], inp["codebooks"])
     y64 = O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], inp["bias"] if with_bias else None)
@@ -31,7 +31,7 @@ def test_tiny_config(out_f32, with_bias):
 
 def test_qkv_projection_full():
     """T=4096, K=960, N=2880, 2x8 codebooks: every output against the oracle."""
-    inp = make_linear(CONFIGS[1], seed=1)
+    inp = make_linear(WORKLOADS["qkv"], seed=SEEDS["qkv"])
     y = run_linear(inp)
     assert_close(y, O.layer_f64(inp), "qkv")
 

@@ -7,7 +7,7 @@ oracle's output passed through the quantizer rule."""
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, ConvSpec, LinearSpec, make_conv, make_linear
+from aq_synth import SEEDS, WORKLOADS, ConvSpec, LinearSpec, make_conv, make_linear
 from oracle import aq_oracle as O
 
 from gpu_util import dev, pack
@@ -84,11 +84,11 @@ def test_linear_q8_scales_with_exact_ties(s_out, path):
     assert np.array_equal(q, q_chain)
 
 
-@pytest.mark.parametrize("cfg,path", [(2, AUTO), (3, AUTO)])
-def test_conv_q8_equals_chain(cfg, path):
+@pytest.mark.parametrize("wl,path", [("conv64", AUTO), ("conv8_book16", AUTO)])
+def test_conv_q8_equals_chain(wl, path):
     import torch
     import paper_2506_05960_gb300 as aq
-    inp = make_conv(CONFIGS[cfg], seed=cfg)
+    inp = make_conv(WORKLOADS[wl], seed=SEEDS[wl])
     s = inp["spec"]
     N, G, M = inp["codes"].shape
     B = 8 if inp["codes"].dtype == np.uint8 else 16

@@ -15,7 +15,7 @@ from fractions import Fraction
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, ConvSpec, LinearSpec, make_conv, make_linear
+from aq_synth import SEEDS, WORKLOADS, ConvSpec, LinearSpec, make_conv, make_linear
 from oracle import aq_oracle as O
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
@@ -254,9 +254,9 @@ def test_one_hot_codebooks_reproduce_dense_int_layer():
 
 
 def test_bits_per_weight_closed_form():
-    for cfg in (0, 1):
-        spec = CONFIGS[cfg]
-        inp = make_linear(spec, seed=cfg) if cfg == 0 else None
+    for wl in ("tiny_linear", "qkv"):
+        spec = WORKLOADS[wl]
+        inp = make_linear(spec, seed=SEEDS[wl]) if wl == "tiny_linear" else None
         if inp is None:
             continue
         got = O.bits_per_weight(inp["codes"], inp["codebooks"], inp["scale"], spec.N, spec.K)

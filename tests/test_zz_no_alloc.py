@@ -12,7 +12,7 @@ import ctypes
 import numpy as np
 import pytest
 
-from aq_synth import CONFIGS, LinearSpec, make_linear
+from aq_synth import WORKLOADS, LinearSpec, make_linear
 from oracle import aq_oracle as O
 
 
@@ -58,7 +58,7 @@ def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
 
     # two different layers, one call each, back to back: the second call must not see
     # anything left in the shared scratch by the first
-    inps = [make_linear(CONFIGS[1], seed=101),
+    inps = [make_linear(WORKLOADS["qkv"], seed=101),
             make_linear(LinearSpec(T=300, K=1024, N=1152, M=4, B=8, cb_std=0.025), seed=102)]
     layers = [layer_inputs(i) for i in inps]
     got = [no_alloc(L) for L in layers]
