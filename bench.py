@@ -178,6 +178,21 @@ def time_oracle(inp, flops, min_seconds: float = 10.0, max_steps: int = 50) -> d
                       f"{el:.1f} s, numpy float64 BLAS on {cores} host cores"}
 
 
+def max_over_ranks(dist, value: float, device) -> float:
+    """The largest `value` over all ranks of the process group (every rank receives it):
+    the job takes as long as its slowest replica."""
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, flops_per_step: float, ms_per_step: float) -> float:
+    """Whole-job dense-equivalent TFLOP/s: every rank runs its own replica of the step
+    (weak scaling), so the job does `world` steps in the slowest rank's step time."""
+    return world * flops_per_step / (ms_per_step * 1e-3) / 1e12
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -641,11 +656,9 @@ def main():
     ms_decode_step = ev[2].elapsed_time(ev[3]) / (reps_nogemm * NSETS)
     assert aq.aq_device_error() == 0
     if pg:
-        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms_total = float(t.item())
+        ms_total = max_over_ranks(pg, ms_total, dev)
     ms_step = ms_total / steps
-    value = world * fl / (ms_step * 1e-3) / 1e12
+    value = job_throughput(world, fl, ms_step)
     gemm_ms = ms_layer_step - ms_decode_step
 
     peaks = measured_peaks()
@@ -716,9 +729,7 @@ def main():
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / e2e_steps
         if pg:
-            t = torch.tensor([ms], dtype=torch.float64, device=dev)
-            pg.all_reduce(t, op=pg.ReduceOp.MAX)
-            ms = float(t.item())
+            ms = max_over_ranks(pg, ms, dev)
         return ms
 
     def copies_only(n):
@@ -907,7 +918,7 @@ def main():
                                        alg_bytes(T, K, N, M, B) / (peaks["hbm_gbs"] * 1e9))
                                    / (ms_step * 1e-3)),
             "cpu_baseline": cpu,
-            "e2e": {"value": world * fl / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "e2e": {"value": job_throughput(world, fl, e2e_ms), "unit": "TFLOP/s",
                     "ms_per_step": e2e_ms, "h2d_bytes_per_step": T * K * 2,
                     "d2h_bytes_per_step": T * N * 2,
                     "how": ("aq_linear_f16 from pinned host input to pinned host output, copy-in / "
@@ -915,7 +926,7 @@ def main():
                     "copy_floor_ms_per_step": copy_ms,
                     "copy_floor_how": ("the step's input and output copies alone, on the "
                                        "copy-in and copy-out streams (no compute)"),
-                    "serial": {"value": world * fl / (e2e_serial_ms * 1e-3) / 1e12,
+                    "serial": {"value": job_throughput(world, fl, e2e_serial_ms),
                                "ms_per_step": e2e_serial_ms,
                                "how": "copy in, step, copy out on one stream"}},
             "gpu_launches": launches_per_step * steps + 3 * NSETS * reps_nogemm,

@@ -1,0 +1,58 @@
+"""Host logic of the multi-GPU bench path on CPU: the layer has no exchange step, so
+N GPUs run N independent replicas; the job's step time is the slowest rank's, and
+throughput counts every rank's work.  Two gloo ranks stand in for two GPUs."""
+
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, per_rank_ms, out_dir):
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        ms = bench.max_over_ranks(dist, per_rank_ms[rank], "cpu")
+        value = bench.job_throughput(world, 2.0e9, ms)
+        with open(os.path.join(out_dir, f"rank{rank}.txt"), "w") as f:
+            f.write(f"{ms!r} {value!r}\n")
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_and_job_throughput_two_gloo_ranks(tmp_path):
+    import torch.multiprocessing as mp
+    per_rank_ms = [0.25, 0.40]
+    mp.start_processes(_rank_main, args=(2, _free_port(), per_rank_ms, str(tmp_path)),
+                       nprocs=2, join=True, start_method="spawn")
+    got = [open(tmp_path / f"rank{r}.txt").read().split() for r in range(2)]
+    for ms, value in got:
+        # every rank sees the slowest rank's time; the job did 2 steps in that time
+        assert float(ms) == 0.40
+        assert float(value) == pytest.approx(2 * 2.0e9 / 0.40e-3 / 1e12)
+    assert bench.job_throughput(1, 2.0e9, 0.40) * 2 == pytest.approx(float(got[0][1]))
+
+
+def test_reference_arm_other_ranks_exit_without_output():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--gpus", "2", "--steps", "1", "--warmup", "3"],
+                       env=env, capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.strip() == ""
