@@ -303,22 +303,24 @@ class Dev:
                          aq.AQ_DTYPE_F16, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
                          self.ws_bytes, self.path, stream=st)
 
-    def layer_q8(self, st, s_out=0.02, path=None):
-        """The layer with the next layer's quantizer in its epilogue (int8 output)."""
+    def layer_q8(self, st, s_out=0.02, path=None, ws=None):
+        """The layer with the next layer's quantizer in its epilogue (int8 output); `ws`
+        replaces the layer's workspace (e.g. one holding weights decoded beforehand)."""
         aq, s = self.aq, self.spec
         path = self.path if path is None else path
+        ws_t = self.ws if ws is None else ws
         if self.yq is None:
             self.yq = self.torch.empty(tuple(self.y.shape), dtype=self.torch.int8,
                                        device=self.y.device)
         if self.conv:
             aq.aq_conv2d_nhwc_q8(self.xq, self.s_x, self.packed, self.books, self.scale,
                                  self.bias, self.yq, s_out, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
-                                 s.stride, 1, 8, self.M, self.B, self.ws, self.ws_bytes,
+                                 s.stride, 1, 8, self.M, self.B, ws_t, ws_t.numel(),
                                  path, stream=st)
         else:
             aq.aq_linear_q8(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias,
-                            self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, self.ws,
-                            self.ws_bytes, path, stream=st)
+                            self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, ws_t,
+                            ws_t.numel(), path, stream=st)
 
     def decode_only(self, st, wbuf):
         self.aq.aq_decode(self.packed, self.books, wbuf, self.N, self.K, 8, self.M, self.B,
@@ -402,20 +404,33 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
                     layers.append(Dev(aq, torch, make_linear(spec, seed), dev))
     torch.cuda.synchronize()
 
-    # decode_ahead (with fused_quant): the dense-path layers take AQ_PATH_PREDECODED and a
-    # second stream decodes every such layer's weights (aq_decode into its workspace)
-    # ahead of the layer chain; each layer waits only for its own decode.  Every weight
-    # is still decoded once per forward; each dense layer then needs its decoded weights
-    # resident until it runs (here: one workspace per layer).
+    # decode_ahead (with fused_quant): the dense-path layers -- and, with 4 or more
+    # codebooks, also the token-poor ones that AUTO sends down the fused path -- take
+    # AQ_PATH_PREDECODED, and a second stream decodes those layers' weights (aq_decode into
+    # a workspace) ahead of the layer chain; each layer waits only for its own decode.
+    # (Measured at batch 2: predecoding the fused-path layers too took the W4A8 forward from
+    # 1.457 to 1.408 ms but the W2A8 one from 1.288 to 1.359 ms -- with two codebooks the
+    # in-GEMM decode costs less than streaming the 8x larger decoded weights.)
+    # Every weight is still decoded once per forward; each such layer then needs its decoded
+    # weights resident until it runs (here: one workspace per layer).
     side = torch.cuda.Stream(device=dev) if decode_ahead else None
     for L in layers:
         L.dense = False
+        L.ws_pre = L.ws
         if decode_ahead:
             s = L.spec
             plan = (aq.aq_conv2d_plan(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3, s.stride, 1, 8, L.M,
                                       L.B, L.path) if L.conv
                     else aq.aq_linear_plan(L.T, L.K, L.N, 8, L.M, L.B, L.path))
             L.dense = plan["path"] == aq.AQ_PATH_DENSE
+            if L.M >= 4 and not L.dense:
+                L.dense = True
+                nb = (aq.aq_conv2d_workspace_size(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3, s.stride,
+                                                  1, 8, L.M, L.B, aq.AQ_PATH_PREDECODED)
+                      if L.conv else
+                      aq.aq_linear_workspace_size(L.T, L.K, L.N, 8, L.M, L.B,
+                                                  aq.AQ_PATH_PREDECODED))
+                L.ws_pre = torch.empty(nb, dtype=torch.uint8, device=dev)
 
     def fwd():
         if decode_ahead:
@@ -425,7 +440,7 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
             ready = []
             for L in layers:
                 if L.dense:
-                    aq.aq_decode(L.packed, L.books, L.ws, L.N, L.K, 8, L.M, L.B, stream=side)
+                    aq.aq_decode(L.packed, L.books, L.ws_pre, L.N, L.K, 8, L.M, L.B, stream=side)
                     e = torch.cuda.Event()
                     e.record(side)
                     ready.append(e)
@@ -434,7 +449,8 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
             for L, e in zip(layers, ready):
                 if e is not None:
                     stream.wait_event(e)
-                L.layer_q8(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None)
+                L.layer_q8(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None,
+                           ws=L.ws_pre)
             return
         for L in layers:
             if fused_quant:
