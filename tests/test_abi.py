@@ -168,3 +168,24 @@ def test_plan_query_and_override(lib):
         assert p["cluster"] == 1 and aq.aq_conv2d_workspace_size(2, 8, 8, 960, 960, M=2) == 0
     finally:
         aq.aq_set_plan_override()
+
+
+def test_missing_library_fails_loudly():
+    """Without the compiled library every entry point raises: there is no Python or CPU
+    fallback for any step of the path."""
+    import subprocess
+    import sys
+    code = (
+        "import paper_2506_05960_gb300._binding as b\n"
+        "b._LIB_PATH = '/nonexistent/libaq_gb300.so'\n"
+        "import paper_2506_05960_gb300 as aq\n"
+        "try:\n"
+        "    aq.aq_packed_size(256, 256, 8, 2, 8)\n"
+        "except ImportError as e:\n"
+        "    print('raised:', e)\n"
+        "else:\n"
+        "    print('no error')\n")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True,
+                       timeout=120)
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.startswith("raised:") and "no CPU fallback" in r.stdout, r.stdout
