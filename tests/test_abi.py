@@ -109,6 +109,13 @@ def test_null_and_alignment_errors_do_not_launch(lib):
     # T == 0 is a no-op even with NULL buffers
     assert lib.aq_linear(None, 0.02, None, None, None, None, None, 0, 0, 64, 64, 8, 2, 8, None,
                          0, 0, None) == 0
+    # ... and so are an empty batch of images and the fp16-input / int8-output variants
+    assert lib.aq_conv2d_nhwc(None, 0.02, None, None, None, None, None, 0, 0, 8, 8, 64, 64, 3, 3,
+                              1, 1, 8, 2, 8, None, 0, 0, None) == 0
+    assert lib.aq_linear_f16(None, 0.02, None, None, None, None, None, 0, 0, 64, 64, 8, 2, 8,
+                             None, 0, 0, None) == 0
+    assert lib.aq_linear_q8(None, 0.02, None, None, None, None, None, 0.02, 0, 64, 64, 8, 2, 8,
+                            None, 0, 0, None) == 0
     # quantizer: numel 0 no-op; bad scale
     assert lib.aq_quant_act(None, None, 0, 0.5, None) == 0
     assert lib.aq_quant_act(16, 16, 16, 0.0, None) == -2
