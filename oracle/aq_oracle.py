@@ -214,7 +214,10 @@ def quant_act(x: np.ndarray, s_x: float) -> np.ndarray:
     x / s_x taken in IEEE fp32 (x is fp16, so widening is exact), round half to
     even, clip to [-127, 127] (-128 unused), NaN maps to 0.
     """
-    q = np.asarray(x).astype(np.float32) / np.float32(s_x)
+    # widening a signalling-NaN fp16 pattern raises the IEEE invalid flag; the value is
+    # a NaN either way and maps to 0 below
+    with np.errstate(invalid="ignore"):
+        q = np.asarray(x).astype(np.float32) / np.float32(s_x)
     q = np.rint(q)
     q = np.where(np.isnan(q), np.float32(0.0), q)
     q = np.clip(q, -127.0, 127.0)
