@@ -57,7 +57,7 @@ NSETS = 8
 # reported only while the kernel sources are the ones it was measured on.
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 9553152, "sources_sha": "72471d44371e52c3"}
+TRAFFIC = {"bytes": 9553152, "sources_sha": "10abd9cc89e33978"}
 
 
 def sources_sha() -> str:
@@ -888,6 +888,23 @@ def main():
                                   "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
                                   "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
                     del gs, Ls
+        # the few-token path on a layer large enough to amortise its launch: how fast it
+        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes)
+        for Ts in (1, 4):
+            inp_s = _mlin(LinearSpec(T=Ts, K=8192, N=16384, M=2, B=8), seed=90 + Ts)
+            Ls = [Dev(aq, torch, inp_s, dev, path=aq.AQ_PATH_FEW_TOKENS) for _ in range(4)]
+            with torch.cuda.stream(stream):
+                for L in Ls:
+                    L.step(stream)
+            stream.synchronize()
+            gs = capture(torch, stream, lambda: [L.layer(stream) for L in Ls])
+            ms = replay_ms(torch, stream, gs, 10) / len(Ls)
+            wbytes = alg_bytes(Ts, 8192, 16384, 2, 8)
+            sweep[f"K=8192 N=16384 2x8 T={Ts} FEW (layer only, 4 rotating buffer sets)"] = {
+                "us_per_step": ms * 1e3, "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
+                "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
+            del gs, Ls
+            torch.cuda.empty_cache()
         layers["small-T sweep (quantizer + layer per step, 8 rotating buffer sets)"] = sweep
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):

@@ -972,6 +972,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     sp.N = N;
     sp.M = M;
     sp.B = B;
+    sp.sms = sm_count();
     ProfScope ps(kProfLutGather, static_cast<cudaStream_t>(stream));
     return cuda_status(aq::launch_skinny(sp, static_cast<cudaStream_t>(stream)),
                        "few-token launch");

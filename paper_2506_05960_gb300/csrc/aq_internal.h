@@ -85,7 +85,7 @@ struct SkinnyParams {
   int out_f32, out_q8;
   float s_x, s_out;
   int T, K, N, M, B;
-  int quads;                    // row quads per CTA (set by the launcher)
+  int sms;                      // SMs of the device (the caller's count; sizes the grid)
 };
 
 // Launch with programmatic stream serialization (the kernel must call
