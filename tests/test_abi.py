@@ -196,3 +196,53 @@ def test_missing_library_fails_loudly():
                        timeout=120)
     assert r.returncode == 0, r.stderr
     assert r.stdout.startswith("raised:") and "no CPU fallback" in r.stdout, r.stdout
+
+
+def test_plans_of_every_unet_layer_are_well_formed(lib):
+    """Every layer shape of the UNet sweep, at batch 2, 16 and 64, both weight formats and
+    every tensor-core path: the planner returns a runnable plan (host only, no device)."""
+    import paper_2506_05960_gb300 as aq
+    from aq_synth import unet_sweep_layers
+    aq.aq_set_plan_override()
+    n_checked = 0
+    for batch in (2, 16, 64):
+        for M in (2, 4):
+            for kind, res, cin, cout, stride, _ in unet_sweep_layers():
+                for path in (aq.AQ_PATH_AUTO, aq.AQ_PATH_DENSE, aq.AQ_PATH_FUSED,
+                             aq.AQ_PATH_PREDECODED):
+                    if kind == "conv3":
+                        H = res * stride
+                        T = batch * res * res
+                        K = 9 * cin
+                        p = aq.aq_conv2d_plan(batch, H, H, cin, cout, 3, 3, stride, 1, 8, M, 8,
+                                              path)
+                        ws = aq.aq_conv2d_workspace_size(batch, H, H, cin, cout, 3, 3, stride,
+                                                         1, 8, M, 8, path)
+                    else:
+                        T, K = batch * res * res, cin
+                        p = aq.aq_linear_plan(T, K, cout, 8, M, 8, path)
+                        ws = aq.aq_linear_workspace_size(T, K, cout, 8, M, 8, path)
+                    if p["path"] == aq.AQ_PATH_FEW_TOKENS:
+                        assert ws == 0
+                        continue
+                    assert p["path"] in (aq.AQ_PATH_DENSE, aq.AQ_PATH_FUSED,
+                                         aq.AQ_PATH_PREDECODED)
+                    if path != aq.AQ_PATH_AUTO:
+                        assert p["path"] == path
+                    BN, S = p["BN"], p["splits"]
+                    assert BN % 32 == 0 and 32 <= BN <= 192, p
+                    assert p["stages"] >= 2, p
+                    m_tiles = (T + 127) // 128
+                    n_tiles = (cout + BN - 1) // BN
+                    assert p["work_items"] == m_tiles * n_tiles * S, (p, T, cout)
+                    k_blocks = (K + 63) // 64
+                    assert 1 <= S <= k_blocks, p
+                    if p["cluster"]:
+                        assert 2 <= S <= 8, p
+                    if p["path"] != aq.AQ_PATH_FUSED:
+                        # the decoded weights (fp16, N x K) sit at the start of the workspace
+                        assert ws >= cout * K * 2, (p, ws)
+                    if S > 1 and not p["cluster"]:
+                        assert ws >= S * T * cout * 4, (p, ws)   # fp32 split-K partials
+                    n_checked += 1
+    assert n_checked > 1000
