@@ -246,3 +246,16 @@ def test_plans_of_every_unet_layer_are_well_formed(lib):
                         assert ws >= S * T * cout * 4, (p, ws)   # fp32 split-K partials
                     n_checked += 1
     assert n_checked > 1000
+
+
+def test_noalloc_argument_checks_before_any_cuda_call(lib):
+    """aq_linear_noalloc refuses layers whose decoded weights exceed its fixed scratch
+    (16 MiB) and bad arguments on the host, so these calls need no GPU."""
+    args = lambda T, K, N, out=0, s=0.02: (None, s, None, None, None, None, None, out, T, K, N,
+                                           8, 2, 8, None)
+    assert lib.aq_linear_noalloc(*args(4, 4096, 2056)) == -5        # 4096*2056*2 > 16 MiB
+    assert lib.aq_linear_noalloc(*args(4, 4096, 2048)) == -1        # fits: then NULL buffers
+    assert lib.aq_linear_noalloc(*args(0, 4096, 2048)) == 0         # empty: no-op
+    assert lib.aq_linear_noalloc(*args(4, 4096, 2048, out=2)) == -3  # int8 output not offered
+    assert lib.aq_linear_noalloc(*args(4, 4096, 2048, s=float("nan"))) == -2
+    assert lib.aq_linear_noalloc(*args(4, 4100, 2048)) == -2        # K % 16
