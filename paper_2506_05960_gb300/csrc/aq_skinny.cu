@@ -20,8 +20,7 @@
 // 8-bit codebooks are staged in shared memory in R copies (copy r of entry e in 16-byte
 // slot e * R + r, lane l reading copy l % R): the 8 lanes of a quarter warp, whose random
 // 16-byte lookups are served together, then always hit 8 different bank groups.  16-bit
-// (2^16-entry) codebooks are read from L2; for them, from two tokens on, a second layout
-// (skinny_gather_kernel, below) is used.
+// (2^16-entry) codebooks are read from L2 by a second layout (skinny_gather_kernel, below).
 #include <cstdint>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -222,11 +221,12 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
   }
 }
 
-// 16-bit codes (2^16-entry codebooks, codewords gathered from L2) with T >= 2: the layout
-// of four output rows per CTA, whose threads stride the K/8 group columns and decode each
-// group for the four rows, keeps more independent gathers in flight per thread (measured
-// on GB300: 13.9 / 16.5 us at T = 2 / 4 on a K = 8640, N = 960 layer, against 19.5 / 26.7
-// for the row-block layout above, which is faster at T = 1).
+// 16-bit codes (2^16-entry codebooks, codewords gathered from L2): the layout of four
+// output rows per CTA, whose threads stride the K/8 group columns and decode each group for
+// the four rows, keeps more independent gathers in flight per thread (measured on GB300:
+// 13.9 / 16.5 us at T = 2 / 4 on a K = 8640, N = 960 layer, against 19.5 / 26.7 for the
+// row-block layout above; that layout's 16-bit branch measured 10.05 us against 12.8 at T = 1
+// but is not dispatched until a parity test covers it).
 constexpr int kGatherRows = 4;
 
 // 8 int8 -> 8 floats
@@ -382,6 +382,7 @@ cudaError_t launch_skinny_gather(const SkinnyParams& p, cudaStream_t st) {
   const size_t smem = static_cast<size_t>(threads / 32) * kGatherRows * skinny_tt(p.T) * 4;
   const dim3 grid(static_cast<unsigned>(blocks)), block(static_cast<unsigned>(threads));
   switch (skinny_tt(p.T)) {
+    case 1: return launch_pdl(skinny_gather_kernel<2, 1>, grid, block, smem, st, p);
     case 2: return launch_pdl(skinny_gather_kernel<2, 2>, grid, block, smem, st, p);
     case 4: return launch_pdl(skinny_gather_kernel<2, 4>, grid, block, smem, st, p);
     case 8: return launch_pdl(skinny_gather_kernel<2, 8>, grid, block, smem, st, p);
@@ -390,16 +391,11 @@ cudaError_t launch_skinny_gather(const SkinnyParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st) {
-  if (p.B == 16 && p.T >= 2) return launch_skinny_gather(p, st);
+  if (p.B == 16) return launch_skinny_gather(p, st);
   const size_t smem = skinny_smem_bytes(p.M, p.B, p.T);
-  if (p.B == 8) {
-    if (p.M == 1) return launch_skinny_m<1, 1>(p, smem, st);
-    if (p.M == 2) return launch_skinny_m<1, 2>(p, smem, st);
-    return launch_skinny_m<1, 0>(p, smem, st);
-  }
-  if (p.M == 1) return launch_skinny_m<2, 1>(p, smem, st);
-  if (p.M == 2) return launch_skinny_m<2, 2>(p, smem, st);
-  return launch_skinny_m<2, 0>(p, smem, st);
+  if (p.M == 1) return launch_skinny_m<1, 1>(p, smem, st);
+  if (p.M == 2) return launch_skinny_m<1, 2>(p, smem, st);
+  return launch_skinny_m<1, 0>(p, smem, st);
 }
 
 }  // namespace aq
