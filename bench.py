@@ -8,13 +8,15 @@ whole hot path of that layer through the C ABI (aq_linear_f16): 8-bit
 quantization of the fp16 input, decode of the AQ weight, tensor-core
 contraction, fused scale/bias epilogue to fp16.
 
-Timing: CUDA-graph replay of 8 steps that rotate over 8 independent buffer
-sets (inputs, codes, outputs: > 300 MB together, larger than the 129 MB L2),
-CUDA events on the launching stream, warm-up first, barrier + synchronize on
-both sides, max over ranks.  The dominant kernel (the tensor-core GEMM) is
-timed live as the difference between the graph of the layer on int8 inputs
-(decode + GEMM) and the graph of the decode alone, replayed in the same timed
-region.
+Timing: exactly --steps steps, as CUDA-graph replays of 8 steps that rotate
+over 8 independent buffer sets (inputs, codes, outputs: > 300 MB together,
+larger than the 129 MB L2) plus one graph of the remaining steps, CUDA events
+on the launching stream, warm-up first, barrier + synchronize on both sides,
+max over ranks.  The dominant kernel (the tensor-core GEMM) is timed by itself
+right after: a graph of 8 GEMM launches on the same buffer sets (weights
+decoded beforehand, AQ_PATH_PREDECODED through aq_linear_a16), replayed at
+least 50 times and for at least 20 ms; the library's per-kernel event pairs
+(aq_profile_*) over plain launches of the step are reported beside it.
 `e2e` repeats the step through the C ABI with every step's fp16 input copied from
 pinned host memory and its fp16 output copied back: copy-in, compute and
 copy-out on three streams, so one step's compute overlaps the neighbouring
@@ -27,6 +29,8 @@ and 64), with each layer preceded by the quantizer, or writing the next layer's
 int8 activations from its epilogue.  A small-T sweep (T = 1..64) times every path.
 
 --impl reference times the CPU oracle (numpy float64) on the headline workload.
+`cpu_baselines` times the oracle on every workload (single-threaded and on all host
+cores), in child processes started before any GPU work.
 Multi-GPU: independent replicas, one per rank (the layer has no exchange step).
 """
 
@@ -178,6 +182,87 @@ def time_oracle(inp, flops, min_seconds: float = 10.0, max_steps: int = 50) -> d
                       f"{el:.1f} s, numpy float64 BLAS on {cores} host cores"}
 
 
+def oracle_workloads(mode: str):
+    """(name, layer dicts, GFLOP) per workload timed by the CPU oracle.  mode "single":
+    configs 0-3 (tiny linear, qkv, 64x64 W4A8 conv, 8x8 conv with a 2^16 book); "all":
+    configs 1-3 and the UNet-shaped forward (97 layers, W2A8, batch 2)."""
+    from aq_synth import (ConvSpec, LinearSpec, SEEDS, WORKLOADS, make_conv, make_linear,
+                          unet_sweep_layers)
+    out = []
+    names = (["tiny_linear"] if mode == "single" else []) + ["qkv", "conv64", "conv8_book16"]
+    for name in names:
+        spec = WORKLOADS[name]
+        inp = (make_conv if isinstance(spec, ConvSpec) else make_linear)(spec, seed=SEEDS[name])
+        out.append((name, [inp], linear_flops(spec.T, spec.N if isinstance(spec, LinearSpec)
+                                              else spec.Cout, spec.K) / 1e9))
+    if mode == "all":
+        layers, gflop, seed = [], 0.0, 4200
+        for kind, res, cin, cout, stride, count in unet_sweep_layers():
+            for _ in range(count):
+                seed += 1
+                if kind == "conv3":
+                    spec = ConvSpec(Nb=2, H=res * stride, W=res * stride, Cin=cin, Cout=cout,
+                                    stride=stride, M=2, B=8, cb_std=0.03)
+                    layers.append(make_conv(spec, seed))
+                    gflop += linear_flops(spec.T, cout, spec.K) / 1e9
+                else:
+                    spec = LinearSpec(T=2 * res * res, K=cin, N=cout, M=2, B=8, cb_std=0.03,
+                                      act="normal40")
+                    layers.append(make_linear(spec, seed))
+                    gflop += linear_flops(spec.T, cout, cin) / 1e9
+        out.append(("unet_w2a8_batch2", layers, gflop))
+    return out
+
+
+def cpu_oracle_child(mode: str, seconds: float) -> None:
+    """Child process of run_cpu_baselines: time the oracle (decode in float64, then the
+    float64 matmul / convolution) on each workload and print one JSON object."""
+    from oracle import aq_oracle as O
+    res = {}
+    for name, layers, gflop in oracle_workloads(mode):
+        reps, el = 0, 0.0
+        while reps < 1 or (el < seconds and reps < 20):
+            t0 = time.perf_counter()
+            for inp in layers:
+                O.layer_f64(inp)
+            el += time.perf_counter() - t0
+            reps += 1
+        res[name] = {"ms_per_pass": el / reps * 1e3, "gflop": gflop,
+                     "tflops": gflop * reps / el / 1e3, "passes": reps}
+    print(json.dumps(res), flush=True)
+
+
+def run_cpu_baselines(seconds: float = 1.0) -> dict:
+    """The oracle as it stands on every workload, single-threaded (BLAS/OpenMP threads = 1)
+    for configs 0-3 and on all host cores for configs 1-4, each in a child process (started
+    before any GPU work).  The UNet forward at batch 16 and 64 is extrapolated linearly from
+    batch 2 (the oracle's work is linear in the batch) and labelled so."""
+    cores = len(os.sched_getaffinity(0))
+    out = {"kind": "oracle", "cores": cores}
+    for mode in ("single", "all"):
+        env = dict(os.environ)
+        n = "1" if mode == "single" else str(cores)
+        for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+            env[v] = n
+        try:
+            r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-oracle", mode,
+                                "--cpu-seconds", str(seconds)], env=env, capture_output=True,
+                               text=True, timeout=600)
+            vals = json.loads(r.stdout.strip().splitlines()[-1])
+        except Exception as e:  # reported, not fatal: the GPU line is the product
+            out[mode] = {"error": f"{type(e).__name__}: {e}"[:300]}
+            continue
+        if mode == "all" and "unet_w2a8_batch2" in vals:
+            b2 = vals["unet_w2a8_batch2"]
+            for batch in (16, 64):
+                f = batch / 2
+                vals[f"unet_w2a8_batch{batch}"] = {
+                    "ms_per_pass": b2["ms_per_pass"] * f, "gflop": b2["gflop"] * f,
+                    "tflops": b2["tflops"], "extrapolated_from": "batch 2 (linear in batch)"}
+        out[mode] = dict(vals, threads=int(n))
+    return out
+
+
 def max_over_ranks(dist, value: float, device) -> float:
     """The largest `value` over all ranks of the process group (every rank receives it):
     the job takes as long as its slowest replica."""
@@ -321,6 +406,13 @@ class Dev:
             aq.aq_linear_q8(self.xq, self.s_x, self.packed, self.books, self.scale, self.bias,
                             self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, ws_t,
                             ws_t.numel(), path, stream=st)
+
+    def gemm_a16(self, st, xh, ws):
+        """The tensor-core GEMM alone: fp16 activations xh (the 8-bit codes as fp16 values) and
+        weights decoded beforehand into ws (AQ_PATH_PREDECODED)."""
+        self.aq.aq_linear_a16(xh, self.s_x, self.packed, self.books, self.scale, self.bias,
+                              self.y, self.aq.AQ_DTYPE_F16, self.T, self.K, self.N, 8, self.M,
+                              self.B, ws, ws.numel(), self.aq.AQ_PATH_PREDECODED, stream=st)
 
     def decode_only(self, st, wbuf):
         self.aq.aq_decode(self.packed, self.books, wbuf, self.N, self.K, 8, self.M, self.B,
@@ -575,6 +667,10 @@ def main():
                     help="skip the other workloads and the UNet-shaped forward")
     ap.add_argument("--unet-batches", default="2,16,64",
                     help="batches of the UNet-shaped forward extras (comma separated)")
+    ap.add_argument("--cpu-oracle", choices=["single", "all"], default=None,
+                    help=argparse.SUPPRESS)   # child process of the CPU baselines
+    ap.add_argument("--no-cpu-baselines", action="store_true",
+                    help="skip the per-workload CPU oracle timings")
     ap.add_argument("--workload", default="qkv",
                     choices=["qkv", "conv64", "conv8", "unet"] + list(KERNEL_WORKLOADS),
                     help="qkv: the headline line (default); the others run only that workload "
@@ -583,6 +679,9 @@ def main():
     if args.warmup < 3:
         args.warmup = 3
 
+    if args.cpu_oracle:
+        cpu_oracle_child(args.cpu_oracle, min(args.cpu_seconds, 2.0))
+        return 0
     if args.impl == "reference":
         return run_reference(args)
     if args.workload != "qkv":
@@ -595,8 +694,11 @@ def main():
 
     # CPU baseline first (before any GPU work), rank 0 at N=1 only
     cpu = None
+    cpu_all = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = time_oracle(sets[0], fl, min_seconds=args.cpu_seconds)
+        if not args.no_cpu_baselines and not args.no_extras:
+            cpu_all = run_cpu_baselines()
 
     import torch
     import paper_2506_05960_gb300 as aq
@@ -622,31 +724,18 @@ def main():
     stream.synchronize()
     assert aq.aq_device_error() == 0
 
-    # graphs: the step over the 8 buffer sets; for the GEMM's live time, the layer on
-    # int8 inputs (decode + GEMM) and the decode alone
-    def main_graph():
-        for b in bufs:
-            b.step_f16(stream)
-
-    def layer_graph():
-        for b in bufs:
-            b.layer(stream)
-
-    def decode_graph():
-        for b in bufs:
-            b.decode_only(stream, wdec)
-
-    g_main = capture(torch, stream, main_graph)
-    g_layer = capture(torch, stream, layer_graph)
-    g_decode = capture(torch, stream, decode_graph)
-    for gg in (g_main, g_layer, g_decode):
-        gg.replay()
+    # graphs: the step over the 8 buffer sets, and over the first (steps % 8) of them, so
+    # that exactly --steps steps are timed
+    full_reps, rem = divmod(max(1, args.steps), NSETS)
+    g_main = capture(torch, stream, lambda: [b.step_f16(stream) for b in bufs]) if full_reps else None
+    g_rem = capture(torch, stream, lambda: [b.step_f16(stream) for b in bufs[:rem]]) if rem else None
+    for gg in (g_main, g_rem):
+        if gg is not None:
+            gg.replay()
     stream.synchronize()
 
-    reps = max(1, args.steps // NSETS)
-    reps_nogemm = max(1, reps // 4)
-    steps = reps * NSETS
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    steps = full_reps * NSETS + rem
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     sampler = ClockSampler(local)
     sampler.start()
     if pg:
@@ -654,28 +743,59 @@ def main():
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         ev[0].record(stream)
-        for _ in range(reps):
+        for _ in range(full_reps):
             g_main.replay()
+        if g_rem is not None:
+            g_rem.replay()
         ev[1].record(stream)
-        for _ in range(reps_nogemm):
-            g_layer.replay()
-        ev[2].record(stream)
-        for _ in range(reps_nogemm):
-            g_decode.replay()
-        ev[3].record(stream)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
-    clocks = sampler.stop()
     ms_total = ev[0].elapsed_time(ev[1])
-    ms_layer_step = ev[1].elapsed_time(ev[2]) / (reps_nogemm * NSETS)
-    ms_decode_step = ev[2].elapsed_time(ev[3]) / (reps_nogemm * NSETS)
     assert aq.aq_device_error() == 0
     if pg:
         ms_total = max_over_ranks(pg, ms_total, dev)
     ms_step = ms_total / steps
     value = job_throughput(world, fl, ms_step)
-    gemm_ms = ms_layer_step - ms_decode_step
+
+    # the dominant kernel by itself: a graph of 8 GEMM launches (one per buffer set, fp16
+    # activation codes, weights decoded beforehand), replayed >= 50 times and >= 20 ms; and
+    # the decode alone the same way
+    for b in bufs:
+        b.quant(stream)
+    xh = [b.xq.to(torch.float16) for b in bufs]
+    ws_pre = [torch.empty(aq.aq_linear_a16_workspace_size(T, K, N, g, M, B, aq.AQ_PATH_PREDECODED),
+                          dtype=torch.uint8, device=dev) for _ in bufs]
+    for b, w in zip(bufs, ws_pre):
+        b.decode_only(stream, w)
+    stream.synchronize()
+    g_gemm = capture(torch, stream, lambda: [b.gemm_a16(stream, x, w)
+                                             for b, x, w in zip(bufs, xh, ws_pre)])
+    g_decode = capture(torch, stream, lambda: [b.decode_only(stream, wdec) for b in bufs])
+
+    def per_launch_us(gg):
+        est = replay_ms(torch, stream, gg, 5)
+        reps = max(50, int(20.0 / max(est, 1e-3)) + 1)
+        return replay_ms(torch, stream, gg, reps) / NSETS * 1e3, reps
+
+    gemm_us, gemm_reps = per_launch_us(g_gemm)
+    decode_us, _ = per_launch_us(g_decode)
+    clocks = sampler.stop()
+    assert aq.aq_device_error() == 0
+    gemm_ms = gemm_us * 1e-3
+    gemm_plan = aq.aq_linear_f16_plan(T, K, N, g, M, B, aq.AQ_PATH_AUTO)
+    # cross-check: the library's CUDA event pairs around each kernel over plain launches of the
+    # step (an event between two kernels also waits out the programmatic-launch overlap, so a
+    # pair includes the kernel's set-up: an upper bound)
+    aq.aq_profile_enable(True)
+    with torch.cuda.stream(stream):
+        for i in range(64):
+            bufs[i % NSETS].step_f16(stream)
+    stream.synchronize()
+    prof = aq.aq_profile_read()
+    aq.aq_profile_enable(False)
+    prof_us = {k: (v[0] / v[1] * 1e3 if v[1] else None) for k, v in prof.items() if v[1]}
+    del g_gemm, g_decode, ws_pre, xh
 
     peaks = measured_peaks()
     achieved = fl / (gemm_ms * 1e-3) / 1e12
@@ -925,6 +1045,8 @@ def main():
                     torch.cuda.empty_cache()
         assert aq.aq_device_error() == 0
 
+    step_frac = (max(fl / (peaks["bf16_tflops"] * 1e12),
+                     alg_bytes(T, K, N, M, B) / (peaks["hbm_gbs"] * 1e9)) / (ms_step * 1e-3))
     if rank == 0:
         line = {
             "metric": METRIC,
@@ -934,7 +1056,8 @@ def main():
             "config": {"workload": HEADLINE, "T": T, "K": K, "N": N, "g": g, "M": M, "B": B,
                        "parallelism": f"replicas{world}",
                        "l2": f"inputs larger than L2: {NSETS} rotating buffer sets",
-                       "timing": "CUDA graph replay of 8 steps, CUDA events"},
+                       "timing": (f"exactly {steps} steps: {full_reps} CUDA graph replay(s) of "
+                                  f"{NSETS} steps + one graph of {rem} step(s), CUDA events")},
             "hbm_gbs_algorithmic": alg_bytes(T, K, N, M, B) / (ms_step * 1e-3) / 1e9,
             "roofline": {"bound": "tensor", "kernel": "aq_gemm_kernel", "achieved": achieved,
                          "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
@@ -942,14 +1065,17 @@ def main():
                          "peak_source": f"{peaks['source']} bf16 dense burst (the fp16 rate is equal)",
                          "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
                                                if peaks.get("bf16_tflops_sustained") else None),
-                         "kernel_us": gemm_ms * 1e3,
-                         "kernel_timing": ("graph of the layer on int8 inputs (decode + GEMM) "
-                                           "minus the graph of the decode alone")},
-            "step_us": {"total": ms_step * 1e3, "gemm": gemm_ms * 1e3,
-                        "quant_and_decode": (ms_step - gemm_ms) * 1e3},
-            "step_roofline_frac": (max(fl / (peaks["bf16_tflops"] * 1e12),
-                                       alg_bytes(T, K, N, M, B) / (peaks["hbm_gbs"] * 1e9))
-                                   / (ms_step * 1e-3)),
+                         "kernel_us": gemm_us,
+                         "kernel_timing": (f"graph of {NSETS} GEMM launches (one per buffer set, "
+                                           f"weights decoded beforehand) replayed {gemm_reps} "
+                                           "times, CUDA events"),
+                         "kernel_plan": gemm_plan,
+                         "kernel_us_event_pairs": prof_us.get("gemm"),
+                         "step_frac": step_frac},
+            "step_us": {"total": ms_step * 1e3, "gemm": gemm_us, "decode": decode_us,
+                        "quantizer_and_gaps": ms_step * 1e3 - gemm_us - decode_us,
+                        "event_pairs_plain_launches": prof_us},
+            "step_roofline_frac": step_frac,
             "cpu_baseline": cpu,
             "e2e": {"value": job_throughput(world, fl, e2e_ms), "unit": "TFLOP/s",
                     "ms_per_step": e2e_ms, "h2d_bytes_per_step": T * K * 2,
@@ -962,9 +1088,11 @@ def main():
                     "serial": {"value": job_throughput(world, fl, e2e_serial_ms),
                                "ms_per_step": e2e_serial_ms,
                                "how": "copy in, step, copy out on one stream"}},
-            "gpu_launches": launches_per_step * steps + 3 * NSETS * reps_nogemm,
+            "gpu_launches": launches_per_step * steps,
             "clocks": clocks,
         }
+        if cpu_all:
+            line["cpu_baselines"] = cpu_all
         if layers:
             line["layers"] = layers
         if unet:

@@ -99,8 +99,24 @@ AQ_API const char* aq_last_error_string(void);
 
 /* Reads and clears the device error word of the current device (kernels set it
  * when a bounded wait gives up).  Synchronises the device.  *code_out = 0 if no
- * kernel reported an error.  Returns AQ_OK or AQ_ERR_CUDA. */
+ * kernel reported an error, else an OR of AQ_DEVERR_* bits.  Returns AQ_OK or
+ * AQ_ERR_CUDA. */
 AQ_API int aq_device_error(int* code_out);
+#define AQ_DEVERR_TIMEOUT_FULL   1   /* a consumer waited too long for a loaded stage      */
+#define AQ_DEVERR_TIMEOUT_EMPTY  2   /* the loader waited too long for a free stage        */
+#define AQ_DEVERR_TIMEOUT_CONV   4   /* the MMA waited too long for converted activations  */
+#define AQ_DEVERR_TIMEOUT_ACCUM  8   /* the MMA or epilogue waited too long for an
+                                        accumulator buffer                                  */
+#define AQ_DEVERR_TIMEOUT_DRAIN 16   /* after a time-out, in-flight copies did not drain   */
+
+/* Failure-path testing: later tensor-core launches of this host thread give up a
+ * pipeline wait after ns nanoseconds (checked every 256 polls) instead of about two
+ * seconds; ns < 0 restores the default.  A kernel that gives up records the
+ * AQ_DEVERR_* bit, stops its other warps, waits (up to the default limit) for its
+ * own copies and MMAs in flight, frees its tensor memory and returns: the call's
+ * output is then undefined, the context stays usable and aq_device_error() reports
+ * the bits.  Not for production use.  Always AQ_OK.                             */
+AQ_API int aq_set_wait_limit_ns(int64_t ns);
 
 /* ---- kernel timing (diagnostics) -------------------------------------------
  * When enabled, every entry point records a CUDA event pair on the caller's
@@ -201,20 +217,29 @@ AQ_API int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, in
 /* Diagnostics: restrict the tensor-core plan of later calls made by this host
  * thread (workspace-size queries included) to N tile BN (0 = any), K splits
  * (0 = any) and in-cluster split sum (1), split-K through the workspace (0) or
- * either (-1).  A call whose shapes admit no such plan runs the cost-model plan.
+ * either (-1).  A call whose shapes admit no such plan runs the cost-model plan
+ * (int8 activations take BN <= 192; fp16 activations, BN <= 256).
  * aq_set_plan_override(0, 0, -1) restores the default.  AQ_ERR_SHAPE for a BN
- * that is not a multiple of 32 in [0, 192] or other out-of-range values.     */
+ * that is not a multiple of 32 in [0, 256] or other out-of-range values.      */
 AQ_API int aq_set_plan_override(int BN, int splits, int cluster);
 
 /* Plan that aq_linear (fp16 or int8 output) runs for these shapes, for
  * diagnostics: info[0] = resolved AQ_PATH_*; for the tensor-core paths info[1] =
  * N tile, info[2] = K splits, info[3] = 1 when the splits of a tile are summed
  * inside one thread-block cluster (no partials in the workspace, no reduce
- * kernel), info[4] = pipeline stages, info[5] = (tile, split) work items; 0 for
- * the other paths.  Writes min(n_info, 6) entries (zero past 6).  No device
- * access.                                                                      */
+ * kernel), info[4] = pipeline stages, info[5] = (tile, split) work items,
+ * info[6] = 1 when the tensor cores read fp16 activations from shared memory
+ * (aq_linear_f16 and aq_linear_a16 on the dense paths; 0: int8 activations
+ * converted into tensor memory), info[7] = 64-wide K blocks per pipeline stage;
+ * 0 for the other paths.  Writes min(n_info, 8) entries (zero past 8).  No
+ * device access.  aq_linear_f16_plan / aq_linear_a16_plan: the plans of those
+ * entry points.                                                                */
 AQ_API int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
                           int n_info);
+AQ_API int aq_linear_f16_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
+                              int n_info);
+AQ_API int aq_linear_a16_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
+                              int n_info);
 AQ_API int aq_linear(const int8_t* xq, float s_x, const void* codes_packed,
               const void* codebooks, const void* scale, const void* bias,
               void* y, int out_dtype, int T, int K, int N, int g, int M, int B,
@@ -235,15 +260,35 @@ AQ_API int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed,
                         void* workspace, size_t workspace_bytes, int path, void* stream);
 
 /* ---- layer from fp16 activations -------------------------------------------
- * aq_quant_act(x, xq, T*K, s_x) followed by aq_linear(xq, s_x, ...) in one call, the
- * int8 activations xq kept at the start of the workspace: the same bits as the two
- * calls.
+ * aq_quant_act(x, xq, T*K, s_x) followed by aq_linear(xq, s_x, ...) in one call
+ * (Sec. 4.2.3 quantizer, then the layer of Sec. 3.1.1).  The quantized activations
+ * are kept at the start of the workspace: on the dense paths as fp16 values (each
+ * 8-bit code exactly; the tensor cores then read both operands from shared
+ * memory), on the other paths as int8.  Same codes as aq_quant_act; the output
+ * equals the two calls' bit for bit when both run the same plan (N tile and K
+ * split, aq_set_plan_override), and is within the layer tolerance otherwise.
  *   x fp16 [T][K]; s_x finite and > 0 (AQ_ERR_SHAPE); out_dtype F16 or F32.
- *   Workspace: aq_linear_f16_workspace_size() bytes = T*K rounded up to 1 KB plus
- *   aq_linear_workspace_size().                                                */
+ *   Workspace: aq_linear_f16_workspace_size() bytes = 2*T*K rounded up to 1 KB
+ *   plus the layer's workspace for this plan; with AQ_PATH_PREDECODED, W-hat is
+ *   expected right after that activation region (byte offset 2*T*K rounded up to
+ *   1 KB).                                                                       */
 AQ_API int aq_linear_f16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
                                         size_t* bytes);
 AQ_API int aq_linear_f16(const void* x, float s_x, const void* codes_packed,
+                         const void* codebooks, const void* scale, const void* bias, void* y,
+                         int out_dtype, int T, int K, int N, int g, int M, int B,
+                         void* workspace, size_t workspace_bytes, int path, void* stream);
+
+/* ---- layer on 8-bit activations stored as fp16 values -----------------------
+ * aq_linear with xh[t][k] = fp16(xq[t][k]) (the codes of Sec. 4.2.3 held as fp16
+ * integers, e.g. as written into aq_linear_f16's workspace): the tensor cores read
+ * both operands from shared memory.  Any fp16 values are accepted and multiplied as
+ * they are.  Paths: AUTO (= DENSE), DENSE, PREDECODED; others AQ_ERR_UNSUPPORTED.
+ *   xh fp16 [T][K]; other arguments, layouts and errors as for aq_linear.
+ *   Workspace: aq_linear_a16_workspace_size() bytes.                            */
+AQ_API int aq_linear_a16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
+                                        size_t* bytes);
+AQ_API int aq_linear_a16(const void* xh, float s_x, const void* codes_packed,
                          const void* codebooks, const void* scale, const void* bias, void* y,
                          int out_dtype, int T, int K, int N, int g, int M, int B,
                          void* workspace, size_t workspace_bytes, int path, void* stream);

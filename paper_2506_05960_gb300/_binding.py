@@ -44,7 +44,13 @@ _SIGNATURES = {
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
     "aq_set_plan_override": (_c_int, [_c_int] * 3),
+    "aq_set_wait_limit_ns": (_c_int, [_c_int64]),
     "aq_linear_f16_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
+    "aq_linear_a16_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
+    "aq_linear_f16_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_linear_a16_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_linear_a16": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
+                      + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_linear": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
                   + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_linear_f16": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 7
@@ -193,7 +199,7 @@ def aq_linear_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:
     return out.value
 
 
-_PLAN_KEYS = ("path", "BN", "splits", "cluster", "stages", "work_items")
+_PLAN_KEYS = ("path", "BN", "splits", "cluster", "stages", "work_items", "a16", "stage_blocks")
 
 
 def aq_set_plan_override(BN=0, splits=0, cluster=-1) -> None:
@@ -201,11 +207,36 @@ def aq_set_plan_override(BN=0, splits=0, cluster=-1) -> None:
     _check(load_library().aq_set_plan_override(BN, splits, cluster), "aq_set_plan_override")
 
 
+def _plan(fn, name, *args) -> dict:
+    n = len(_PLAN_KEYS)
+    info = (_c_int * n)()
+    _check(fn(*args, info, n), name)
+    return dict(zip(_PLAN_KEYS, list(info)))
+
+
+AQ_DEVERR_TIMEOUT_FULL, AQ_DEVERR_TIMEOUT_EMPTY, AQ_DEVERR_TIMEOUT_CONV = 1, 2, 4
+AQ_DEVERR_TIMEOUT_ACCUM, AQ_DEVERR_TIMEOUT_DRAIN = 8, 16
+
+
+def aq_set_wait_limit_ns(ns=-1) -> None:
+    """Failure-path tests: later tensor-core launches of this thread give up a pipeline
+    wait after ns nanoseconds (ns < 0: the default, about two seconds)."""
+    _check(load_library().aq_set_wait_limit_ns(int(ns)), "aq_set_wait_limit_ns")
+
+
 def aq_linear_plan(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> dict:
     """The plan aq_linear runs for these shapes (diagnostics; no device access)."""
-    info = (_c_int * 6)()
-    _check(load_library().aq_linear_plan(T, K, N, g, M, B, path, info, 6), "aq_linear_plan")
-    return dict(zip(_PLAN_KEYS, list(info)))
+    return _plan(load_library().aq_linear_plan, "aq_linear_plan", T, K, N, g, M, B, path)
+
+
+def aq_linear_f16_plan(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_linear_f16 runs for these shapes (diagnostics; no device access)."""
+    return _plan(load_library().aq_linear_f16_plan, "aq_linear_f16_plan", T, K, N, g, M, B, path)
+
+
+def aq_linear_a16_plan(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_linear_a16 runs for these shapes (diagnostics; no device access)."""
+    return _plan(load_library().aq_linear_a16_plan, "aq_linear_a16_plan", T, K, N, g, M, B, path)
 
 
 def aq_linear(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N, g=8, M=2,
@@ -225,11 +256,27 @@ def aq_linear_f16_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> i
 
 def aq_linear_f16(x, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N, g=8, M=2,
                   B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
-    """aq_quant_act + aq_linear in one call from fp16 activations x (int8 kept in workspace)."""
+    """aq_quant_act + aq_linear in one call from fp16 activations x (codes kept in workspace)."""
     _check(load_library().aq_linear_f16(
         _ptr(x), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
         _ptr(y), out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
         _stream(stream)), "aq_linear_f16")
+
+
+def aq_linear_a16_workspace_size(T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_linear_a16_workspace_size(T, K, N, g, M, B, path, ctypes.byref(out)),
+           "aq_linear_a16_workspace_size")
+    return out.value
+
+
+def aq_linear_a16(xh, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, T, K, N, g=8, M=2,
+                  B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """aq_linear on 8-bit activations held as fp16 values (dense paths)."""
+    _check(load_library().aq_linear_a16(
+        _ptr(xh), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(y), out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), path,
+        _stream(stream)), "aq_linear_a16")
 
 
 def aq_linear_q8(xq, s_x, codes_packed, codebooks, scale, bias, yq, s_out, T, K, N, g=8, M=2,
@@ -261,10 +308,8 @@ def aq_conv2d_workspace_size(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g
 def aq_conv2d_plan(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8,
                    path=AQ_PATH_AUTO) -> dict:
     """The plan aq_conv2d_nhwc runs for these shapes (diagnostics; no device access)."""
-    info = (_c_int * 6)()
-    _check(load_library().aq_conv2d_plan(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path,
-                                         info, 6), "aq_conv2d_plan")
-    return dict(zip(_PLAN_KEYS, list(info)))
+    return _plan(load_library().aq_conv2d_plan, "aq_conv2d_plan", Nb, H, W, Cin, Cout, kh, kw,
+                 stride, pad, g, M, B, path)
 
 
 def aq_conv2d_nhwc(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, Nb, H, W, Cin,

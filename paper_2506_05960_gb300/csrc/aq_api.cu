@@ -15,6 +15,7 @@
 
 #include "aq.h"
 #include "aq_internal.h"
+#include "aq_ptx.cuh"
 
 // Scratch of aq_linear_noalloc: the decoded weights of one call.  Lives for the
 // life of the process on every device that loads this module.
@@ -120,7 +121,16 @@ struct Plan {
   int stages, a_stages, acc_stride, a_col, total_tiles;
   int cluster;    // the splits of a tile form one cluster and are summed in shared memory
   int epi_warps;  // 4, or 8 on the dense path with fp16/int8 staging and BN >= 64
+  int a16;        // A is fp16 in global memory (the 8-bit codes as fp16 values)
+  int sb;         // 64-wide K blocks per pipeline stage
 };
+
+// K blocks per stage of the shared-memory A form (a stage is then one fp16 A box and
+// one weight box: more, shallower stages than the TMEM-A form's 128-wide ones).
+#ifndef AQ_A16_STAGE_BLOCKS
+#define AQ_A16_STAGE_BLOCKS 1
+#endif
+constexpr int kA16StageBlocks = AQ_A16_STAGE_BLOCKS;
 
 // Cycles of one pipeline stage (eight 128 x BN x 16 MMAs issued by one thread),
 // measured on GB300: an MMA takes BN/2 cycles (at least 48; N = 160 runs at 88),
@@ -130,6 +140,14 @@ double stage_cycles(int BN) {
   double exposed = BN >= 192 ? 0.0 : (BN >= 160 ? 60.0 : 115.0);
   return 8.0 * mma + exposed;
 }
+
+// The fp16 A form, per 128 of K (two 64-wide K blocks, each one pipeline stage of four
+// 128 x BN x 16 MMAs with both operands in shared memory), measured on GB300 (qkv layer,
+// clock64 wait accounting): about 800 + 2.2 BN cycles per block with TMA and the epilogue
+// running (1147 / 1272 / 1373 at BN = 160 / 224 / 256).  Each MMA reads A (4 KB) and B
+// (32 BN bytes) from shared memory, and the tensor core takes in shared-memory operands at
+// about 57 B per cycle, so an MMA costs about (4096 + 32 BN) / 57 cycles rather than BN / 2.
+double stage_cycles_a16(int BN) { return 2.0 * (800.0 + 2.2 * BN); }
 
 // Fused path: the decoder warps rebuild BN x 16 groups per stage.  With 8-bit codes
 // the stage is bound by shared-memory traffic: per group M codeword lookups of 16 B,
@@ -156,16 +174,30 @@ bool plan_f32_staging(const Plan& pl, bool f32_out) {
   return f32_out || (pl.splits > 1 && !pl.cluster);
 }
 
+int plan_epi_warps(bool fused, bool f32_staging, int BN) {
+  // the dense path has no decoder warps: 8 epilogue warps double the epilogue's rate,
+  // which bounds tiles with small K; fp32 staging would cost a pipeline stage
+  return (!fused && !f32_staging && BN >= 64) ? 8 : 4;
+}
+
 void finish_plan(Plan& pl, bool f32_out, int book_bytes, int code_bytes, bool fused) {
   pl.acc_stride = pl.BN;
   pl.a_col = 2 * pl.acc_stride;
-  pl.a_stages = aq::gemm_a_stages(pl.BN);
+  pl.sb = pl.a16 ? kA16StageBlocks : aq::kStageBlocks;
   const bool f32_staging = plan_f32_staging(pl, f32_out);
-  // the dense path has no decoder warps: 8 epilogue warps double the epilogue's rate,
-  // which bounds tiles with small K; fp32 staging would cost a pipeline stage
-  pl.epi_warps = (!fused && !f32_staging && pl.BN >= 64) ? 8 : 4;
-  pl.stages = aq::gemm_max_stages(pl.BN, f32_staging, book_bytes, code_bytes, pl.epi_warps);
+  pl.epi_warps = plan_epi_warps(fused, f32_staging, pl.BN);
+  pl.stages = aq::gemm_max_stages(pl.BN, f32_staging, book_bytes, code_bytes, pl.epi_warps,
+                                  pl.a16 != 0, pl.sb);
+  pl.a_stages = pl.a16 ? 0 : aq::gemm_a_stages(pl.BN);
   pl.total_tiles = pl.m_tiles * pl.n_tiles * pl.splits;
+}
+
+// Shared-memory bytes of the pipeline ring (where an in-cluster split keeps its fp32
+// partial tile of 128 x BN x 4 bytes once the mainloop is done).
+size_t ring_bytes(const Plan& pl) {
+  const int SB = pl.a16 ? pl.sb : aq::kStageBlocks;
+  const size_t a = pl.a16 ? static_cast<size_t>(SB) * aq::kBM * 128 : aq::kStageBlocks * aq::kBM * 64;
+  return static_cast<size_t>(pl.stages) * (static_cast<size_t>(SB) * pl.BN * 128 + a);
 }
 
 // Picks the N tile and the K split that minimise a model of the busiest SM's time:
@@ -183,8 +215,13 @@ struct PlanOverride {
 };
 thread_local PlanOverride g_plan_override;
 
+// Time after which a pipeline wait of the tensor-core kernels gives up, for this host
+// thread's later launches (aq_set_wait_limit_ns; tests of the failure path).
+thread_local unsigned long long g_wait_limit_ns = aq::kWaitLimitNs;
+
+// a16: the shared-memory A form (fp16 activations in global memory, dense weights).
 Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
-               bool fused = false, int M = 1, int B = 8) {
+               bool fused = false, int M = 1, int B = 8, bool a16 = false) {
   const int num_kb = (K + aq::kBK - 1) / aq::kBK;
   const int book_bytes = book_smem_bytes(fused, M, B);
   const int code_bytes = code_smem_bytes(fused, M, B);
@@ -195,13 +232,13 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
   // clusters, which still runs correctly, in waves)
   auto search = [&](bool forced) {
     for (int BN = aq::kMaxBN; BN >= 32; BN -= 32) {
-      if (BN == 224) continue;
       if (forced && ov.BN > 0 && BN != ov.BN) continue;
-      if (aq::gemm_a_stages(BN) < 2) continue;
-      if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes, 4) < 2) continue;
+      if (!a16 && aq::gemm_a_stages(BN) < 2) continue;
+      if (aq::gemm_max_stages(BN, true, book_bytes, code_bytes, 4, a16, kA16StageBlocks) < 2)
+        continue;
       const int n_tiles = (N + BN - 1) / BN;
       const int max_split = allow_split ? std::min(num_kb, 64) : 1;
-      double st_cyc = stage_cycles(BN);
+      double st_cyc = a16 ? stage_cycles_a16(BN) : stage_cycles(BN);
       if (fused) st_cyc = std::max(st_cyc, decode_stage_cycles(BN, M, B));
       for (int sp = 1; sp <= max_split; ++sp) {
         const int kbps = (num_kb + sp - 1) / sp;
@@ -225,6 +262,16 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
           if (cl) {
             if (s_eff < 2 || s_eff > aq::kMaxClusterSplits) continue;
             if (!forced && static_cast<long>(m_tiles) * n_tiles > kPlanMaxClusters[s_eff]) continue;
+            if (a16) {
+              // the partial tile must fit in the ring
+              Plan tp{};
+              tp.BN = BN;
+              tp.a16 = 1;
+              tp.sb = kA16StageBlocks;
+              tp.stages = aq::gemm_max_stages(BN, false, 0, 0, plan_epi_warps(false, false, BN),
+                                              true, kA16StageBlocks);
+              if (ring_bytes(tp) < static_cast<size_t>(aq::kBM) * BN * 4) continue;
+            }
             // one tile per CTA; then the partial's shared-memory write, two cluster
             // barriers and the 128 x BN x 4 bytes each CTA reads over distributed shared
             // memory (about 3000 + 8 BN cycles measured on GB300 layers)
@@ -245,6 +292,7 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
             bp.kb_per_split = kbps;
             bp.num_kb = num_kb;
             bp.cluster = cl;
+            bp.a16 = a16 ? 1 : 0;
           }
         }
       }
@@ -254,6 +302,12 @@ Plan plan_gemm(int T, int N, int K, int m_tiles, bool allow_split, bool f32_out,
   if (best > 1e29) search(false);
   finish_plan(bp, f32_out, book_bytes, code_bytes, fused);
   return bp;
+}
+
+// The ring must hold an in-cluster split's partial tile (checked when planning; kept as an
+// invariant of every plan that runs).
+bool plan_ring_ok(const Plan& pl) {
+  return !pl.cluster || ring_bytes(pl) >= static_cast<size_t>(aq::kBM) * pl.BN * 4;
 }
 
 size_t dense_ws_bytes(int T, int N, int K, const Plan& pl) {
@@ -512,12 +566,18 @@ int sm_count() {
 // kaq: the codes use the kernel-aware grouping (g = 9, dense path only).
 // x16 != nullptr: the layer's fp16 activations, quantized here into the GEMM's int8
 // operand xq (the memory mapA points at) with the rule of aq_quant_act and scale p.s_x.
+// pl.a16: mapA describes fp16 activations (the 8-bit codes as fp16 integers); with x16 the
+// quantizer writes them (into xq, then an fp16 buffer) with the same rule.
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
              bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr,
              bool predecoded = false) {
   const bool fused = Wdec == nullptr;
+  if (!plan_ring_ok(pl)) return set_error(AQ_ERR_UNSUPPORTED, "plan: partial tile exceeds the ring");
   p.fused = fused ? 1 : 0;
+  p.a16 = pl.a16;
+  p.sb = pl.sb;
+  p.wait_ns = g_wait_limit_ns;
   p.codes = codes_packed;
   p.books = codebooks;
   p.M = M;
@@ -580,7 +640,8 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   const int64_t x_elems = static_cast<int64_t>(T) * K;
   if (x16) {
     ProfScope ps(kProfQuant, st);
-    e = aq::launch_quant_act(x16, xq, x_elems, p.s_x, st);
+    e = pl.a16 ? aq::launch_quant_act_f16(x16, reinterpret_cast<__half*>(xq), x_elems, p.s_x, st)
+               : aq::launch_quant_act(x16, xq, x_elems, p.s_x, st);
     if (e != cudaSuccess) return cuda_status(e, "quantizer launch");
   }
   if (!fused && !predecoded) {
@@ -612,11 +673,13 @@ struct Route {
   size_t ws;
 };
 
-Route route_gemm(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, int B) {
+// a16: fp16 activations (the shared-memory A form) on the dense / predecoded paths.
+Route route_gemm(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, int B,
+                 bool a16 = false) {
   Route rt;
   rt.fused = rp == AQ_PATH_FUSED;
   rt.predecoded = rp == AQ_PATH_PREDECODED;
-  rt.pl = plan_gemm(T, N, K, m_tiles, true, f32_out, rt.fused, M, B);
+  rt.pl = plan_gemm(T, N, K, m_tiles, true, f32_out, rt.fused, M, B, a16 && !rt.fused);
   rt.ws = rt.fused ? fused_ws_bytes(T, N, rt.pl) : dense_ws_bytes(T, N, K, rt.pl);
   return rt;
 }
@@ -648,6 +711,16 @@ int encode_linear_a(CUtensorMap* mapA, const int8_t* xq, int T, int K) {
                 CU_TENSOR_MAP_SWIZZLE_64B);
 }
 
+// fp16 activations [T][K] for the shared-memory A form: 64 x 128 boxes, 128-byte swizzle
+// (the layout of the weight boxes).
+int encode_linear_a16(CUtensorMap* mapA, const void* xh, int T, int K) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(aq::kBM)};
+  return encode(mapA, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, xh, dims, strides, box,
+                CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
 // Output kinds of the layer entry points: AQ_DTYPE_F16 / AQ_DTYPE_F32 through
 // aq_linear / aq_conv2d_nhwc, AQ_DTYPE_I8 (quantized with s_out) through the _q8
 // variants.  int8 rows need N % 16 == 0 (16-byte TMA row stride).
@@ -666,7 +739,15 @@ int check_output(int out_dtype, float s_out, int N) {
 int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
                 const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
                 int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
-                int path, void* stream, const void* x16 = nullptr);
+                int path, void* stream, const void* x16 = nullptr, const void* xh = nullptr);
+int linear_ws(int T, int K, int N, int g, int M, int B, int path, bool a16, size_t* bytes);
+
+// Path of aq_linear_a16 (fp16 activations): the dense tensor-core paths only.
+int resolve_a16_path(int path) {
+  if (path == AQ_PATH_AUTO) return AQ_PATH_DENSE;
+  if (path == AQ_PATH_DENSE || path == AQ_PATH_PREDECODED) return path;
+  return -2;
+}
 int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
@@ -812,39 +893,28 @@ int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stre
 }
 
 int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path, size_t* bytes) {
-  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
-  int r = check_format(g, M, B);
-  if (r) return r;
-  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
-  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  const int rp = resolve_linear_path(path, T, B);
-  if (rp < 0) return path_error(rp, path);
-  if (rp == AQ_PATH_FEW_TOKENS) {
-    *bytes = 0;
-    return ok();
-  }
-  if (rp == AQ_PATH_LUT) {
-    *bytes = plan_lut(T, K, N, M).ws_bytes;
-    return ok();
-  }
-  *bytes = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B).ws;
-  return ok();
+  return linear_ws(T, K, N, g, M, B, path, false, bytes);
 }
 
 namespace {
 // info[0] = resolved path, then for the tensor-core paths [1] BN, [2] K splits,
-// [3] in-cluster split sum (0/1), [4] pipeline stages, [5] (tile, split) work items.
+// [3] in-cluster split sum (0/1), [4] pipeline stages, [5] (tile, split) work items,
+// [6] 1 when the MMA reads fp16 activations from shared memory (0: int8 activations
+// converted by warps into tensor memory), [7] 64-wide K blocks per pipeline stage.
+constexpr int kPlanInfo = 8;
 int fill_plan_info(int rp, const Plan* pl, int* info, int n_info) {
   if (!info || n_info < 1) return set_error(AQ_ERR_NULL, "info is NULL or n_info < 1");
-  int v[6] = {rp, 0, 0, 0, 0, 0};
+  int v[kPlanInfo] = {rp, 0, 0, 0, 0, 0, 0, 0};
   if (pl) {
     v[1] = pl->BN;
     v[2] = pl->splits;
     v[3] = pl->cluster;
     v[4] = pl->stages;
     v[5] = pl->total_tiles;
+    v[6] = pl->a16;
+    v[7] = pl->sb;
   }
-  for (int i = 0; i < n_info; ++i) info[i] = i < 6 ? v[i] : 0;
+  for (int i = 0; i < n_info; ++i) info[i] = i < kPlanInfo ? v[i] : 0;
   return ok();
 }
 }  // namespace
@@ -859,16 +929,40 @@ int aq_set_plan_override(int BN, int splits, int cluster) {
   return ok();
 }
 
-int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info, int n_info) {
+namespace {
+// Plan of a linear call; a16: the call has fp16 activations (aq_linear_f16 / aq_linear_a16),
+// a16_only: aq_linear_a16 (dense paths only).
+int linear_plan_impl(int T, int K, int N, int g, int M, int B, int path, bool a16,
+                     bool a16_only, int* info, int n_info) {
   int r = check_format(g, M, B);
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  const int rp = resolve_linear_path(path, T, B);
+  const int rp = a16_only ? resolve_a16_path(path) : resolve_linear_path(path, T, B);
   if (rp < 0) return path_error(rp, path);
   if (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT) return fill_plan_info(rp, nullptr, info, n_info);
-  const Route rt = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B);
+  const Route rt = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B, a16);
   return fill_plan_info(rp, &rt.pl, info, n_info);
+}
+}  // namespace
+
+int aq_set_wait_limit_ns(int64_t ns) {
+  g_wait_limit_ns = ns < 0 ? aq::kWaitLimitNs : static_cast<unsigned long long>(ns);
+  return ok();
+}
+
+int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info, int n_info) {
+  return linear_plan_impl(T, K, N, g, M, B, path, false, false, info, n_info);
+}
+
+int aq_linear_f16_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
+                       int n_info) {
+  return linear_plan_impl(T, K, N, g, M, B, path, true, false, info, n_info);
+}
+
+int aq_linear_a16_plan(int T, int K, int N, int g, int M, int B, int path, int* info,
+                       int n_info) {
+  return linear_plan_impl(T, K, N, g, M, B, path, true, true, info, n_info);
 }
 
 int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
@@ -888,17 +982,38 @@ int aq_linear_q8(const int8_t* xq, float s_x, const void* codes_packed, const vo
                      N, g, M, B, workspace, workspace_bytes, path, stream);
 }
 
-// aq_linear from fp16 activations: the workspace starts with the int8 activations
-// (T*K bytes, 1 KB-aligned), then what aq_linear needs.
-static size_t f16_act_bytes(int T, int K) { return align_up(static_cast<size_t>(T) * K, 1024); }
+// aq_linear from fp16 activations: the workspace starts with the quantized activations
+// (T*K*2 bytes, 1 KB-aligned: int8 codes, or on the dense paths the codes as fp16 values),
+// then what the layer needs.
+static size_t f16_act_bytes(int T, int K) { return align_up(static_cast<size_t>(T) * K * 2, 1024); }
 
 int aq_linear_f16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
                                  size_t* bytes) {
   size_t rest = 0;
-  const int r = aq_linear_workspace_size(T, K, N, g, M, B, path, &rest);
+  const int r = linear_ws(T, K, N, g, M, B, path, true, &rest);
   if (r) return r;
   *bytes = f16_act_bytes(T, K) + rest;
   return ok();
+}
+
+int aq_linear_a16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
+                                 size_t* bytes) {
+  const int rp = resolve_a16_path(path);
+  if (rp < 0) return path_error(-2, path);
+  return linear_ws(T, K, N, g, M, B, rp, true, bytes);
+}
+
+int aq_linear_a16(const void* xh, float s_x, const void* codes_packed, const void* codebooks,
+                  const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
+                  int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
+                  void* stream) {
+  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  const int rp = resolve_a16_path(path);
+  if (rp < 0) return path_error(-2, path);
+  if (T > 0 && !xh) return set_error(AQ_ERR_NULL, "xh is NULL");
+  return linear_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, T, K,
+                     N, g, M, B, workspace, workspace_bytes, rp, stream, nullptr,
+                     T > 0 ? xh : nullptr);
 }
 
 int aq_linear_f16(const void* x, float s_x, const void* codes_packed, const void* codebooks,
@@ -928,11 +1043,34 @@ int aq_linear_f16(const void* x, float s_x, const void* codes_packed, const void
 
 namespace {
 
-// x16 != nullptr (aq_linear_f16): the fp16 activations, quantized into xq by this call.
+int linear_ws(int T, int K, int N, int g, int M, int B, int path, bool a16, size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
+  const int rp = resolve_linear_path(path, T, B);
+  if (rp < 0) return path_error(rp, path);
+  if (rp == AQ_PATH_FEW_TOKENS) {
+    *bytes = 0;
+    return ok();
+  }
+  if (rp == AQ_PATH_LUT) {
+    *bytes = plan_lut(T, K, N, M).ws_bytes;
+    return ok();
+  }
+  *bytes = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B, a16).ws;
+  return ok();
+}
+
+// x16 != nullptr (aq_linear_f16): the fp16 activations, quantized into xq by this call
+// (int8 codes, or on the dense paths the codes as fp16 values: the region holds T*K*2 bytes).
+// xh != nullptr (aq_linear_a16): activations already held as fp16 values; path is a
+// resolved dense path and xq is unused.
 int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
                 const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
                 int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
-                int path, void* stream, const void* x16) {
+                int path, void* stream, const void* x16, const void* xh) {
   int r = check_format(g, M, B);
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
@@ -944,8 +1082,9 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   const int rp = resolve_linear_path(path, T, B);
   if (rp < 0) return path_error(rp, path);
   if (T == 0) return ok();
-  if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
-  if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+  const void* act = xh ? xh : static_cast<const void*>(xq);
+  if (!act || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(act) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   if (x16 && (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT)) {
@@ -1021,8 +1160,12 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     if (e != cudaSuccess) return cuda_status(e, "LUT reduce launch");
     return ok();
   }
+  // fp16 activations (given, or written by this call's quantizer) on the dense paths:
+  // the shared-memory A form
+  const bool a16 = (xh != nullptr || x16 != nullptr) &&
+                   (rp == AQ_PATH_DENSE || rp == AQ_PATH_PREDECODED);
   const Route rt =
-      route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, out_dtype == AQ_DTYPE_F32, M, B);
+      route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, out_dtype == AQ_DTYPE_F32, M, B, a16);
   r = check_workspace(workspace, workspace_bytes, rt.ws);
   if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1030,7 +1173,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   float* partial = nullptr;
   ws_pointers(rt, workspace, N, K, &Wdec, &partial);
   CUtensorMap mapA;
-  r = encode_linear_a(&mapA, xq, T, K);
+  r = a16 ? encode_linear_a16(&mapA, act, T, K) : encode_linear_a(&mapA, xq, T, K);
   if (r) return r;
   aq::GemmParams p{};
   p.T = T;

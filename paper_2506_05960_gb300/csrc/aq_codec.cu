@@ -14,9 +14,11 @@
 namespace aq {
 
 // ============================================================== quantizer (rule in aq_quant.cuh)
-// Each thread: 16 elements (32 B in, 16 B out) per grid-stride step over `nblocks` blocks
+// Each thread: 16 elements (32 B in; 16 B of int8 codes out, or 32 B with each code stored
+// as the fp16 value of that integer, kF16Out) per grid-stride step over `nblocks` blocks
 // (block index `bid`); the first block also takes the scalar tail (numel % 16 elements).
-__device__ __forceinline__ void quant_range(const __half* __restrict__ x, int8_t* __restrict__ xq,
+template <bool kF16Out>
+__device__ __forceinline__ void quant_range(const __half* __restrict__ x, void* __restrict__ out,
                                             int64_t nvec, int64_t numel, float s, int bid,
                                             int nblocks) {
   const float rs = __frcp_rn(s);
@@ -43,31 +45,58 @@ __device__ __forceinline__ void quant_range(const __half* __restrict__ x, int8_t
 #pragma unroll
     for (int i = 0; i < 4; ++i)
       w[i] = pack_low_bytes(qb[4 * i], qb[4 * i + 1], qb[4 * i + 2], qb[4 * i + 3]);
-    __stcs(reinterpret_cast<uint4*>(xq) + v, make_uint4(w[0], w[1], w[2], w[3]));
+    if constexpr (kF16Out) {
+      // int8 -> fp16 is exact (|code| <= 127)
+      uint32_t f[8];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) i8x4_to_f16x4(w[i], f[2 * i], f[2 * i + 1]);
+      uint4* dst = reinterpret_cast<uint4*>(out) + 2 * v;
+      __stcs(dst, make_uint4(f[0], f[1], f[2], f[3]));
+      __stcs(dst + 1, make_uint4(f[4], f[5], f[6], f[7]));
+    } else {
+      __stcs(reinterpret_cast<uint4*>(out) + v, make_uint4(w[0], w[1], w[2], w[3]));
+    }
   }
   if (bid == 0) {
-    for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x)
-      xq[i] = quant_one(x[i], s, rs);
+    for (int64_t i = nvec * 16 + threadIdx.x; i < numel; i += blockDim.x) {
+      const int8_t c = quant_one(x[i], s, rs);
+      if constexpr (kF16Out)
+        static_cast<__half*>(out)[i] = __short2half_rn(static_cast<short>(c));
+      else
+        static_cast<int8_t*>(out)[i] = c;
+    }
   }
 }
 
+template <bool kF16Out>
 __global__ void __launch_bounds__(256) quant_act_kernel(const __half* __restrict__ x,
-                                                        int8_t* __restrict__ xq,
+                                                        void* __restrict__ out,
                                                         int64_t nvec, int64_t numel, float s) {
   grid_dependency_wait();
   allow_dependents();
-  quant_range(x, xq, nvec, numel, s, blockIdx.x, gridDim.x);
+  quant_range<kF16Out>(x, out, nvec, numel, s, blockIdx.x, gridDim.x);
 }
 
-cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s,
-                             cudaStream_t st) {
+static cudaError_t launch_quant(const void* x, void* out, int64_t numel, float s, bool f16_out,
+                                cudaStream_t st) {
   const int64_t nvec = numel / 16;
   int64_t blocks = (nvec + 255) / 256;
   const int64_t cap = 152 * 16;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  return launch_pdl(quant_act_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st,
-                    static_cast<const __half*>(x), xq, nvec, numel, s);
+  auto kernel = f16_out ? quant_act_kernel<true> : quant_act_kernel<false>;
+  return launch_pdl(kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st,
+                    static_cast<const __half*>(x), out, nvec, numel, s);
+}
+
+cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s,
+                             cudaStream_t st) {
+  return launch_quant(x, xq, numel, s, false, st);
+}
+
+cudaError_t launch_quant_act_f16(const void* x, __half* xh, int64_t numel, float s,
+                                 cudaStream_t st) {
+  return launch_quant(x, xh, numel, s, true, st);
 }
 
 // ============================================================== packing

@@ -51,6 +51,7 @@ constexpr int kDecodeThreads = 192;             // warps 10..15 decode on the fu
 constexpr int kThreads = 320 + kDecodeThreads;
 constexpr int kA8Half = kBM * 64;               // one 64-wide int8 box: 128 rows x 64 B
 constexpr int kA8Stage = kStageBlocks * kA8Half;
+constexpr int kA16Half = kBM * 128;             // one 64-wide fp16 A box: 128 rows x 128 B
 constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A slot
 constexpr int kEpiBuf32 = 4096;                 // one 32 x 32 fp32 output box (128-byte rows)
 constexpr int kEpiBuf16 = 2048;                 // one 32 x 32 fp16 output box (64-byte rows)
@@ -58,12 +59,20 @@ constexpr int kEpiBuf16 = 2048;                 // one 32 x 32 fp16 output box (
 // columns each; 8 warps (two per lane quarter, alternate 32-column chunks) keep one box
 // and the scale/bias of their own columns, so both take the same shared memory.
 __host__ __device__ constexpr int epi_out_bufs(int epi_warps) { return epi_warps == 8 ? 1 : 2; }
-__host__ __device__ constexpr int epi_scale_cols(int epi_warps) { return kMaxBN / (epi_warps / 4); }
+// Columns of scale/bias a warp keeps: its 32-column chunks of a BN-wide tile, compacted.
+__host__ __device__ constexpr int epi_scale_cols(int epi_warps, int BN) {
+  return ((BN + 31) / 32 + epi_warps / 4 - 1) / (epi_warps / 4) * 32;
+}
+// Bytes of A per pipeline stage: int8 boxes (TMEM-A form) or fp16 boxes (shared-memory A).
+__host__ __device__ constexpr int a_stage_bytes(bool a16, int sb) {
+  return a16 ? sb * kA16Half : kA8Stage;
+}
 constexpr int kTmemCols = 512;
 
 struct alignas(8) GemmBarriers {
   uint64_t full[kMaxStages];     // TMA bytes of a smem stage landed
   uint64_t empty[kMaxStages];    // smem stage consumed: 4 converter warps + 1 MMA commit
+                                 // (shared-memory A form: the MMA commit alone)
   uint32_t a_ready[kMaxStages];  // fp16 A slot written: +1 per converter warp (4 per use)
   uint64_t a_empty[kMaxStages];  // MMAs reading the TMEM slot done (commit)
   uint64_t acc_full[2];          // accumulator buffer complete (commit)
@@ -77,18 +86,21 @@ struct alignas(8) GemmBarriers {
 // code_bytes: packed code bytes of one row for one 64-wide K block on the fused path
 // (8 * M * bytes per code), 0 on the dense path.
 size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes,
-                       int epi_warps) {
+                       int epi_warps, bool a16, int sb) {
+  const int SB = a16 ? sb : kStageBlocks;
   return 1024 +
          static_cast<size_t>(stages) *
-             (kStageBlocks * BN * 128 + kA8Stage + kStageBlocks * BN * code_bytes) +
+             (SB * BN * 128 + a_stage_bytes(a16, sb) + SB * BN * code_bytes) +
          static_cast<size_t>(epi_warps) * (epi_out_bufs(epi_warps) * (f32_out ? kEpiBuf32 : kEpiBuf16) +
-                                           2 * epi_scale_cols(epi_warps) * 4) +
+                                           2 * epi_scale_cols(epi_warps, BN) * 4) +
          book_bytes + sizeof(GemmBarriers);
 }
 
-int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes, int epi_warps) {
-  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes, code_bytes, epi_warps);
-  const size_t per = static_cast<size_t>(kStageBlocks) * BN * (128 + code_bytes) + kA8Stage;
+int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes, int epi_warps,
+                    bool a16, int sb) {
+  const size_t fixed = gemm_smem_bytes(BN, 0, f32_out, book_bytes, code_bytes, epi_warps, a16, sb);
+  const int SB = a16 ? sb : kStageBlocks;
+  const size_t per = static_cast<size_t>(SB) * BN * (128 + code_bytes) + a_stage_bytes(a16, sb);
   const int s = static_cast<int>((232448 - fixed) / per);
   return s < kMaxStages ? s : kMaxStages;
 }
@@ -124,6 +136,13 @@ __device__ __forceinline__ TileCoord tile_coord(const GemmParams& p, int t) {
   c.kb_begin = c.split * p.kb_per_split;
   c.kb_end = min(p.num_kb, c.kb_begin + p.kb_per_split);
   return c;
+}
+
+// N of the tile's MMAs: its valid output columns rounded up to 16 (the instruction's
+// granularity for M = 128); columns past them are never stored.
+__device__ __forceinline__ int tile_mma_n(const GemmParams& p, const TileCoord& tc) {
+  const int valid = p.N - tc.n_tile * p.BN;
+  return valid >= p.BN ? p.BN : ((valid + 15) & ~15);
 }
 
 // Ring position: slot index and the parity of the slot's current lap.
@@ -304,6 +323,10 @@ __device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n
   }
 }
 
+// kA16: the shared-memory A form (GemmParams::a16): fp16 A boxes with the 128-byte swizzle
+// beside the weight boxes, tcgen05.mma with both operands from shared memory, no converter
+// warps; warps 2.. are the epilogue and the TMEM holds only the two accumulators (BN <= 256).
+template <bool kA16>
 __global__ void __launch_bounds__(kThreads, 1)
     aq_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                    const __grid_constant__ CUtensorMap mapB,
@@ -314,18 +337,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int S = p.stages;
   const int SA = p.a_stages;
   const int BN = p.BN;
+  const int SB = kA16 ? p.sb : kStageBlocks;  // 64-wide K blocks per stage
+  const int a_half = kA16 ? kA16Half : kA8Half;  // one 64-wide A box
+  const int a_stage = a_stage_bytes(kA16, SB);
   const int b_half = BN * 128;                 // one 64-wide fp16 B box
-  const int b_stage = kStageBlocks * b_half;
+  const int b_stage = SB * b_half;
   const bool raw = p.partial != nullptr;
   const bool f32 = raw || p.out_f32;
   const int epi_buf = f32 ? kEpiBuf32 : kEpiBuf16;
   uint8_t* bring = smem;
   uint8_t* aring = bring + S * b_stage;
-  uint8_t* epi = aring + S * kA8Stage;
+  uint8_t* epi = aring + S * a_stage;
   const int EW = p.epi_warps;                  // 4, or 8 (two per TMEM lane quarter)
+  const int epi_first = kA16 ? 2 : 6;          // first epilogue warp
   float* sscale = reinterpret_cast<float*>(epi + EW * epi_out_bufs(EW) * epi_buf);
   uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) +
-                                          EW * 2 * epi_scale_cols(EW) * 4);
+                                          EW * 2 * epi_scale_cols(EW, BN) * 4);
   // fused path: each stage's packed codes, [h][BN rows][code_bytes] (16-byte aligned)
   const int code_bytes = p.fused ? 8 * p.M * (p.B >> 3) : 0;
   const int code_stage = kStageBlocks * BN * code_bytes;
@@ -342,7 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < S; ++s) {
       // fused path: the producer's expect_tx arrival + one arrival per decoder warp
       mbar_init(&bar->full[s], p.fused ? 1 + kDecodeThreads / 32 : 1);
-      mbar_init(&bar->empty[s], 5);
+      // fp16 A form: the MMA commit alone
+      mbar_init(&bar->empty[s], kA16 ? 1 : 5);
     }
     for (int s = 0; s < SA; ++s) {
       bar->a_ready[s] = 0;
@@ -406,9 +434,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tap = tc.kb_begin / p.cin_blocks;
           cb = tc.kb_begin - tap * p.cin_blocks;
         }
-        for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
-          const int nb = min(kStageBlocks, tc.kb_end - kb);
-          if (!rg.lap0 && !mbar_wait(&bar->empty[rg.s], rg.ph ^ 1u, abort_flag)) {
+        for (int kb = tc.kb_begin; kb < tc.kb_end; kb += SB) {
+          const int nb = min(SB, tc.kb_end - kb);
+          if (!rg.lap0 && !mbar_wait(&bar->empty[rg.s], rg.ph ^ 1u, abort_flag, p.wait_ns)) {
             if (!*abort_flag) record_failure(bar, kDevErrTimeoutEmpty);
             failed = true;
             break;
@@ -427,16 +455,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                             (static_cast<int64_t>(kb + h) * p.N + n0) * code_bytes,
                         bytes, cbar);
           }
-          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (kA8Half + (p.fused ? 0 : b_half))));
-          uint8_t* a_dst = aring + rg.s * kA8Stage;
+          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb * (a_half + (p.fused ? 0 : b_half))));
+          uint8_t* a_dst = aring + rg.s * a_stage;
           uint8_t* b_dst = bring + rg.s * b_stage;
           for (int h = 0; h < nb; ++h) {
             const int k = kb + h;
             if (!p.conv) {
-              tma_load_2d(a_dst + h * kA8Half, &mapA, fb, k * kBK, m0);
+              tma_load_2d(a_dst + h * a_half, &mapA, fb, k * kBK, m0);
             } else {
               const int kh = tap / 3, kw = tap - 3 * (tap / 3);
-              tma_load_4d(a_dst + h * kA8Half, &mapA, fb, cb * kBK, kw - p.pad, ho0 * p.stride + kh - p.pad, b0);
+              tma_load_4d(a_dst + h * a_half, &mapA, fb, cb * kBK, kw - p.pad, ho0 * p.stride + kh - p.pad, b0);
               if (++cb == p.cin_blocks) {
                 cb = 0;
                 ++tap;
@@ -463,10 +491,64 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+  } else if (warp == 1 && kA16) {
+    // ================================================================ MMA issuer (A in smem)
+    // Per stage: wait for its TMA bytes, four 128 x BN x 16 MMAs per 64-wide K block with
+    // both operands read from the swizzled shared-memory boxes, one commit that frees the
+    // stage for the producer.
+    if (lane == 0) {
+      const uint64_t adesc0 = sw128_kmajor_desc(smem_u32(aring));
+      const uint64_t bdesc0 = sw128_kmajor_desc(smem_u32(bring));
+      const uint64_t astep = static_cast<uint64_t>(a_stage >> 4);  // descriptor units: 16 B
+      const uint64_t bstep = static_cast<uint64_t>(b_stage >> 4);
+      const uint64_t ahalf = static_cast<uint64_t>(kA16Half >> 4);
+      const uint64_t bhalf = static_cast<uint64_t>(b_half >> 4);
+      Ring rg;
+      uint32_t lt = 0;
+      bool failed = false;
+      for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
+        const TileCoord tc = tile_coord(p, t);
+        const int nblk = tc.kb_end - tc.kb_begin;
+        // a ragged last N tile runs narrower MMAs (its valid columns, rounded up to 16)
+        const uint32_t idesc = idesc_f16_f32(kBM, tile_mma_n(p, tc));
+        const int buf = static_cast<int>(lt & 1u);
+        if (lt >= 2 && !mbar_wait(&bar->acc_empty[buf], ((lt >> 1) & 1u) ^ 1u, abort_flag, p.wait_ns)) {
+          if (!*abort_flag) record_failure(bar, kDevErrTimeoutAccum);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
+        for (int kb = 0; kb < nblk; kb += SB) {
+          const int nb = min(SB, nblk - kb);
+          if (!mbar_wait(&bar->full[rg.s], rg.ph, abort_flag, p.wait_ns)) {
+            if (!*abort_flag) record_failure(bar, kDevErrTimeoutFull);
+            failed = true;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t a0 = adesc0 + static_cast<uint64_t>(rg.s) * astep;
+          const uint64_t b0 = bdesc0 + static_cast<uint64_t>(rg.s) * bstep;
+          for (int h = 0; h < nb; ++h) {
+            const uint64_t ah = a0 + static_cast<uint64_t>(h) * ahalf;
+            const uint64_t bh = b0 + static_cast<uint64_t>(h) * bhalf;
+            mma_f16_ss(d, ah, bh, idesc, (kb | h) ? 1u : 0u);
+            mma_f16_ss(d, ah + 2u, bh + 2u, idesc, 1u);
+            mma_f16_ss(d, ah + 4u, bh + 4u, idesc, 1u);
+            mma_f16_ss(d, ah + 6u, bh + 6u, idesc, 1u);
+          }
+          mma_commit(&bar->empty[rg.s]);
+          rg.next(S);
+        }
+        if (!failed) mma_commit(&bar->acc_full[buf]);
+      }
+      // every MMA of this CTA completes before teardown frees tensor memory
+      mma_commit(&bar->drain);
+      const int zero = 0;
+      if (!mbar_wait(&bar->drain, 0, &zero)) atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
+    }
   } else if (warp == 1) {
     // ================================================================ MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_f16_f32(kBM, BN);
       const uint64_t bdesc0 = sw128_kmajor_desc(smem_u32(bring));
       const uint64_t bstep = static_cast<uint64_t>(b_stage >> 4);  // descriptor units: 16 B
       const uint64_t bhalf = static_cast<uint64_t>(b_half >> 4);
@@ -476,22 +558,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t lt = 0;
       bool failed = false;
       for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
-        int nblk = p.num_kb;
-        if (p.splits > 1) {
-          const TileCoord tc = tile_coord(p, t);
-          nblk = tc.kb_end - tc.kb_begin;
-        }
+        const TileCoord tc = tile_coord(p, t);
+        const int nblk = tc.kb_end - tc.kb_begin;
+        const uint32_t idesc = idesc_f16_f32(kBM, tile_mma_n(p, tc));
         const int nst = (nblk + 1) >> 1;
         const bool half_tail = (nblk & 1) != 0;
         const int buf = static_cast<int>(lt & 1u);
-        if (lt >= 2 && !mbar_wait(&bar->acc_empty[buf], ((lt >> 1) & 1u) ^ 1u, abort_flag)) {
+        if (lt >= 2 && !mbar_wait(&bar->acc_empty[buf], ((lt >> 1) & 1u) ^ 1u, abort_flag, p.wait_ns)) {
           if (!*abort_flag) record_failure(bar, kDevErrTimeoutAccum);
           break;
         }
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
         for (int st = 0; st < nst; ++st) {
-          if (!ctr_wait(&bar->a_ready[sa], a_target, abort_flag)) {
+          if (!ctr_wait(&bar->a_ready[sa], a_target, abort_flag, p.wait_ns)) {
             if (!*abort_flag) record_failure(bar, kDevErrTimeoutConv);
             failed = true;
             break;
@@ -525,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int zero = 0;
       if (!mbar_wait(&bar->drain, 0, &zero)) atomicOr(&g_gemm_err, kDevErrTimeoutDrain);
     }
-  } else if (warp < 6) {
+  } else if (!kA16 && warp < 6) {
     // ================================================================ converters
     const int q = warp & 3;
     const int row = q * 32 + lane;
@@ -538,8 +618,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const TileCoord tc = tile_coord(p, t);
       for (int kb = tc.kb_begin; kb < tc.kb_end; kb += kStageBlocks) {
         const int nb = min(kStageBlocks, tc.kb_end - kb);
-        bool okw = mbar_wait(&bar->full[rg.s], rg.ph, abort_flag);
-        if (okw && !ra.lap0) okw = mbar_wait(&bar->a_empty[ra.s], ra.ph ^ 1u, abort_flag);
+        bool okw = mbar_wait(&bar->full[rg.s], rg.ph, abort_flag, p.wait_ns);
+        if (okw && !ra.lap0) okw = mbar_wait(&bar->a_empty[ra.s], ra.ph ^ 1u, abort_flag, p.wait_ns);
         if (!okw) {
           if (!*abort_flag) record_failure(bar, kDevErrTimeoutFull);
           failed = true;
@@ -571,14 +651,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ra.next(SA);
       }
     }
-  } else if (warp < 6 + EW) {
+  } else if (warp < epi_first + EW) {
     // ================================================================ epilogue
     const int q = warp & 3;
-    const int ew = warp - 6;
+    const int ew = warp - epi_first;
     // with 8 epilogue warps the two warps of a lane quarter take alternate 32-column chunks
     const int c_first = 32 * (ew >> 2);
     const int c_step = 32 * (EW >> 2);
-    const int wcols = epi_scale_cols(EW);    // this warp's chunks' columns, compacted
+    const int wcols = epi_scale_cols(EW, BN);  // this warp's chunks' columns, compacted
     const int nbuf = epi_out_bufs(EW);
     float* wscale = sscale + ew * 2 * wcols;
     float* wbias = wscale + wcols;
@@ -601,21 +681,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           wbias[i] = (in && p.bias != nullptr) ? __half2float(p.bias[n]) : 0.0f;
         }
       }
-      if (!mbar_wait(&bar->acc_full[buf], (lt >> 1) & 1u, abort_flag)) {
+      if (!mbar_wait(&bar->acc_full[buf], (lt >> 1) & 1u, abort_flag, p.wait_ns)) {
         if (!*abort_flag) record_failure(bar, kDevErrTimeoutAccum);
         break;
       }
       tc_fence_after();
       __syncwarp();
       const uint32_t tacc = t_row + static_cast<uint32_t>(buf * p.acc_stride);
+      // the 32-column chunks that hold valid output columns (a ragged last N tile has fewer)
+      const int ncols = min(BN, tile_mma_n(p, tc));
       int kc = 0;   // chunk index of this warp within the tile
-      for (int c0 = c_first; c0 < BN; c0 += c_step, ++chunk, ++kc) {
+      if (c_first >= ncols) {
+        // no chunk of this tile for this warp: the accumulator buffer is free at once
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar->acc_empty[buf]);
+      }
+      for (int c0 = c_first; c0 < ncols; c0 += c_step, ++chunk, ++kc) {
         const float* csc = wscale + kc * 32;
         const float* cbi = wbias + kc * 32;
         uint32_t r[32];
         tmem_ld_32x32b_x32(tacc + static_cast<uint32_t>(c0), r);
         tmem_wait_ld();
-        if (c0 + c_step >= BN) {
+        if (c0 + c_step >= ncols) {
           // last read of this accumulator buffer: hand it back to the MMA warp
           tc_fence_before();
           __syncwarp();
@@ -729,7 +817,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (lane == 0) bulk_wait_group_all();
-  } else if (p.fused) {
+  } else if (!kA16 && p.fused) {
     // ================================================================ decoders (fused path)
     // Each decoded group (8 consecutive k of one output row) is written as one
     // 16-byte chunk of the 128B-swizzled K-major B stage, so W-hat never leaves
@@ -761,7 +849,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nb = min(kStageBlocks, tc.kb_end - kb);
         // the producer copies a stage's codes only after the stage is free, so their
         // arrival also means the B stage may be overwritten
-        if (!mbar_wait(&bar->codes_full[rg.s], rg.ph, abort_flag)) {
+        if (!mbar_wait(&bar->codes_full[rg.s], rg.ph, abort_flag, p.wait_ns)) {
           if (!*abort_flag) record_failure(bar, kDevErrTimeoutFull);
           failed = true;
           break;
@@ -873,18 +961,30 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
 
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st) {
-  static std::atomic<int> configured[64] = {};
+  static std::atomic<int> configured_i8[64] = {};
+  static std::atomic<int> configured_a16[64] = {};
+  const bool a16 = p.a16 != 0;
+  // the shared-memory A form: dense weights only, 1 or 2 K blocks per stage, and the
+  // TMEM holds just the two accumulators; the TMEM-A form needs two A slots beside them
+  if (a16 && (p.fused || (p.sb != 1 && p.sb != 2) || 2 * p.BN > kTmemCols))
+    return cudaErrorInvalidConfiguration;
+  if (!a16 && (p.BN > 192 || 2 * p.acc_stride + 2 * kASlotCols > kTmemCols))
+    return cudaErrorInvalidConfiguration;
+  if (p.BN % 32 != 0 || p.BN < 32 || p.BN > kMaxBN || p.stages < 1 || p.stages > kMaxStages)
+    return cudaErrorInvalidConfiguration;
   const size_t bytes =
       gemm_smem_bytes(p.BN, p.stages, p.out_f32 || p.partial != nullptr, p.book_bytes,
-                      p.fused ? 8 * p.M * (p.B >> 3) : 0, p.epi_warps);
-  const cudaError_t se = ensure_dynamic_smem(aq_gemm_kernel, bytes, configured);
+                      p.fused ? 8 * p.M * (p.B >> 3) : 0, p.epi_warps, a16, p.sb);
+  auto kernel = a16 ? aq_gemm_kernel<true> : aq_gemm_kernel<false>;
+  const cudaError_t se = ensure_dynamic_smem(kernel, bytes, a16 ? configured_a16 : configured_i8);
   if (se != cudaSuccess) return se;
   // the decoder warps (10..15) exist only on the fused path
   if (p.epi_warps != 4 && !(p.epi_warps == 8 && !p.fused && p.BN >= 64))
     return cudaErrorInvalidConfiguration;
-  const int threads = p.fused ? kThreads : 32 * (6 + p.epi_warps);
+  // fp16 A form: producer, MMA and epilogue warps
+  const int threads = a16 ? 32 * (2 + p.epi_warps) : (p.fused ? kThreads : 32 * (6 + p.epi_warps));
   if (!p.cluster)
-    return launch_pdl(aq_gemm_kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
+    return launch_pdl(kernel, dim3(grid), dim3(threads), bytes, st, mapA, mapB, mapY, p);
   // in-cluster split-K: one CTA per (tile, split), the splits of a tile in one cluster
   if (p.splits < 2 || p.splits > kMaxClusterSplits || grid != p.total_tiles ||
       grid % p.splits != 0)
@@ -903,7 +1003,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, aq_gemm_kernel, mapA, mapB, mapY, p);
+  return cudaLaunchKernelEx(&cfg, kernel, mapA, mapB, mapY, p);
 }
 
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st) {

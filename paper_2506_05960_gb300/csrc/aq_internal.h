@@ -15,7 +15,8 @@ namespace aq {
 constexpr int kBM = 128;        // rows (tokens / output pixels) per tile = TMEM lanes
 constexpr int kBK = 64;         // K per TMA box / swizzle row (128 bytes of fp16)
 constexpr int kStageBlocks = 2; // 64-wide K blocks per pipeline stage (8 MMAs of K = 16)
-constexpr int kMaxBN = 192;     // widest N tile: 2 fp32 accumulators + >= 2 A stages in TMEM
+constexpr int kMaxBN = 256;     // widest N tile: 2 fp32 accumulators in TMEM (the TMEM-A
+                                // form also needs >= 2 A slots beside them: BN <= 192)
 constexpr int kMaxStages = 8;   // pipeline ring depth bound
 constexpr int kMaxClusterSplits = 8;  // K splits summed inside one cluster (portable size)
 
@@ -32,6 +33,11 @@ __host__ __device__ constexpr int fused_book_copies(int M) {
 struct GemmParams {
   int T, N, K;                  // rows, output channels, reduction length
   int BN;                       // N tile (multiple of 32, <= kMaxBN)
+  int a16;                      // 1: A is fp16 in global memory (the 8-bit codes as fp16
+                                // integers), TMA-loaded with the 128-byte swizzle and read by
+                                // the MMA from shared memory; no converter warps.  0: int8 A,
+                                // converted into a TMEM A ring
+  int sb;                       // 64-wide K blocks per pipeline stage (a16: 1 or 2; else 2)
   int num_kb;                   // ceil(K / 64)
   int kb_per_split;             // K blocks per split
   int m_tiles, n_tiles, splits, total_tiles;
@@ -59,6 +65,8 @@ struct GemmParams {
   const void* books;            // codebooks [M][2^B][8] fp16
   int M, B;
   int book_bytes;               // codebooks staged in shared memory (8-bit codes), else 0
+  unsigned long long wait_ns;   // a pipeline wait gives up after this long (the error word
+                                // then records which; drains always wait the full ~2 s)
 };
 
 // Parameters of the lookup-table kernel (linear layer, 8-bit codes, T <= 16).
@@ -130,6 +138,9 @@ cudaError_t ensure_dynamic_smem(Kernel kernel, size_t bytes, std::atomic<int> (&
 
 // Launchers (return the launch status; they never synchronise).
 cudaError_t launch_quant_act(const void* x, int8_t* xq, int64_t numel, float s, cudaStream_t st);
+// The same rule, each 8-bit code stored as the fp16 value of that integer (exact).
+cudaError_t launch_quant_act_f16(const void* x, __half* xh, int64_t numel, float s,
+                                 cudaStream_t st);
 cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, int B,
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
@@ -148,10 +159,11 @@ cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int
                               int B, cudaStream_t st);
 // code_bytes: packed code bytes per row and 64-wide K block staged per stage on
 // the fused path (8 * M * bytes per code), 0 on the dense path.
+// a16, sb: the shared-memory A form and its K blocks per stage (GemmParams).
 size_t gemm_smem_bytes(int BN, int stages, bool f32_out, int book_bytes, int code_bytes,
-                       int epi_warps);
+                       int epi_warps, bool a16 = false, int sb = 2);
 int gemm_max_stages(int BN, bool f32_out, int book_bytes, int code_bytes,
-                    int epi_warps);              // ring depth that fits
+                    int epi_warps, bool a16 = false, int sb = 2);   // ring depth that fits
 int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-column accumulators
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st);

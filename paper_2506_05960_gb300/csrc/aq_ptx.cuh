@@ -64,15 +64,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase with the given parity.  Returns false (and does
-// not wait further) when *abort becomes non-zero or the time limit passes.
+// not wait further) when *abort becomes non-zero or more than limit_ns have passed.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
-                                          const volatile int* abort) {
+                                          const volatile int* abort,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if ((it & 255u) == 0u && globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    // the clock is read every 256 polls, every poll under a short (test) limit
+    if (((it & 255u) == 0u || limit_ns < 1000000ull) && globaltimer_ns() - t0 > limit_ns)
+      return false;
   }
 }
 
@@ -106,13 +109,15 @@ __device__ __forceinline__ uint32_t smem_acquire_load(const uint32_t* ctr) {
 
 // Bounded wait until *ctr >= target (wrap-safe signed difference).
 __device__ __forceinline__ bool ctr_wait(const uint32_t* ctr, uint32_t target,
-                                         const volatile int* abort) {
+                                         const volatile int* abort,
+                                         unsigned long long limit_ns = kWaitLimitNs) {
   if (static_cast<int>(smem_acquire_load(ctr) - target) >= 0) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (static_cast<int>(smem_acquire_load(ctr) - target) >= 0) return true;
     if (*abort) return false;
-    if ((it & 255u) == 0u && globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    if (((it & 255u) == 0u || limit_ns < 1000000ull) && globaltimer_ns() - t0 > limit_ns)
+      return false;
   }
 }
 

@@ -167,12 +167,30 @@ def test_plan_query_and_override(lib):
         forced = aq.aq_linear_plan(128, 960, 960)
         aq.aq_set_plan_override()
         assert forced == aq.aq_linear_plan(128, 960, 960)  # the cost-model plan runs
-        for bad in [(48, 0, -1), (-32, 0, -1), (224 + 32, 0, -1), (0, -1, -1), (0, 0, 2)]:
+        for bad in [(48, 0, -1), (-32, 0, -1), (256 + 32, 0, -1), (0, -1, -1), (0, 0, 2)]:
             with pytest.raises(aq.AQError) as e:
                 aq.aq_set_plan_override(*bad)
             assert e.value.status == -2
         p = aq.aq_conv2d_plan(2, 8, 8, 960, 960, M=2)
         assert p["cluster"] == 1 and aq.aq_conv2d_workspace_size(2, 8, 8, 960, 960, M=2) == 0
+        # fp16 activations on the dense paths: the shared-memory A form, N tiles up to 256;
+        # int8 activations keep the TMEM A form (N tiles up to 192)
+        assert aq.aq_linear_plan(4096, 960, 2880)["a16"] == 0
+        pf = aq.aq_linear_f16_plan(4096, 960, 2880)
+        assert pf["path"] == 1 and pf["a16"] == 1 and pf["stage_blocks"] >= 1
+        assert aq.aq_linear_a16_plan(4096, 960, 2880) == pf
+        assert aq.aq_linear_f16_plan(128, 960, 960)["a16"] == 0      # fused path: int8
+        aq.aq_set_plan_override(256, 1, 0)
+        assert aq.aq_linear_a16_plan(4096, 960, 2880)["BN"] == 256
+        assert aq.aq_linear_plan(4096, 960, 2880)["BN"] <= 192       # falls back to the model
+        aq.aq_set_plan_override()
+        # the quantized activations are kept as fp16 values: 2*T*K bytes of workspace
+        assert (aq.aq_linear_f16_workspace_size(4096, 960, 2880)
+                >= 2 * 4096 * 960 + aq.aq_linear_a16_workspace_size(4096, 960, 2880))
+        for path in (2, 3, 4):
+            with pytest.raises(aq.AQError) as e:
+                aq.aq_linear_a16_plan(64, 256, 256, path=path)
+            assert e.value.status == -3
     finally:
         aq.aq_set_plan_override()
 

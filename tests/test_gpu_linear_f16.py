@@ -1,6 +1,6 @@
 """GPU parity of aq_linear_f16 (the layer from fp16 activations in one call): the same
-bits as aq_quant_act followed by aq_linear on every path and output type, and within
-tolerance of the fp64 oracle on the quantized activations."""
+bits as aq_quant_act followed by aq_linear on every path and output type when both run
+the same plan, and within tolerance of the fp64 oracle on the quantized activations."""
 
 import numpy as np
 import pytest
@@ -39,19 +39,34 @@ def _pair(inp, x16, s_x, path, out_f32):
     ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device="cuda")
     y_chain = torch.full((T, N), float("nan"), dtype=tdt, device="cuda")
     aq.aq_linear(xq, s_x, packed, books, scale, bias, y_chain, dt, T, K, N, 8, M, B, ws, wsb, path)
-    # one call
-    wsb2 = aq.aq_linear_f16_workspace_size(T, K, N, 8, M, B, path)
-    assert wsb2 >= T * K + wsb
-    ws2 = torch.full((wsb2,), 0x55, dtype=torch.uint8, device="cuda")
-    y = torch.full((T, N), float("nan"), dtype=tdt, device="cuda")
-    aq.aq_profile_enable(True)
-    aq.aq_linear_f16(x, s_x, packed, books, scale, bias, y, dt, T, K, N, 8, M, B, ws2, wsb2, path)
-    torch.cuda.synchronize()
-    prof = aq.aq_profile_read()
-    aq.aq_profile_enable(False)
+    # one call, on the chain's plan (on the dense paths aq_linear_f16 feeds the tensor cores
+    # fp16 activations from shared memory and may choose another N tile or K split)
+    pl = aq.aq_linear_plan(T, K, N, 8, M, B, path)
+    if pl["BN"]:
+        aq.aq_set_plan_override(pl["BN"], pl["splits"], pl["cluster"])
+    try:
+        pf = aq.aq_linear_f16_plan(T, K, N, 8, M, B, path)
+        assert (pf["path"], pf["BN"], pf["splits"], pf["cluster"]) == (
+            pl["path"], pl["BN"], pl["splits"], pl["cluster"])
+        wsb2 = aq.aq_linear_f16_workspace_size(T, K, N, 8, M, B, path)
+        assert wsb2 >= 2 * T * K
+        ws2 = torch.full((wsb2,), 0x55, dtype=torch.uint8, device="cuda")
+        y = torch.full((T, N), float("nan"), dtype=tdt, device="cuda")
+        aq.aq_profile_enable(True)
+        aq.aq_linear_f16(x, s_x, packed, books, scale, bias, y, dt, T, K, N, 8, M, B, ws2, wsb2,
+                         path)
+        torch.cuda.synchronize()
+        prof = aq.aq_profile_read()
+        aq.aq_profile_enable(False)
+    finally:
+        aq.aq_set_plan_override()
     assert aq.aq_device_error() == 0
-    xq_ws = ws2[:T * K].view(torch.int8).reshape(T, K)
-    assert torch.equal(xq_ws, xq)                           # the workspace holds the int8 operand
+    if pf["a16"]:   # the workspace holds the codes as fp16 values
+        xq_ws = ws2[:2 * T * K].view(torch.float16).reshape(T, K)
+        assert torch.equal(xq_ws, xq.to(torch.float16))
+    else:           # the workspace holds the int8 codes
+        xq_ws = ws2[:T * K].view(torch.int8).reshape(T, K)
+        assert torch.equal(xq_ws, xq)
     return y.cpu().numpy(), y_chain.cpu().numpy(), xq.cpu().numpy(), prof
 
 

@@ -95,7 +95,7 @@ def test_linear_f16_predecoded():
         wsb = aq.aq_linear_f16_workspace_size(T, K, N, 8, 2, 8, path)
         ws = torch.zeros(wsb, dtype=torch.uint8, device="cuda")
         if path == PRE:
-            off = (T * K + 1023) // 1024 * 1024            # W-hat follows the int8 activations
+            off = (2 * T * K + 1023) // 1024 * 1024        # W-hat follows the activation codes
             aq.aq_decode(packed, books, ws[off:], N, K, 8, 2, 8)
         y = torch.empty((T, N), dtype=torch.float16, device="cuda")
         aq.aq_linear_f16(x, 0.05, packed, books, scale, bias, y, aq.AQ_DTYPE_F16, T, K, N, 8, 2,
