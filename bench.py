@@ -57,11 +57,12 @@ METRIC = "AQ layer dense-equivalent TFLOP/s (2*T*N*K / step time)"
 NSETS = 8
 
 # DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from
-# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (summary under profiles/);
-# reported only while the kernel sources are the ones it was measured on.
+# `ncu --set full` capture of one launch (dram__bytes_read.sum + dram__bytes_write.sum;
+# summary in profiles/aq_gemm_kernel_a16_qkv_T4096_K960_N2880.md); reported only while the
+# kernel sources are the ones it was measured on.
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 9553152, "sources_sha": "10abd9cc89e33978"}
+TRAFFIC = {"bytes": 13475584, "sources_sha": "f05866774bf5cce8"}
 
 
 def sources_sha() -> str:
@@ -567,6 +568,8 @@ KERNEL_WORKLOADS = {
     "quant": "aq_quant_act on the qkv input (4096 x 960 fp16)",
     "decode": "aq_decode of the qkv weight (2880 x 960, 2x8)",
     "linear_f16": "aq_linear_f16 on the qkv layer (quantizer, decode, GEMM)",
+    "gemm_a16": ("aq_linear_a16 on the qkv layer, weights decoded beforehand (the tensor-core "
+                 "GEMM alone, fp16 activation codes)"),
     "fused128": "aq_linear, T=128 K=960 N=2880 2x8 (fused decode, K split in cluster)",
     "few4": "aq_linear, T=4 K=960 N=2880 2x8 (few-token kernel)",
     "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
@@ -595,6 +598,14 @@ def run_kernel_workload(args, aq, torch, dev, stream):
             call = lambda: L.decode_only(stream, wdec)
         elif w == "linear_f16":
             call = lambda: L.step_f16(stream)
+        elif w == "gemm_a16":
+            L.quant(stream)
+            xh = L.xq.to(torch.float16)
+            wsp = torch.empty(aq.aq_linear_a16_workspace_size(L.T, K, N, 8, L.M, L.B,
+                                                              aq.AQ_PATH_PREDECODED),
+                              dtype=torch.uint8, device=dev)
+            L.decode_only(stream, wsp)
+            call = lambda: L.gemm_a16(stream, xh, wsp)
         elif w == "grad":
             G = torch.randn((N, K), dtype=torch.float32, device=dev,
                             generator=torch.Generator(device=dev).manual_seed(0))

@@ -299,15 +299,18 @@ AQ_API int aq_linear_a16(const void* xh, float s_x, const void* codes_packed,
  * is reserved up front, a host allocator that must not be re-entered from a
  * callback, or an engine that forbids allocation once it is serving), so they
  * cannot provide the workspace that aq_linear needs for the decoded weights.
- * aq_linear_noalloc computes exactly what aq_linear computes (same kernels,
- * dense path, no K splitting), but decodes the weights into a fixed scratch
- * array that the library holds in device memory: AQ_NOALLOC_SCRATCH_BYTES
- * (16 MiB) per GPU that loads the library, kept until the process exits.
+ * aq_linear_noalloc gives the same result as aq_linear on the dense path
+ * without K splitting (AQ_PATH_DENSE with aq_set_plan_override(0, 1, 0)), bit for
+ * bit, and within the layer tolerance of aq_linear's other plans.  It decodes the
+ * weights into a fixed scratch array that the library holds in device memory:
+ * AQ_NOALLOC_SCRATCH_BYTES (16 MiB) per GPU that loads the library, kept until
+ * the process exits.
  *   - Limit: N * K * 2 <= AQ_NOALLOC_SCRATCH_BYTES (N * K <= 8,388,608
  *     weights); larger layers return AQ_ERR_WORKSPACE before any CUDA call.
- *   - The first call on each device looks up the array's device address
- *     (with that device current); make that first call before any stream
- *     capture.  Later calls make no CUDA runtime call other than launches.
+ *   - The first call on each device, and the first after that device's context
+ *     was re-created (e.g. by cudaDeviceReset), looks up the array's device
+ *     address with that device current; make such a call before any stream
+ *     capture.  No call allocates or synchronises.
  *   - Every call shares the one array and overwrites what it uses (nothing
  *     in it needs to start at zero).  Calls that can overlap on the GPU (on
  *     different streams without ordering) race on the array and give wrong

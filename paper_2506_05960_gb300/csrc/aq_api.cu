@@ -1322,25 +1322,45 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
 
 }  // namespace
 
-// Device address of g_noalloc_scratch on the current device, looked up once per
-// device (the host-side symbol is only a stand-in, never a device address).
+// Device address of g_noalloc_scratch on the current device (the host-side symbol is only
+// a stand-in, never a device address), looked up once per device and context: a context
+// re-created on that device (cudaDeviceReset) gets the array at a new address.
 namespace {
 constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
 void* g_noalloc_dev_ptr[kMaxDevices] = {};
+CUcontext g_noalloc_ctx[kMaxDevices] = {};
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+CtxGetCurrentFn ctx_get_current_fn() {
+  static CtxGetCurrentFn fn = []() -> CtxGetCurrentFn {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    return reinterpret_cast<CtxGetCurrentFn>(p);
+  }();
+  return fn;
+}
 
 int noalloc_scratch_ptr(void** out) {
   int dev = -1;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_status(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices) return set_error(AQ_ERR_CUDA, "device ordinal %d out of range", dev);
+  CUcontext ctx = nullptr;
+  CtxGetCurrentFn get_ctx = ctx_get_current_fn();
+  if (get_ctx == nullptr || get_ctx(&ctx) != CUDA_SUCCESS) ctx = nullptr;
   std::lock_guard<std::mutex> g(g_noalloc_mu);
-  if (g_noalloc_dev_ptr[dev] == nullptr) {
+  if (g_noalloc_dev_ptr[dev] == nullptr || ctx == nullptr || g_noalloc_ctx[dev] != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress(no-alloc scratch)");
     if (p == nullptr || !aligned16(p)) return set_error(AQ_ERR_CUDA, "no-alloc scratch address invalid");
     g_noalloc_dev_ptr[dev] = p;
+    g_noalloc_ctx[dev] = ctx;
   }
   *out = g_noalloc_dev_ptr[dev];
   return AQ_OK;

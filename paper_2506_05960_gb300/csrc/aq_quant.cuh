@@ -8,10 +8,11 @@
 namespace aq {
 
 // x / s in IEEE fp32, round half to even, NaN -> 0, clip to [-127, 127].
-// Fast path: q = x * fl(1/s) lies within 3 * 2^-24 * |x/s| of fl(x/s); for
-// |x/s| < 128 that is < 2.3e-5, so unless q is within 1e-4 of a half-integer
-// both round to the same integer (and for |x/s| >= 128 both clip to the same
-// end).  Near a tie, and for NaN/inf, the exact IEEE quotient decides.
+// Fast path: q = x * fl(1/s) lies within 4u|q| = 2^-22 |q| of fl(x / s) (u = 2^-24;
+// the derivation is at quant_fast_bits below); for |q| < 128 that is < 3.1e-5, so unless
+// q is within 1e-4 of a half-integer both round to the same integer (and for |q| >= 128
+// both clip to the same end).  Near a tie, and for NaN/inf, the exact IEEE quotient
+// decides.
 __device__ __forceinline__ int8_t quant_one(__half h, float s, float rs) {
   const float x = __half2float(h);
   float q = x * rs;

@@ -7,7 +7,7 @@
 // Mapping.  A row block is 8 consecutive output rows.  In a warp, lane 4*r + q owns row
 // n0 + r and the groups 2q, 2q+1 of every 64-wide K block, i.e. 16 consecutive k.  The
 // packed layout [K/64][N][8][M] keeps the 8 rows' codes of one K block contiguous, so a
-// warp reads one 8 * (8 * M * EB)-byte segment per K block (128 B for two 8-bit codes), a
+// warp reads one 8 * (8 * M)-byte segment per K block (128 B for two 8-bit codes), a
 // lane its 2 * M codes in one load.  The CTA's warps take the K blocks round-robin, four
 // at a time (their code loads issued before the first lookup).  Each lane decodes its two
 // groups -- the fp32 sum of the M codewords in ascending m, one round to fp16; for M <= 2
@@ -20,7 +20,7 @@
 // 8-bit codebooks are staged in shared memory in R copies (copy r of entry e in 16-byte
 // slot e * R + r, lane l reading copy l % R): the 8 lanes of a quarter warp, whose random
 // 16-byte lookups are served together, then always hit 8 different bank groups.  16-bit
-// (2^16-entry) codebooks are read from L2 by a second layout (skinny_gather_kernel, below).
+// (2^16-entry) codebooks are read from L2 by a second kernel (skinny_gather_kernel, below).
 #include <cstdint>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -46,50 +46,32 @@ __device__ __forceinline__ void i8x16_to_f32(uint4 v, float (&x)[16]) {
   }
 }
 
-// The 2 * M codes of one lane (groups 2q and 2q+1 of a K block, each [M] codes of EB
-// bytes), widened to 32 bits: c[i * M + m] = code of codebook m in group 2q + i.
-template <int EB, int MM>
+// The 2 * M 8-bit codes of one lane (groups 2q and 2q+1 of a K block, each [M] codes),
+// widened to 32 bits: c[i * M + m] = code of codebook m in group 2q + i.
+template <int MM>
 __device__ __forceinline__ void load_codes(const uint8_t* rec, int q, int M, uint32_t* c) {
-  if constexpr (EB == 1 && MM == 1) {
+  if constexpr (MM == 1) {
     const uint32_t v = *reinterpret_cast<const uint16_t*>(rec + 2 * q);
     c[0] = v & 0xffu;
     c[1] = v >> 8;
-  } else if constexpr (EB == 1 && MM == 2) {
+  } else if constexpr (MM == 2) {
     const uint32_t v = *reinterpret_cast<const uint32_t*>(rec + 4 * q);
     c[0] = v & 0xffu;
     c[1] = (v >> 8) & 0xffu;
     c[2] = (v >> 16) & 0xffu;
     c[3] = v >> 24;
-  } else if constexpr (EB == 2 && MM == 1) {
-    const uint32_t v = *reinterpret_cast<const uint32_t*>(rec + 4 * q);
-    c[0] = v & 0xffffu;
-    c[1] = v >> 16;
-  } else if constexpr (EB == 2 && MM == 2) {
-    const uint2 v = *reinterpret_cast<const uint2*>(rec + 8 * q);
-    c[0] = v.x & 0xffffu;
-    c[1] = v.x >> 16;
-    c[2] = v.y & 0xffffu;
-    c[3] = v.y >> 16;
   } else {
     // any M (3..8): one load per code
-    for (int i = 0; i < 2 * M; ++i) {
-      const int off = (2 * q * M + i) * EB;
-      c[i] = EB == 1 ? static_cast<uint32_t>(rec[off])
-                     : static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(rec + off));
-    }
+    for (int i = 0; i < 2 * M; ++i) c[i] = static_cast<uint32_t>(rec[2 * q * M + i]);
   }
 }
 
-// Decoded weights of one group (8 values, the rule of Eq. 4), as fp32.
-template <int EB, int MM>
-__device__ __forceinline__ void decode_group(const uint32_t* c, int M, const uint4* sbook,
-                                             const uint4* gbook, int R, int copy, float (&w)[8]) {
-  auto word = [&](int m) -> uint4 {
-    if constexpr (EB == 1)
-      return sbook[(m * 256 + static_cast<int>(c[m])) * R + copy];
-    else
-      return __ldg(gbook + (static_cast<int64_t>(m) << 16) + c[m]);
-  };
+// Decoded weights of one group (8 values, the rule of Eq. 4), as fp32, from the shared-
+// memory copies of the 8-bit codebooks.
+template <int MM>
+__device__ __forceinline__ void decode_group(const uint32_t* c, int M, const uint4* sbook, int R,
+                                             int copy, float (&w)[8]) {
+  auto word = [&](int m) -> uint4 { return sbook[(m * 256 + static_cast<int>(c[m])) * R + copy]; };
   if constexpr (MM == 1 || MM == 2) {
     uint4 v = word(0);
     if constexpr (MM == 2) {
@@ -123,31 +105,30 @@ __device__ __forceinline__ void decode_group(const uint32_t* c, int M, const uin
   }
 }
 
-template <int EB, int TT, int MM>
+// 8-bit codes.  TT: tokens rounded up to 1, 2, 4, 8 or 16; MM: M when 1 or 2, else 0.
+template <int TT, int MM>
 __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyParams p) {
   extern __shared__ float4 skinny_smem4[];
   const int M = MM > 0 ? MM : p.M;
-  const int R = EB == 1 ? fused_book_copies(M) : 1;
+  const int R = fused_book_copies(M);
   uint4* sbook = reinterpret_cast<uint4*>(skinny_smem4);                   // [M*256][R]
-  float* wred = reinterpret_cast<float*>(skinny_smem4) + (EB == 1 ? M * 256 * R * 4 : 0);
+  float* wred = reinterpret_cast<float*>(skinny_smem4) + M * 256 * R * 4;
   grid_dependency_wait();
   allow_dependents();
   const uint4* gbook = static_cast<const uint4*>(p.books);
-  if constexpr (EB == 1) {
-    // thread i writes copy (r + i) % R at step r: a quarter warp's stores hit distinct banks
-    for (int i = threadIdx.x; i < M * 256; i += blockDim.x) {
-      const uint4 v = gbook[i];
-      for (int r = 0; r < R; ++r) sbook[i * R + ((r + i) & (R - 1))] = v;
-    }
-    __syncthreads();
+  // thread i writes copy (r + i) % R at step r: a quarter warp's stores hit distinct banks
+  for (int i = threadIdx.x; i < M * 256; i += blockDim.x) {
+    const uint4 v = gbook[i];
+    for (int r = 0; r < R; ++r) sbook[i * R + ((r + i) & (R - 1))] = v;
   }
+  __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, q = lane & 3;
   const int copy = lane & (R - 1);
   const int T = p.T, K = p.K, N = p.N;
   const int KB = (K + 63) >> 6;                  // K blocks (the last may be partial)
   const int G = K >> 3;                          // groups; K % 16 == 0, so G is even
-  const int CB = 8 * M * EB;                     // code bytes of one row in one K block
+  const int CB = 8 * M;                          // code bytes of one row in one K block
   const int n_rb = (N + kSkinnyRows - 1) / kSkinnyRows;
   const uint8_t* codes = static_cast<const uint8_t*>(p.codes);
   const float rs_out = p.out_q8 ? __frcp_rn(p.s_out) : 0.0f;
@@ -168,7 +149,7 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
           // this lane's two groups exist (G even: both or neither)
           ok[u] = kb < KB && kb * 8 + 2 * q < G;
           if (ok[u])
-            load_codes<EB, MM>(codes + (static_cast<int64_t>(kb) * N + n) * CB, q, M, c[u]);
+            load_codes<MM>(codes + (static_cast<int64_t>(kb) * N + n) * CB, q, M, c[u]);
         }
 #pragma unroll
         for (int u = 0; u < kSkinnyUnroll; ++u) {
@@ -177,8 +158,8 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
           float w[16];
           float (&w0)[8] = *reinterpret_cast<float (*)[8]>(w);
           float (&w1)[8] = *reinterpret_cast<float (*)[8]>(w + 8);
-          decode_group<EB, MM>(c[u], M, sbook, gbook, R, copy, w0);
-          decode_group<EB, MM>(c[u] + M, M, sbook, gbook, R, copy, w1);
+          decode_group<MM>(c[u], M, sbook, R, copy, w0);
+          decode_group<MM>(c[u] + M, M, sbook, R, copy, w1);
           const int k0 = kb * 64 + q * 16;
 #pragma unroll
           for (int t = 0; t < TT; ++t) {
@@ -221,12 +202,11 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
   }
 }
 
-// 16-bit codes (2^16-entry codebooks, codewords gathered from L2): the layout of four
-// output rows per CTA, whose threads stride the K/8 group columns and decode each group for
-// the four rows, keeps more independent gathers in flight per thread (measured on GB300:
-// 13.9 / 16.5 us at T = 2 / 4 on a K = 8640, N = 960 layer, against 19.5 / 26.7 for the
-// row-block layout above; that layout's 16-bit branch measured 10.05 us against 12.8 at T = 1
-// but is not dispatched until a parity test covers it).
+// 16-bit codes (2^16-entry codebooks, codewords gathered from L2): four output rows per
+// CTA, whose threads stride the K/8 group columns and decode each group for the four rows,
+// so every thread keeps several independent gathers in flight (measured on GB300: 13.9 /
+// 16.5 us at T = 2 / 4 on a K = 8640, N = 960 layer, against 19.5 / 26.7 for a row-block
+// layout like the one above).
 constexpr int kGatherRows = 4;
 
 // 8 int8 -> 8 floats
@@ -239,18 +219,13 @@ __device__ __forceinline__ void i8x8_to_f32(uint2 v, float (&x)[8]) {
   }
 }
 
-template <int EB, int TT>
+template <int TT>
 __global__ void __launch_bounds__(256, 2) skinny_gather_kernel(const SkinnyParams p) {
   extern __shared__ float4 gather_smem4[];
-  uint4* sbook = reinterpret_cast<uint4*>(gather_smem4);                 // [M][256] (8-bit)
-  float* wred = reinterpret_cast<float*>(gather_smem4) + (EB == 1 ? p.M * 256 * 4 : 0);
+  float* wred = reinterpret_cast<float*>(gather_smem4);
   grid_dependency_wait();
   allow_dependents();
   const uint4* books = static_cast<const uint4*>(p.books);
-  if constexpr (EB == 1) {
-    for (int i = threadIdx.x; i < p.M * 256; i += blockDim.x) sbook[i] = books[i];
-    __syncthreads();
-  }
   // CTA = four output rows; thread = a stride of group columns (8 weights of K each)
   const int n0 = blockIdx.x * kGatherRows;
   const int G = p.K >> 3;
@@ -275,13 +250,8 @@ __global__ void __launch_bounds__(256, 2) skinny_gather_kernel(const SkinnyParam
       if (n < p.N) {
         const int64_t cidx = ((static_cast<int64_t>(kb) * p.N + n) * 8 + j) * M;
         for (int m = 0; m < M; ++m) {
-          uint4 cw;
-          if constexpr (EB == 1) {
-            cw = sbook[m * 256 + __ldg(static_cast<const uint8_t*>(p.codes) + cidx + m)];
-          } else {
-            const int c = __ldg(static_cast<const uint16_t*>(p.codes) + cidx + m);
-            cw = __ldg(books + (static_cast<int64_t>(m) << 16) + c);
-          }
+          const int c = __ldg(static_cast<const uint16_t*>(p.codes) + cidx + m);
+          const uint4 cw = __ldg(books + (static_cast<int64_t>(m) << 16) + c);
           const __half2* h2 = reinterpret_cast<const __half2*>(&cw);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
@@ -341,12 +311,13 @@ __global__ void __launch_bounds__(256, 2) skinny_gather_kernel(const SkinnyParam
 
 static int skinny_tt(int T) { return T <= 1 ? 1 : T <= 2 ? 2 : T <= 4 ? 4 : T <= 8 ? 8 : 16; }
 
-size_t skinny_smem_bytes(int M, int B, int T) {
-  return (B == 8 ? static_cast<size_t>(M) * 256 * 16 * fused_book_copies(M) : 0) +
+// 8-bit codes (the row-block kernel): codebook copies + the warps' partial sums
+size_t skinny_smem_bytes(int M, int T) {
+  return static_cast<size_t>(M) * 256 * 16 * fused_book_copies(M) +
          static_cast<size_t>(kSkinnyWarps) * kSkinnyRows * skinny_tt(T) * 4;
 }
 
-template <int EB, int MM>
+template <int MM>
 cudaError_t launch_skinny_m(const SkinnyParams& p, size_t smem, cudaStream_t st) {
   // persistent CTAs: as many row blocks as fit at once (shared memory and threads bound
   // the CTAs per SM), at most one per row block
@@ -366,11 +337,11 @@ cudaError_t launch_skinny_m(const SkinnyParams& p, size_t smem, cudaStream_t st)
     return launch_pdl(kernel, grid, block, smem, st, p);
   };
   switch (skinny_tt(p.T)) {
-    case 1: return go(skinny_kernel<EB, 1, MM>);
-    case 2: return go(skinny_kernel<EB, 2, MM>);
-    case 4: return go(skinny_kernel<EB, 4, MM>);
-    case 8: return go(skinny_kernel<EB, 8, MM>);
-    default: return go(skinny_kernel<EB, 16, MM>);
+    case 1: return go(skinny_kernel<1, MM>);
+    case 2: return go(skinny_kernel<2, MM>);
+    case 4: return go(skinny_kernel<4, MM>);
+    case 8: return go(skinny_kernel<8, MM>);
+    default: return go(skinny_kernel<16, MM>);
   }
 }
 
@@ -382,20 +353,20 @@ cudaError_t launch_skinny_gather(const SkinnyParams& p, cudaStream_t st) {
   const size_t smem = static_cast<size_t>(threads / 32) * kGatherRows * skinny_tt(p.T) * 4;
   const dim3 grid(static_cast<unsigned>(blocks)), block(static_cast<unsigned>(threads));
   switch (skinny_tt(p.T)) {
-    case 1: return launch_pdl(skinny_gather_kernel<2, 1>, grid, block, smem, st, p);
-    case 2: return launch_pdl(skinny_gather_kernel<2, 2>, grid, block, smem, st, p);
-    case 4: return launch_pdl(skinny_gather_kernel<2, 4>, grid, block, smem, st, p);
-    case 8: return launch_pdl(skinny_gather_kernel<2, 8>, grid, block, smem, st, p);
-    default: return launch_pdl(skinny_gather_kernel<2, 16>, grid, block, smem, st, p);
+    case 1: return launch_pdl(skinny_gather_kernel<1>, grid, block, smem, st, p);
+    case 2: return launch_pdl(skinny_gather_kernel<2>, grid, block, smem, st, p);
+    case 4: return launch_pdl(skinny_gather_kernel<4>, grid, block, smem, st, p);
+    case 8: return launch_pdl(skinny_gather_kernel<8>, grid, block, smem, st, p);
+    default: return launch_pdl(skinny_gather_kernel<16>, grid, block, smem, st, p);
   }
 }
 
 cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st) {
   if (p.B == 16) return launch_skinny_gather(p, st);
-  const size_t smem = skinny_smem_bytes(p.M, p.B, p.T);
-  if (p.M == 1) return launch_skinny_m<1, 1>(p, smem, st);
-  if (p.M == 2) return launch_skinny_m<1, 2>(p, smem, st);
-  return launch_skinny_m<1, 0>(p, smem, st);
+  const size_t smem = skinny_smem_bytes(p.M, p.T);
+  if (p.M == 1) return launch_skinny_m<1>(p, smem, st);
+  if (p.M == 2) return launch_skinny_m<2>(p, smem, st);
+  return launch_skinny_m<0>(p, smem, st);
 }
 
 }  // namespace aq

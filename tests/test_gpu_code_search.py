@@ -1,6 +1,8 @@
 """GPU parity of the greedy code-search step (Stage-1 calibration, Sec. 3.1):
 bit-exact codes against the reference step (same fp32 decision rule), with and
-without the calibration-input weighting, on one codebook and on a sweep over all."""
+without the calibration-input weighting, on one codebook and on a sweep over all;
+and, independently of that rule's operation order, every chosen code is a float64
+minimiser of its group's error up to float32 near-ties."""
 
 import numpy as np
 import pytest
@@ -47,6 +49,31 @@ def test_code_update_bit_exact(N, Gr, M, weighted, m_first, m_count):
     got = _step(W, books, codes, H, m_first, m_count)
     ref = O.code_update_f32(W, books, codes, H, ms=range(m_first, m_first + m_count))
     assert np.array_equal(got, ref)
+    _assert_near_minimisers(W, books, codes, got, H, m_first, m_count)
+
+
+def _assert_near_minimisers(W, books, old, new, H, m_first, m_count):
+    """Independent of the reference step's operation order: each code the GPU chose for
+    codebook m is, in float64, a minimiser of its group's error over all 256 codewords --
+    with the codebooks updated before m at their new codes and those after m at their old
+    ones -- up to float32 near-ties."""
+    N, Gr, M = old.shape
+    C = books.astype(np.float64)                                    # [M][256][8]
+    Wg = W.astype(np.float64).reshape(N, Gr, 8)
+    for m in range(m_first, m_first + m_count):
+        ctx = np.where(np.arange(M)[None, None, :] < m, new, old)      # codes seen by step m
+        r = Wg.copy()
+        for mm in range(M):
+            if mm != m:
+                r -= C[mm][ctx[:, :, mm]]
+        d = C[m][None, None, :, :] - r[:, :, None, :]                 # [N][Gr][256][8]
+        if H is None:
+            score = np.einsum("nice,nice->nic", d, d)
+        else:
+            score = np.einsum("nice,ief,nicf->nic", d, H.astype(np.float64), d)
+        best = score.min(axis=2)
+        chosen = np.take_along_axis(score, new[:, :, m].astype(np.int64)[:, :, None], 2)[:, :, 0]
+        assert np.all(chosen <= best + 1e-5 * (1.0 + best)), (m, float(np.max(chosen - best)))
 
 
 def test_code_update_reduces_error_over_sweeps():

@@ -44,6 +44,21 @@ def test_few_tokens_formats(T, K, N, M, B):
     assert_close(y32, O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], None))
 
 
+@pytest.mark.parametrize("T,K,N,M", [(1, 8640, 960, 1), (1, 1024, 24, 2), (2, 8640, 960, 1),
+                                     (4, 1024, 24, 2)])
+def test_few_tokens_16bit_codes_at_auto_token_counts(T, K, N, M):
+    """2^16-entry codebooks at the token counts AUTO sends down the few-token path
+    (T <= 4): fp16 and fp32 outputs against the oracle, and AUTO gives the same bits."""
+    inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=16, cb_std=0.05 / M ** 0.5),
+                      seed=T * 7 + K + N)
+    y = run_linear(inp, path=FEW)
+    assert_close(y, O.layer_f64(inp), (T, K, N, M))
+    assert np.array_equal(run_linear(inp, path=AUTO), y)
+    y32 = run_linear(inp, path=FEW, out_f32=True)
+    assert_close(y32, O.layer_f64(inp), (T, K, N, M, "f32"))
+    assert np.array_equal(run_linear(inp, path=AUTO, out_f32=True), y32)
+
+
 def test_few_tokens_q8_equals_chain():
     import torch
     import paper_2506_05960_gb300 as aq

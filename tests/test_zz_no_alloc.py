@@ -43,11 +43,19 @@ def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
                     scale=dev(inp["scale"]), bias=dev(inp["bias"]), s_x=inp["s_x"])
 
     def with_workspace(L):
-        ws_bytes = aq.aq_linear_workspace_size(L["T"], L["K"], L["N"], 8, L["M"], L["B"])
-        ws = torch.empty(max(ws_bytes, 16), dtype=torch.uint8, device="cuda")
-        y = torch.full((L["T"], L["N"]), float("nan"), dtype=torch.float16, device="cuda")
-        aq.aq_linear(L["xq"], L["s_x"], L["packed"], L["books"], L["scale"], L["bias"], y,
-                     aq.AQ_DTYPE_F16, L["T"], L["K"], L["N"], 8, L["M"], L["B"], ws, ws_bytes)
+        # aq_linear on the same path as the no-alloc call: decoded weights, no K split (any N
+        # tile: each output's products are accumulated in the same K order)
+        aq.aq_set_plan_override(0, 1, 0)
+        try:
+            ws_bytes = aq.aq_linear_workspace_size(L["T"], L["K"], L["N"], 8, L["M"], L["B"],
+                                                   aq.AQ_PATH_DENSE)
+            ws = torch.empty(max(ws_bytes, 16), dtype=torch.uint8, device="cuda")
+            y = torch.full((L["T"], L["N"]), float("nan"), dtype=torch.float16, device="cuda")
+            aq.aq_linear(L["xq"], L["s_x"], L["packed"], L["books"], L["scale"], L["bias"], y,
+                         aq.AQ_DTYPE_F16, L["T"], L["K"], L["N"], 8, L["M"], L["B"], ws, ws_bytes,
+                         aq.AQ_PATH_DENSE)
+        finally:
+            aq.aq_set_plan_override()
         return y
 
     def no_alloc(L):
@@ -65,9 +73,9 @@ def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
     torch.cuda.synchronize()
     assert aq.aq_device_error() == 0
     for inp, L, y in zip(inps, layers, got):
-        ref = with_workspace(L).float().cpu().numpy().astype(np.float64)
+        ref = with_workspace(L)
+        torch.cuda.synchronize()
+        assert torch.equal(y.view(torch.int16), ref.view(torch.int16))   # bit for bit
         yn = y.float().cpu().numpy().astype(np.float64)
-        m = O.compare(yn, ref)
-        assert m["rel_fro"] <= TOL_REL_FRO and m["max_abs"] <= TOL_MAX_ABS * m["scale_ref"], m
         m64 = O.compare(yn, O.layer_f64(inp))
         assert m64["rel_fro"] <= TOL_REL_FRO and m64["max_abs"] <= TOL_MAX_ABS * m64["scale_ref"], m64
