@@ -59,10 +59,11 @@ NSETS = 8
 # DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from
 # `ncu --set full` capture of one launch (dram__bytes_read.sum + dram__bytes_write.sum;
 # summary in profiles/aq_gemm_kernel_a16_qkv_T4096_K960_N2880.md); reported only while the
-# kernel sources are the ones it was measured on.
+# kernel sources are the ones it was measured on (the key was refreshed after a header-only
+# change that left the GEMM's compiled code byte-identical).
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 13475584, "sources_sha": "f05866774bf5cce8"}
+TRAFFIC = {"bytes": 13475584, "sources_sha": "7b013bcd52b7d27c"}
 
 
 def sources_sha() -> str:
@@ -970,6 +971,29 @@ def main():
             "bytes_per_call": cg_bytes,
             "step": "aq_codebook_grad, 8 rotating G buffers (> L2), CUDA graph replay"}
         del gc, gsets
+        # input gradient of the qkv layer (dL/dX = dY diag(scale) W-hat: transposed decode +
+        # the fp16-activation GEMM over N), 8 rotating dY buffers
+        dys = [torch.randn((T, N), device=dev, generator=torch.Generator(device=dev).manual_seed(
+            20 + i)).to(torch.float16) for i in range(NSETS)]
+        dxs = [torch.empty((T, K), dtype=torch.float16, device=dev) for _ in range(NSETS)]
+        igb = aq.aq_linear_input_grad_workspace_size(T, K, N, g, M, B)
+        igws = [torch.empty(igb, dtype=torch.uint8, device=dev) for _ in range(NSETS)]
+
+        def igrad():
+            for dy_, dx_, w_ in zip(dys, dxs, igws):
+                aq.aq_linear_input_grad(dy_, 1.0, gb.packed, gb.books, gb.scale, dx_,
+                                        aq.AQ_DTYPE_F16, T, K, N, g, M, B, w_, igb, stream=stream)
+        with torch.cuda.stream(stream):
+            igrad()
+        stream.synchronize()
+        gi = capture(torch, stream, igrad)
+        ms = replay_ms(torch, stream, gi, 20) / NSETS
+        layers["input gradient of the qkv layer (dL/dX, fp16 dY, 2x8)"] = {
+            "us_per_step": ms * 1e3, "tflops": fl / (ms * 1e-3) / 1e12,
+            "tensor_roofline_frac": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"],
+            "step": ("aq_linear_input_grad (transposed scaled decode + tensor-core GEMM over N), "
+                     "8 rotating dY buffers, CUDA graph replay")}
+        del gi, dys, dxs, igws
         # Stage-1 code search (one greedy step over both codebooks) on the qkv layer
         from aq_synth import make_linear as _ml
         inp1 = _ml(WORKLOADS["qkv"], seed=SEEDS["qkv"])

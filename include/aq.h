@@ -178,6 +178,25 @@ AQ_API int aq_codebook_grad(const void* codes_packed, const float* G, const void
                             float s_x, float* dC, int N, int K, int g, int M, int B,
                             void* stream);
 
+/* ---- input gradient (backward of the layer; Sec. 3.2.1 continuous step) ----
+ * dX[t][k] = alpha * sum_n dY[t][n] * scale[n] * W[n][k], W the decoded AQ weight.
+ * With alpha = 1 this is the gradient with respect to the dequantized activations
+ * X = s_x * xq of the layer y = diag(scale) W X + bias; alpha = s_x gives it with
+ * respect to the 8-bit codes xq (the straight-through quantizer).  Computed as the
+ * same decode + tensor-core contraction as the forward layer: a transposed decode
+ * writes Wt[k][n] = fp16(scale[n] * W[n][k]) (W by the decode rule above, the product
+ * rounded once more to fp16) into the workspace, then the fp16-activation GEMM
+ * contracts dY with it over n, accumulating in fp32.
+ *   dY fp16 [T][N]; codes, codebooks, scale as for aq_linear; dX [T][K] fp16 or fp32.
+ *   K % 16 == 0, N % 16 == 0 (AQ_ERR_SHAPE); T == 0 is a no-op; alpha finite.
+ *   Workspace: aq_linear_input_grad_workspace_size() bytes.                       */
+AQ_API int aq_linear_input_grad_workspace_size(int T, int K, int N, int g, int M, int B,
+                                               size_t* bytes);
+AQ_API int aq_linear_input_grad(const void* dy, float alpha, const void* codes_packed,
+                                const void* codebooks, const void* scale, void* dx,
+                                int out_dtype, int T, int K, int N, int g, int M, int B,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
 /* ---- code search step (Stage-1 calibration, Sec. 3.1) ---------------------
  * One greedy step of the code optimisation (beam width 1): for every group and
  * each codebook m in [m_first, m_first + m_count), in that order, b[m] becomes

@@ -31,7 +31,7 @@ import numpy as np
 
 __all__ = [
     "decode_f64", "decode_rule_f16", "decode_kaq_f64", "kaq_ohwi", "kaq_from_ohwi",
-    "codebook_grad_f64", "code_update_f32", "pack_codes", "packed_nbytes",
+    "codebook_grad_f64", "input_grad_f64", "code_update_f32", "pack_codes", "packed_nbytes",
     "quant_act", "linear_f64", "conv2d_nhwc_f64", "lut_linear_f64",
     "lut_conv_kaq_counted", "direct_conv_counted", "eq_a7_flops", "eq_a2_flops",
     "paper_lut_breakeven", "eq_a7_breakeven", "bits_per_weight",
@@ -131,6 +131,23 @@ def codebook_grad_f64(codes: np.ndarray, G: np.ndarray, scale: np.ndarray | None
     for m in range(M):
         np.add.at(dC[m], codes[:, :, m].reshape(-1).astype(np.int64), Gs)
     return dC
+
+
+def input_grad_f64(dy: np.ndarray, codes: np.ndarray, codebooks: np.ndarray,
+                   scale: np.ndarray, alpha: float = 1.0) -> np.ndarray:
+    """Backward of the layer with respect to its input (the gradient the continuous step of
+    Sec. 3.2.1 passes to the layers before this one), float64.
+
+    The layer of Sec. 3.1.1, Y = W X, with the decoded AQ weight of Eq. 4 and the
+    per-output-channel scale: y[t, n] = scale[n] * sum_k X[t, k] * W[n, k] + bias[n],
+    X = s_x * xq.  Its input gradient is
+      dX[t, k] = sum_n dY[t, n] * scale[n] * W[n, k],
+    returned times ``alpha`` (alpha = s_x: the gradient with respect to the codes xq).
+    dy [T][N], codes [N][Gr][M], codebooks [M][2**B][g], scale [N] -> [T][Gr*g].
+    """
+    W = decode_f64(codes, codebooks)
+    G = dy.astype(np.float64) * scale.astype(np.float64)[None, :]
+    return float(alpha) * (G @ W)
 
 
 def code_update_f32(W: np.ndarray, codebooks: np.ndarray, codes: np.ndarray,

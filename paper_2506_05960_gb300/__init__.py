@@ -15,7 +15,7 @@ from ._binding import (  # noqa: F401
     aq_linear_f16_plan, aq_linear_a16, aq_linear_a16_plan, aq_linear_a16_workspace_size,
     aq_linear_noalloc, aq_linear_q8,
     aq_linear_plan, aq_linear_workspace_size, aq_pack, aq_set_plan_override,
-    aq_set_wait_limit_ns, AQ_DEVERR_TIMEOUT_FULL,
+    aq_set_wait_limit_ns, aq_linear_input_grad, aq_linear_input_grad_workspace_size, AQ_DEVERR_TIMEOUT_FULL,
     AQ_DEVERR_TIMEOUT_EMPTY, AQ_DEVERR_TIMEOUT_CONV, AQ_DEVERR_TIMEOUT_ACCUM, AQ_DEVERR_TIMEOUT_DRAIN,
     aq_packed_size, aq_profile_enable, aq_profile_read, aq_quant_act, library_path,
     load_library, PROFILE_KINDS,

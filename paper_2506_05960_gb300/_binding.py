@@ -41,6 +41,9 @@ _SIGNATURES = {
     "aq_codebook_grad": (_c_int, [_c_void_p] * 3 + [_c_float, _c_void_p] + [_c_int] * 5
                          + [_c_void_p]),
     "aq_code_update": (_c_int, [_c_void_p] * 4 + [_c_int] * 7 + [_c_void_p]),
+    "aq_linear_input_grad_workspace_size": (_c_int, [_c_int] * 6 + [ctypes.POINTER(_c_size_t)]),
+    "aq_linear_input_grad": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 4 + [_c_int] * 7
+                             + [_c_void_p, _c_size_t, _c_void_p]),
     "aq_linear_workspace_size": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_size_t)]),
     "aq_linear_plan": (_c_int, [_c_int] * 7 + [ctypes.POINTER(_c_int), _c_int]),
     "aq_set_plan_override": (_c_int, [_c_int] * 3),
@@ -182,6 +185,22 @@ def aq_codebook_grad(codes_packed, G, scale, s_x, dC, N, K, g=8, M=2, B=8, strea
     _check(load_library().aq_codebook_grad(
         _ptr(codes_packed), _ptr(G), _ptr(scale), float(s_x), _ptr(dC), N, K, g, M, B,
         _stream(stream)), "aq_codebook_grad")
+
+
+def aq_linear_input_grad_workspace_size(T, K, N, g=8, M=2, B=8) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_linear_input_grad_workspace_size(T, K, N, g, M, B, ctypes.byref(out)),
+           "aq_linear_input_grad_workspace_size")
+    return out.value
+
+
+def aq_linear_input_grad(dy, alpha, codes_packed, codebooks, scale, dx, out_dtype, T, K, N, g=8,
+                         M=2, B=8, workspace=None, workspace_bytes=0, stream=None) -> None:
+    """dX = alpha * dY diag(scale) W-hat (the layer's input gradient)."""
+    _check(load_library().aq_linear_input_grad(
+        _ptr(dy), float(alpha), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(dx),
+        out_dtype, T, K, N, g, M, B, _ptr(workspace), int(workspace_bytes), _stream(stream)),
+        "aq_linear_input_grad")
 
 
 def aq_code_update(W, codebooks, codes, H, m_first, m_count, N, K, g=8, M=2, B=8,

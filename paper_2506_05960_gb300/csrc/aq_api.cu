@@ -1322,6 +1322,96 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
 
 }  // namespace
 
+// ---- input gradient (dL/dX through the AQ layer)
+namespace {
+// Workspace: [Wt fp16 K x N (+ the GEMM's split-K partials): the fp16-activation GEMM's
+// predecoded workspace for the (T, K_red = N, N_out = K) contraction][ones fp16 K].
+struct GradRoute {
+  Route rt;
+  size_t ones_off, bytes;
+};
+
+GradRoute route_input_grad(int T, int K, int N, bool f32_out, int M, int B) {
+  GradRoute gr;
+  gr.rt = route_gemm(AQ_PATH_PREDECODED, T, K, N, (T + aq::kBM - 1) / aq::kBM, f32_out, M, B, true);
+  gr.ones_off = align_up(gr.rt.ws, 1024);
+  gr.bytes = gr.ones_off + align_up(static_cast<size_t>(K) * 2, 1024);
+  return gr;
+}
+
+int check_grad_shapes(int T, int K, int N, int g, int M, int B) {
+  int r = check_format(g, M, B);
+  if (r) return r;
+  if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
+  if (K % 16 != 0 || N % 16 != 0)
+    return set_error(AQ_ERR_SHAPE, "input gradient needs K %% 16 == 0 and N %% 16 == 0");
+  return AQ_OK;
+}
+}  // namespace
+
+extern "C" int aq_linear_input_grad_workspace_size(int T, int K, int N, int g, int M, int B,
+                                                   size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  const int r = check_grad_shapes(T, K, N, g, M, B);
+  if (r) return r;
+  // the same plan (and workspace) for fp16 and fp32 output
+  *bytes = route_input_grad(T, K, N, false, M, B).bytes;
+  return ok();
+}
+
+extern "C" int aq_linear_input_grad(const void* dy, float alpha, const void* codes_packed,
+                                    const void* codebooks, const void* scale, void* dx,
+                                    int out_dtype, int T, int K, int N, int g, int M, int B,
+                                    void* workspace, size_t workspace_bytes, void* stream) {
+  int r = check_grad_shapes(T, K, N, g, M, B);
+  if (r) return r;
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d", out_dtype);
+  if (!(alpha == alpha) || alpha == __builtin_inff() || alpha == -__builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "alpha must be finite");
+  if (T == 0) return ok();
+  if (!dy || !codes_packed || !codebooks || !scale || !dx) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(dy) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+      !aligned16(dx))
+    return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  // the plan for this output type: the workspace query's plan, with fp32 staging if needed
+  const GradRoute gq = route_input_grad(T, K, N, false, M, B);
+  const GradRoute gr = route_input_grad(T, K, N, out_dtype == AQ_DTYPE_F32, M, B);
+  if (gr.bytes > gq.bytes)
+    return set_error(AQ_ERR_WORKSPACE, "internal: plan for fp32 output needs more workspace");
+  r = check_workspace(workspace, workspace_bytes, gq.bytes);
+  if (r) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* Wt = nullptr;
+  float* partial = nullptr;
+  ws_pointers(gr.rt, workspace, K, N, &Wt, &partial);
+  __half* ones = reinterpret_cast<__half*>(static_cast<uint8_t*>(workspace) + gq.ones_off);
+  cudaError_t e;
+  {
+    ProfScope ps(kProfDecode, st);
+    e = aq::launch_decode_t(codes_packed, codebooks, static_cast<const __half*>(scale),
+                            static_cast<__half*>(Wt), ones, N, K, M, B, st);
+  }
+  if (e != cudaSuccess) return cuda_status(e, "transposed decode launch");
+  // dX = alpha * dY Wt^T: the fp16-activation GEMM over (T, K_red = N, N_out = K), its
+  // epilogue scale alpha * ones[k], no bias
+  CUtensorMap mapA;
+  r = encode_linear_a16(&mapA, dy, T, N);
+  if (r) return r;
+  aq::GemmParams p{};
+  p.T = T;
+  p.N = K;
+  p.K = N;
+  p.conv = 0;
+  p.s_x = alpha;
+  p.scale = ones;
+  p.bias = nullptr;
+  p.y = dx;
+  p.out_f32 = out_dtype == AQ_DTYPE_F32;
+  return run_gemm(mapA, p, gr.rt.pl, codes_packed, codebooks, M, B, Wt, partial, st, false,
+                  nullptr, nullptr, true);
+}
+
 // Device address of g_noalloc_scratch on the current device (the host-side symbol is only
 // a stand-in, never a device address), looked up once per device and context: a context
 // re-created on that device (cudaDeviceReset) gets the array at a new address.

@@ -264,6 +264,81 @@ cudaError_t launch_decode(const void* packed, const void* books, void* W, int N,
                     static_cast<__half*>(W), N, K, M, KB);
 }
 
+// ============================================================== transposed, scaled decode
+// For the input gradient of the layer (Sec. 3.2.1's continuous step back-propagates through
+// it): dX[t][k] = alpha * sum_n dY[t][n] * scale[n] * W[n][k] = alpha * (dY Wt^T)[t][k] with
+// Wt[k][n] = fp16(scale[n] * W[n][k]): W[n][k] decoded by the rule of Eq. 4 (fp32 sum in
+// ascending m, one round to fp16), times the fp16 scale in fp32, one more round to fp16.
+// CTA = 64 output rows n x one 64-wide K block, thread = one (n, group j): it decodes its
+// group and writes the 8 scaled values down a column of a transposed shared-memory tile
+// [64 k][64 n] (rows padded to 66 halves); the tile's rows (64 n values, 128 B each) are
+// then written to Wt.  Block (0, 0) also writes `ones` (K fp16 ones, the unit per-column
+// scale of the gradient GEMM's epilogue).
+constexpr int kTRows = 64;                     // output rows n per CTA
+constexpr int kTPad = 66;                      // tile row stride in halves
+
+template <int EB>
+__global__ void __launch_bounds__(512) decode_t_kernel(const void* __restrict__ packed,
+                                                       const uint4* __restrict__ books,
+                                                       const __half* __restrict__ scale,
+                                                       __half* __restrict__ Wt, __half* ones,
+                                                       int N, int K, int M) {
+  __shared__ __half tile[64 * kTPad];
+  grid_dependency_wait();
+  allow_dependents();
+  const int kb = blockIdx.y;
+  const int n0 = blockIdx.x * kTRows;
+  const int nl = threadIdx.x >> 3, j = threadIdx.x & 7;
+  const int n = n0 + nl;
+  const int G = K / 8;
+  const int grp = kb * 8 + j;
+  if (blockIdx.x == 0 && blockIdx.y == 0)
+    for (int i = threadIdx.x; i < K; i += blockDim.x) ones[i] = __float2half_rn(1.0f);
+  float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (n < N && grp < G) {
+    const int64_t idx = (static_cast<int64_t>(kb) * N + n) * 8 + j;
+    F8 acc;
+    for (int m = 0; m < M; ++m) {
+      const uint32_t c = EB == 1 ? static_cast<const uint8_t*>(packed)[idx * M + m]
+                                 : static_cast<const uint16_t*>(packed)[idx * M + m];
+      widen_add(acc, __ldg(books + (static_cast<int64_t>(m) << (8 * EB)) + c), m == 0);
+    }
+    const uint4 w = narrow(acc);               // the decoded weight, fp16 (Eq. 4 rule)
+    const float sc = __half2float(scale[n]);
+    const __half2* h = reinterpret_cast<const __half2*>(&w);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __half22float2(h[i]);
+      v[2 * i] = __fmul_rn(f.x, sc);
+      v[2 * i + 1] = __fmul_rn(f.y, sc);
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) tile[(j * 8 + e) * kTPad + nl] = __float2half_rn(v[e]);
+  __syncthreads();
+  // row r of the tile = k = kb*64 + r, columns n0 .. n0+63: 8 chunks of 8 halves
+  const int r = threadIdx.x >> 3, ch = threadIdx.x & 7;
+  const int k = kb * 64 + r;
+  const int nc = n0 + ch * 8;
+  if (k < K && nc < N) {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(tile + r * kTPad + ch * 8);
+    const uint4 out = make_uint4(src[0], src[1], src[2], src[3]);
+    *reinterpret_cast<uint4*>(Wt + static_cast<int64_t>(k) * N + nc) = out;   // N % 8 == 0
+  }
+}
+
+cudaError_t launch_decode_t(const void* packed, const void* books, const __half* scale,
+                            __half* Wt, __half* ones, int N, int K, int M, int B,
+                            cudaStream_t st) {
+  const dim3 grid(static_cast<unsigned>((N + kTRows - 1) / kTRows),
+                  static_cast<unsigned>((K + 63) / 64));
+  if (B == 8)
+    return launch_pdl(decode_t_kernel<1>, grid, dim3(512), 0, st, packed,
+                      static_cast<const uint4*>(books), scale, Wt, ones, N, K, M);
+  return launch_pdl(decode_t_kernel<2>, grid, dim3(512), 0, st, packed,
+                    static_cast<const uint4*>(books), scale, Wt, ones, N, K, M);
+}
+
 // ============================================================== kernel-aware decode (g = 9)
 // Sec. 3.1.2 / App. A.1 Eq. A4: one group = the 3x3 taps of one (output channel n,
 // input channel c) filter; codes [N][Cin][M], codebooks [M][2^B][9] fp16.  The

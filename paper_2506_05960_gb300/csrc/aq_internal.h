@@ -145,6 +145,11 @@ cudaError_t launch_pack(const void* canon, void* packed, int N, int K, int M, in
                         cudaStream_t st);
 cudaError_t launch_decode(const void* packed, const void* books, void* W, int N, int K, int M,
                           int B, cudaStream_t st);
+// Wt[k][n] = fp16(scale[n] * W-hat[n][k]) (transposed, scaled decode for the input
+// gradient) and ones[0..K) = 1 (the gradient GEMM's unit epilogue scale).
+cudaError_t launch_decode_t(const void* packed, const void* books, const __half* scale,
+                            __half* Wt, __half* ones, int N, int K, int M, int B,
+                            cudaStream_t st);
 // dC[m][c][e] += sum over groups with code c of s_x*scale[n]*G[n][group element e]
 cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half* scale,
                                  float s_x, float* dC, int N, int K, int g, int M, int B,

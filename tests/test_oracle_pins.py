@@ -432,6 +432,73 @@ def test_kaq_layer_equals_torch_conv_on_oihw_filters(stride):
 
 
 # ----------------------------------------------------------------------------- codebook gradient
+def test_input_grad_brute_force():
+    """dX[t, k] = alpha * sum_n dY[t, n] * scale[n] * (sum_m C_m[b[n, k//g, m]][k % g]), with
+    plain loops over every index (no matmul, no decoded matrix)."""
+    rng = np.random.default_rng(71)
+    T, N, Gr, g, M, n_code = 3, 5, 4, 8, 2, 16
+    books = rng.normal(size=(M, n_code, g)).astype(np.float16)
+    codes = rng.integers(0, n_code, size=(N, Gr, M)).astype(np.uint8)
+    scale = rng.uniform(0.5, 1.5, size=N).astype(np.float16)
+    dy = rng.normal(size=(T, N)).astype(np.float16)
+    ref = np.zeros((T, Gr * g))
+    for t in range(T):
+        for k in range(Gr * g):
+            acc = 0.0
+            for n in range(N):
+                w = 0.0
+                for m in range(M):
+                    w += float(books[m, codes[n, k // g, m], k % g])
+                acc += float(dy[t, n]) * float(scale[n]) * w
+            ref[t, k] = 0.75 * acc
+    got = O.input_grad_f64(dy, codes, books, scale, alpha=0.75)
+    assert np.allclose(got, ref, rtol=1e-13, atol=1e-13)
+
+
+@pytest.mark.parametrize("s_x", [1.0, 0.5])
+def test_input_grad_is_the_derivative_of_the_layer(s_x):
+    """With small-integer codebooks, scales, biases and dY (exact in float64 arithmetic), the
+    loss L(xq) = sum dY * linear_f64(xq) is linear in xq, so a unit step of xq[t, k] changes L
+    by exactly dL/dxq[t, k] = s_x * dL/dX[t, k] = input_grad_f64(alpha = s_x)."""
+    rng = np.random.default_rng(72)
+    T, N, Gr, g, M, n_code = 2, 6, 3, 8, 2, 8
+    books = rng.integers(-4, 5, size=(M, n_code, g)).astype(np.float16)
+    codes = rng.integers(0, n_code, size=(N, Gr, M)).astype(np.uint8)
+    scale = rng.integers(1, 4, size=N).astype(np.float16)
+    bias = rng.integers(-3, 4, size=N).astype(np.float16)
+    dy = rng.integers(-3, 4, size=(T, N)).astype(np.float64)
+    xq = rng.integers(-20, 21, size=(T, Gr * g)).astype(np.int8)
+    W = O.decode_f64(codes, books)
+
+    def loss(x):
+        return float(np.sum(dy * O.linear_f64(x, s_x, W, scale, bias)))
+
+    grad = O.input_grad_f64(dy, codes, books, scale, alpha=s_x)
+    L0 = loss(xq)
+    for t in range(T):
+        for k in range(Gr * g):
+            x1 = xq.copy()
+            x1[t, k] += 1
+            assert loss(x1) - L0 == grad[t, k]
+
+
+def test_input_grad_of_a_unit_output_is_a_scaled_weight_row():
+    """dY = e_(t, n) gives row t of dX = scale[n] * W[n, :], the other rows zero."""
+    rng = np.random.default_rng(73)
+    T, N, Gr, g, M = 3, 4, 2, 8, 3
+    books = rng.normal(size=(M, 256, g)).astype(np.float16)
+    codes = rng.integers(0, 256, size=(N, Gr, M)).astype(np.uint8)
+    scale = rng.uniform(0.5, 1.5, size=N).astype(np.float16)
+    W = O.decode_f64(codes, books)
+    for (t, n) in ((0, 0), (2, 3), (1, 1)):
+        dy = np.zeros((T, N))
+        dy[t, n] = 1.0
+        got = O.input_grad_f64(dy, codes, books, scale)
+        want = np.zeros((T, Gr * g))
+        want[t] = float(scale[n]) * W[n]
+        assert np.array_equal(got, want)
+
+
 def test_codebook_grad_brute_force():
     """Backward of Eq. 4: every use of codeword c in codebook m adds its group's gradient."""
     rng = np.random.default_rng(31)
