@@ -932,6 +932,18 @@ def main():
         lib["aq_gemm_over_cublas_qkv"] = achieved / lib["qkv T=4096 K=960 N=2880"]["tflops"]
         layers["library GEMM of the same shapes (context)"] = lib
         torch.cuda.empty_cache()
+        # the fixed cost of one dependent launch under graph replay: our quantizer on 16
+        # elements (the least work a library kernel can do), 8 launches per graph
+        fx = torch.zeros(16, dtype=torch.float16, device=dev)
+        fq = torch.empty(16, dtype=torch.int8, device=dev)
+        gfl = capture(torch, stream, lambda: [aq.aq_quant_act(fx, fq, 16, 0.02, stream=stream)
+                                              for _ in range(8)])
+        floor_us = replay_ms(torch, stream, gfl, 50) / 8 * 1e3
+        del gfl
+        layers["launch floor (one dependent library launch, graph replay)"] = {
+            "us_per_launch": floor_us,
+            "what": "aq_quant_act on 16 elements, 8 launches per CUDA graph: the per-launch "
+                    "fixed cost that bounds the token-poor layers below"}
         from aq_synth import SEEDS, WORKLOADS, make_conv
         for name, wl in (("conv3x3 16x64x64x192->192 W4A8 (4x8)", "conv64"),
                          ("conv3x3 2x8x8x960->960 one 2^16 codebook (1x16)", "conv8_book16")):
@@ -942,9 +954,14 @@ def main():
             stream.synchronize()
             gl = capture(torch, stream, lambda: [L.step(stream) for _ in range(8)])
             ms = replay_ms(torch, stream, gl, 20) / 8
+            s_ = L.spec
+            plan = aq.aq_conv2d_plan(s_.Nb, s_.H, s_.W, s_.Cin, s_.Cout, 3, 3, s_.stride, 1, 8,
+                                     L.M, L.B, L.path)
             layers[name] = {"us_per_step": ms * 1e3,
                             "tflops": L.flops / (ms * 1e-3) / 1e12,
                             "tensor_roofline_frac": L.flops / (peaks["bf16_tflops"] * 1e12) / (ms * 1e-3),
+                            "plan": plan,
+                            "launch_floor_us": floor_us,
                             "step": "quantizer + layer (AUTO path), CUDA graph replay"}
             del gl, L
         # backward of Eq. 4 (codebook gradient) on the headline layer: HBM-bound read of G
