@@ -374,6 +374,34 @@ AQ_API int aq_conv2d_nhwc_q8(const int8_t* xq, float s_x, const void* codes_pack
                              int kh, int kw, int stride, int pad, int g, int M, int B,
                              void* workspace, size_t workspace_bytes, int path, void* stream);
 
+/* ---- 3x3 convolution from fp16 activations ---------------------------------
+ * aq_quant_act(x, xq, Nb*H*W*Cin, s_x) followed by aq_conv2d_nhwc(xq, s_x, ...)
+ * in one call (Sec. 4.2.3 quantizer, then the convolution above).  As for
+ * aq_linear_f16, the quantized activations stay at the start of the workspace:
+ * on the dense paths as fp16 values (each 8-bit code exactly), which the tensor
+ * cores read from shared memory through 4-D NHWC boxes with the 128-byte
+ * swizzle; on the fused path as int8.  Same codes as aq_quant_act; the output
+ * equals the two calls' bit for bit when both run the same plan (N tile and K
+ * split, aq_set_plan_override), and is within the layer tolerance otherwise.
+ *   x fp16 [Nb][H][W][Cin]; s_x finite and > 0 (AQ_ERR_SHAPE); out_dtype F16 or
+ *   F32 (AQ_DTYPE_I8: AQ_ERR_UNSUPPORTED).  Shapes, codes and the other arrays
+ *   as for aq_conv2d_nhwc.
+ *   Workspace: aq_conv2d_f16_workspace_size() bytes = 2*Nb*H*W*Cin rounded up
+ *   to 1 KB, then the layer's workspace for this plan (with AQ_PATH_PREDECODED,
+ *   W-hat is expected right after the activation region).
+ *   aq_conv2d_f16_plan: the plan these calls run; info as for aq_linear_plan.  */
+AQ_API int aq_conv2d_f16_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh,
+                                        int kw, int stride, int pad, int g, int M, int B,
+                                        int path, size_t* bytes);
+AQ_API int aq_conv2d_f16_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
+                              int stride, int pad, int g, int M, int B, int path, int* info,
+                              int n_info);
+AQ_API int aq_conv2d_nhwc_f16(const void* x, float s_x, const void* codes_packed,
+                              const void* codebooks, const void* scale, const void* bias,
+                              void* y, int out_dtype, int Nb, int H, int W, int Cin, int Cout,
+                              int kh, int kw, int stride, int pad, int g, int M, int B,
+                              void* workspace, size_t workspace_bytes, int path, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

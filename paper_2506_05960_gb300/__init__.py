@@ -10,7 +10,7 @@ raises.
 
 from ._binding import (  # noqa: F401
     AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_DTYPE_I8, AQ_PATH_AUTO, AQ_PATH_DENSE, AQ_PATH_FUSED, AQ_PATH_LUT, AQ_PATH_FEW_TOKENS, AQ_PATH_PREDECODED,
-    AQError, aq_abi_version, aq_codebook_grad, aq_code_update, aq_conv2d_nhwc, aq_conv2d_nhwc_q8, aq_conv2d_plan, aq_conv2d_workspace_size, aq_decode,
+    AQError, aq_abi_version, aq_codebook_grad, aq_code_update, aq_conv2d_f16_plan, aq_conv2d_f16_workspace_size, aq_conv2d_nhwc, aq_conv2d_nhwc_f16, aq_conv2d_nhwc_q8, aq_conv2d_plan, aq_conv2d_workspace_size, aq_decode,
     aq_device_error, aq_last_error_string, aq_linear, aq_linear_f16, aq_linear_f16_workspace_size,
     aq_linear_f16_plan, aq_linear_a16, aq_linear_a16_plan, aq_linear_a16_workspace_size,
     aq_linear_noalloc, aq_linear_q8,

@@ -68,6 +68,10 @@ _SIGNATURES = {
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_nhwc_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float]
                           + [_c_int] * 12 + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_conv2d_f16_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
+    "aq_conv2d_f16_plan": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_conv2d_nhwc_f16": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
+                           + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
 }
 
 _lib = None
@@ -349,3 +353,28 @@ def aq_conv2d_nhwc_q8(xq, s_x, codes_packed, codebooks, scale, bias, yq, s_out, 
         _ptr(yq), float(s_out), Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B,
         _ptr(workspace), int(workspace_bytes), path, _stream(stream)), "aq_conv2d_nhwc_q8")
 
+
+def aq_conv2d_f16_workspace_size(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4,
+                                 B=8, path=AQ_PATH_AUTO) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_conv2d_f16_workspace_size(Nb, H, W, Cin, Cout, kh, kw, stride, pad,
+                                                       g, M, B, path, ctypes.byref(out)),
+           "aq_conv2d_f16_workspace_size")
+    return out.value
+
+
+def aq_conv2d_f16_plan(Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8,
+                       path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_conv2d_nhwc_f16 runs for these shapes (diagnostics; no device access)."""
+    return _plan(load_library().aq_conv2d_f16_plan, "aq_conv2d_f16_plan", Nb, H, W, Cin, Cout,
+                 kh, kw, stride, pad, g, M, B, path)
+
+
+def aq_conv2d_nhwc_f16(x, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, Nb, H, W, Cin,
+                       Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8, workspace=None,
+                       workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """aq_quant_act + aq_conv2d_nhwc in one call from fp16 NHWC activations."""
+    _check(load_library().aq_conv2d_nhwc_f16(
+        _ptr(x), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
+        _ptr(y), out_dtype, Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, _ptr(workspace),
+        int(workspace_bytes), path, _stream(stream)), "aq_conv2d_nhwc_f16")

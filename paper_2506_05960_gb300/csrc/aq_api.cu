@@ -571,7 +571,7 @@ int sm_count() {
 int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const void* codes_packed,
              const void* codebooks, int M, int B, void* Wdec, float* partial, cudaStream_t st,
              bool kaq = false, const void* x16 = nullptr, int8_t* xq = nullptr,
-             bool predecoded = false) {
+             bool predecoded = false, int64_t x_elems = 0) {
   const bool fused = Wdec == nullptr;
   if (!plan_ring_ok(pl)) return set_error(AQ_ERR_UNSUPPORTED, "plan: partial tile exceeds the ring");
   p.fused = fused ? 1 : 0;
@@ -637,7 +637,9 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   }
   if (r) return r;
   cudaError_t e;
-  const int64_t x_elems = static_cast<int64_t>(T) * K;
+  // the activation tensor x16 quantized into xq: T x K for a linear layer; the caller gives the
+  // input tensor's size for a convolution (T, K there are output pixels and 9 * Cin)
+  if (x_elems == 0) x_elems = static_cast<int64_t>(T) * K;
   if (x16) {
     ProfScope ps(kProfQuant, st);
     e = pl.a16 ? aq::launch_quant_act_f16(x16, reinterpret_cast<__half*>(xq), x_elems, p.s_x, st)
@@ -682,6 +684,32 @@ Route route_gemm(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, 
   rt.pl = plan_gemm(T, N, K, m_tiles, true, f32_out, rt.fused, M, B, a16 && !rt.fused);
   rt.ws = rt.fused ? fused_ws_bytes(T, N, rt.pl) : dense_ws_bytes(T, N, K, rt.pl);
   return rt;
+}
+
+// Activations of a layer call: int8 codes (aq_linear, aq_conv2d_nhwc), fp16 activations this
+// call quantizes (aq_linear_f16, aq_conv2d_nhwc_f16), or the codes already held as fp16 values
+// (aq_linear_a16).
+enum ActKind { kActInt8 = 0, kActF16 = 1, kActF16Codes = 2 };
+
+// The tensor-core form of a layer on the dense paths.  The shared-memory A form (fp16 A) takes N
+// tiles up to 256 wide but each of its MMAs costs at least ~138 cycles (128 x N x 16, measured);
+// the tensor-memory A form (int8 codes converted into tensor memory) takes N tiles up to 192.  A
+// call that quantizes fp16 activations itself writes fp16 codes only when the fp16 form's plan
+// has no K split and a wider N tile than the int8 form's plan; codes given as fp16 always take
+// it.  Measured on GB300 (GEMM alone, weights decoded beforehand, us int8 / fp16 form): qkv
+// 4096 x 960 x 2880 28.1 / 25.1 (N tiles 160 / 224); 8192 x 576 x 1728 24.0 / 21.9 (192 / 256);
+// 16384 x 192 x 576 18.0 / 14.5 (96 / 192); 2048 x 960 x 2880 16.8 / 17.3 (160 / 160);
+// 2048 x 960 x 960 9.5 / 15.1 (fp16 plan split 2); the 64x64 W4A8 3x3 conv, whole call,
+// 54.7 / 60.9 (192 / 192).
+Route route_layer(int rp, int T, int N, int K, int m_tiles, bool f32_out, int M, int B,
+                  ActKind act) {
+  const bool dense = rp == AQ_PATH_DENSE || rp == AQ_PATH_PREDECODED;
+  if (act == kActInt8 || !dense) return route_gemm(rp, T, N, K, m_tiles, f32_out, M, B, false);
+  const Route r16 = route_gemm(rp, T, N, K, m_tiles, f32_out, M, B, true);
+  // (a plan override wider than the int8 form's widest tile can only mean the fp16 form)
+  if (act == kActF16Codes || g_plan_override.BN > aq::kA8MaxBN) return r16;
+  const Route r8 = route_gemm(rp, T, N, K, m_tiles, f32_out, M, B, false);
+  return (r16.pl.splits == 1 && r16.pl.BN > r8.pl.BN) ? r16 : r8;
 }
 
 int check_workspace(const void* workspace, size_t workspace_bytes, size_t need) {
@@ -740,7 +768,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
                 const void* scale, const void* bias, void* y, int out_dtype, float s_out, int T,
                 int K, int N, int g, int M, int B, void* workspace, size_t workspace_bytes,
                 int path, void* stream, const void* x16 = nullptr, const void* xh = nullptr);
-int linear_ws(int T, int K, int N, int g, int M, int B, int path, bool a16, size_t* bytes);
+int linear_ws(int T, int K, int N, int g, int M, int B, int path, ActKind act, size_t* bytes);
 
 // Path of aq_linear_a16 (fp16 activations): the dense tensor-core paths only.
 int resolve_a16_path(int path) {
@@ -751,7 +779,10 @@ int resolve_a16_path(int path) {
 int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
-              int B, void* workspace, size_t workspace_bytes, int path, void* stream);
+              int B, void* workspace, size_t workspace_bytes, int path, void* stream,
+              const void* x16 = nullptr);
+int conv_ws(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
+            int M, int B, int path, bool a16, size_t* bytes);
 
 }  // namespace
 
@@ -893,7 +924,7 @@ int aq_quant_act(const void* x, int8_t* xq, int64_t numel, float s_x, void* stre
 }
 
 int aq_linear_workspace_size(int T, int K, int N, int g, int M, int B, int path, size_t* bytes) {
-  return linear_ws(T, K, N, g, M, B, path, false, bytes);
+  return linear_ws(T, K, N, g, M, B, path, kActInt8, bytes);
 }
 
 namespace {
@@ -941,7 +972,8 @@ int linear_plan_impl(int T, int K, int N, int g, int M, int B, int path, bool a1
   const int rp = a16_only ? resolve_a16_path(path) : resolve_linear_path(path, T, B);
   if (rp < 0) return path_error(rp, path);
   if (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT) return fill_plan_info(rp, nullptr, info, n_info);
-  const Route rt = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B, a16);
+  const Route rt = route_layer(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B,
+                              a16_only ? kActF16Codes : (a16 ? kActF16 : kActInt8));
   return fill_plan_info(rp, &rt.pl, info, n_info);
 }
 }  // namespace
@@ -990,7 +1022,7 @@ static size_t f16_act_bytes(int T, int K) { return align_up(static_cast<size_t>(
 int aq_linear_f16_workspace_size(int T, int K, int N, int g, int M, int B, int path,
                                  size_t* bytes) {
   size_t rest = 0;
-  const int r = linear_ws(T, K, N, g, M, B, path, true, &rest);
+  const int r = linear_ws(T, K, N, g, M, B, path, kActF16, &rest);
   if (r) return r;
   *bytes = f16_act_bytes(T, K) + rest;
   return ok();
@@ -1000,7 +1032,7 @@ int aq_linear_a16_workspace_size(int T, int K, int N, int g, int M, int B, int p
                                  size_t* bytes) {
   const int rp = resolve_a16_path(path);
   if (rp < 0) return path_error(-2, path);
-  return linear_ws(T, K, N, g, M, B, rp, true, bytes);
+  return linear_ws(T, K, N, g, M, B, rp, kActF16Codes, bytes);
 }
 
 int aq_linear_a16(const void* xh, float s_x, const void* codes_packed, const void* codebooks,
@@ -1043,7 +1075,7 @@ int aq_linear_f16(const void* x, float s_x, const void* codes_packed, const void
 
 namespace {
 
-int linear_ws(int T, int K, int N, int g, int M, int B, int path, bool a16, size_t* bytes) {
+int linear_ws(int T, int K, int N, int g, int M, int B, int path, ActKind act, size_t* bytes) {
   if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
   int r = check_format(g, M, B);
   if (r) return r;
@@ -1059,7 +1091,7 @@ int linear_ws(int T, int K, int N, int g, int M, int B, int path, bool a16, size
     *bytes = plan_lut(T, K, N, M).ws_bytes;
     return ok();
   }
-  *bytes = route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B, a16).ws;
+  *bytes = route_layer(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B, act).ws;
   return ok();
 }
 
@@ -1160,12 +1192,12 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     if (e != cudaSuccess) return cuda_status(e, "LUT reduce launch");
     return ok();
   }
-  // fp16 activations (given, or written by this call's quantizer) on the dense paths:
-  // the shared-memory A form
-  const bool a16 = (xh != nullptr || x16 != nullptr) &&
-                   (rp == AQ_PATH_DENSE || rp == AQ_PATH_PREDECODED);
-  const Route rt =
-      route_gemm(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, out_dtype == AQ_DTYPE_F32, M, B, a16);
+  // fp16 activations (given as codes, or quantized by this call) on the dense paths may run
+  // the shared-memory A form (route_layer)
+  const Route rt = route_layer(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM,
+                               out_dtype == AQ_DTYPE_F32, M, B,
+                               xh ? kActF16Codes : (x16 ? kActF16 : kActInt8));
+  const bool a16 = rt.pl.a16 != 0;
   r = check_workspace(workspace, workspace_bytes, rt.ws);
   if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1197,7 +1229,12 @@ extern "C" {
 
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
                              int pad, int g, int M, int B, int path, size_t* bytes) {
-  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  return conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, false, bytes);
+}
+
+namespace {
+int conv_plan_impl(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                   int g, int M, int B, int path, bool a16, int* info, int n_info) {
   int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
@@ -1207,25 +1244,60 @@ int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, in
   if (r) return r;
   const int rp = resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
-  const int K = kh * kw * Cin;
-  const int T = Nb * cg.Ho * cg.Wo;
-  *bytes = route_gemm(rp, T, Cout, K, cg.m_tiles, false, M, B).ws;
-  return ok();
+  const Route rt = route_layer(rp, Nb * cg.Ho * cg.Wo, Cout, kh * kw * Cin, cg.m_tiles, false, M,
+                               B, a16 ? kActF16 : kActInt8);
+  return fill_plan_info(rp, &rt.pl, info, n_info);
 }
+}  // namespace
 
 int aq_conv2d_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
                    int g, int M, int B, int path, int* info, int n_info) {
-  int r = check_format(g, M, B, true);
+  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, false, info,
+                        n_info);
+}
+
+int aq_conv2d_f16_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
+                       int pad, int g, int M, int B, int path, int* info, int n_info) {
+  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, true, info,
+                        n_info);
+}
+
+int aq_conv2d_f16_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
+                                 int stride, int pad, int g, int M, int B, int path,
+                                 size_t* bytes) {
+  size_t rest = 0;
+  const int r = conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, true, &rest);
   if (r) return r;
-  r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
-  if (r) return r;
-  ConvGeom cg;
-  r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
-  if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles, g);
-  if (rp < 0) return path_error(rp, path);
-  const Route rt = route_gemm(rp, Nb * cg.Ho * cg.Wo, Cout, kh * kw * Cin, cg.m_tiles, false, M, B);
-  return fill_plan_info(rp, &rt.pl, info, n_info);
+  *bytes = f16_act_bytes(Nb * H * W, Cin) + rest;
+  return ok();
+}
+
+int aq_conv2d_nhwc_f16(const void* x, float s_x, const void* codes_packed, const void* codebooks,
+                       const void* scale, const void* bias, void* y, int out_dtype, int Nb, int H,
+                       int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
+                       int M, int B, void* workspace, size_t workspace_bytes, int path,
+                       void* stream) {
+  if (out_dtype == AQ_DTYPE_I8)
+    return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_conv2d_nhwc_q8");
+  if (!(s_x > 0.0f) || s_x == __builtin_inff())
+    return set_error(AQ_ERR_SHAPE, "s_x must be finite and > 0");
+  if (Nb < 0 || H <= 0 || W <= 0 || Cin <= 0)
+    return set_error(AQ_ERR_SHAPE, "conv sizes must be positive (Nb >= 0)");
+  if (Nb == 0)  // argument checks only, as aq_conv2d_nhwc
+    return conv_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, 0, H,
+                     W, Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes, path,
+                     stream);
+  if (!x) return set_error(AQ_ERR_NULL, "x is NULL");
+  if (!aligned16(x)) return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
+  const size_t xq_bytes = f16_act_bytes(Nb * H * W, Cin);
+  if (!workspace || workspace_bytes < xq_bytes || !aligned16(workspace))
+    return set_error(AQ_ERR_WORKSPACE, "workspace needs at least %zu bytes (got %zu)", xq_bytes,
+                     workspace_bytes);
+  int8_t* xq = static_cast<int8_t*>(workspace);
+  void* rest = static_cast<uint8_t*>(workspace) + xq_bytes;
+  return conv_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, Nb, H, W,
+                   Cin, Cout, kh, kw, stride, pad, g, M, B, rest, workspace_bytes - xq_bytes, path,
+                   stream, x);
 }
 
 int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
@@ -1253,10 +1325,14 @@ int aq_conv2d_nhwc_q8(const int8_t* xq, float s_x, const void* codes_packed,
 
 namespace {
 
+// x16 != nullptr (aq_conv2d_nhwc_f16): the fp16 NHWC activations, quantized into xq by this
+// call -- on the dense paths as the codes' fp16 values (the region holds Nb*H*W*Cin*2 bytes)
+// read by the shared-memory A form of the GEMM, else as int8 codes.
 int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
-              int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
+              int B, void* workspace, size_t workspace_bytes, int path, void* stream,
+              const void* x16) {
   int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
@@ -1277,7 +1353,10 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  const Route rt = route_gemm(rp, T, Cout, K, cg.m_tiles, out_dtype == AQ_DTYPE_F32, M, B);
+  // fp16 activations quantized by this call may run the shared-memory A form (route_layer)
+  const Route rt = route_layer(rp, T, Cout, K, cg.m_tiles, out_dtype == AQ_DTYPE_F32, M, B,
+                               x16 ? kActF16 : kActInt8);
+  const bool a16 = rt.pl.a16 != 0;
   r = check_workspace(workspace, workspace_bytes, rt.ws);
   if (r) return r;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1286,16 +1365,19 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
   ws_pointers(rt, workspace, Cout, K, &Wdec, &partial);
   CUtensorMap mapA;
   {
+    // element size 1 (int8 codes, 64-byte swizzle) or 2 (fp16 codes, 128-byte swizzle: the
+    // 64-channel box row is one 128-byte swizzle span, the layout of the weight boxes)
+    const cuuint64_t es_bytes = a16 ? 2 : 1;
     cuuint64_t dims[4] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W),
                           static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(Nb)};
-    cuuint64_t strides[3] = {static_cast<cuuint64_t>(Cin), static_cast<cuuint64_t>(W) * Cin,
-                             static_cast<cuuint64_t>(H) * W * Cin};
+    cuuint64_t strides[3] = {es_bytes * Cin, es_bytes * W * Cin, es_bytes * H * W * Cin};
     // stride s: the box spans s*bw x s*bh input pixels and delivers every s-th one
     cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(stride * cg.bw),
                          static_cast<cuuint32_t>(stride * cg.bh), static_cast<cuuint32_t>(cg.bn)};
     cuuint32_t es[4] = {1, static_cast<cuuint32_t>(stride), static_cast<cuuint32_t>(stride), 1};
-    r = encode(&mapA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq, dims, strides, box,
-               CU_TENSOR_MAP_SWIZZLE_64B, es);
+    r = encode(&mapA, a16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq,
+               dims, strides, box, a16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+               es);
     if (r) return r;
   }
   aq::GemmParams p{};
@@ -1317,7 +1399,26 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
   p.out_q8 = out_dtype == AQ_DTYPE_I8;
   p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st,
-                  g == kKaqGroup, nullptr, nullptr, rt.predecoded);
+                  g == kKaqGroup, x16, const_cast<int8_t*>(xq), rt.predecoded,
+                  static_cast<int64_t>(Nb) * H * W * Cin);
+}
+
+int conv_ws(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
+            int M, int B, int path, bool a16, size_t* bytes) {
+  if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
+  int r = check_format(g, M, B, true);
+  if (r) return r;
+  r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
+  if (r) return r;
+  ConvGeom cg;
+  r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
+  if (r) return r;
+  const int rp = resolve_conv_path(path, cg.m_tiles, g);
+  if (rp < 0) return path_error(rp, path);
+  const int K = kh * kw * Cin;
+  const int T = Nb * cg.Ho * cg.Wo;
+  *bytes = route_layer(rp, T, Cout, K, cg.m_tiles, false, M, B, a16 ? kActF16 : kActInt8).ws;
+  return ok();
 }
 
 }  // namespace

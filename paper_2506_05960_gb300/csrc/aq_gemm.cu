@@ -968,7 +968,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
   // TMEM holds just the two accumulators; the TMEM-A form needs two A slots beside them
   if (a16 && (p.fused || (p.sb != 1 && p.sb != 2) || 2 * p.BN > kTmemCols))
     return cudaErrorInvalidConfiguration;
-  if (!a16 && (p.BN > 192 || 2 * p.acc_stride + 2 * kASlotCols > kTmemCols))
+  if (!a16 && (p.BN > kA8MaxBN || 2 * p.acc_stride + 2 * kASlotCols > kTmemCols))
     return cudaErrorInvalidConfiguration;
   if (p.BN % 32 != 0 || p.BN < 32 || p.BN > kMaxBN || p.stages < 1 || p.stages > kMaxStages)
     return cudaErrorInvalidConfiguration;

@@ -15,8 +15,8 @@ namespace aq {
 constexpr int kBM = 128;        // rows (tokens / output pixels) per tile = TMEM lanes
 constexpr int kBK = 64;         // K per TMA box / swizzle row (128 bytes of fp16)
 constexpr int kStageBlocks = 2; // 64-wide K blocks per pipeline stage (8 MMAs of K = 16)
-constexpr int kMaxBN = 256;     // widest N tile: 2 fp32 accumulators in TMEM (the TMEM-A
-                                // form also needs >= 2 A slots beside them: BN <= 192)
+constexpr int kMaxBN = 256;     // widest N tile: 2 fp32 accumulators in TMEM
+constexpr int kA8MaxBN = 192;   // the TMEM-A form also needs >= 2 A slots beside them
 constexpr int kMaxStages = 8;   // pipeline ring depth bound
 constexpr int kMaxClusterSplits = 8;  // K splits summed inside one cluster (portable size)
 

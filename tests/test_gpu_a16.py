@@ -187,7 +187,7 @@ def test_f16_quantizer_writes_codes_as_fp16():
     its workspace: exactly the codes of aq_quant_act (the oracle's rule)."""
     import torch
     import paper_2506_05960_gb300 as aq
-    T, K, N = 640, 960, 2880
+    T, K, N = 4096, 960, 2880
     inp, packed = _layer(T, K, N, seed=21)
     x16 = make_f16_activations((T, K), seed=4, std=2.0)
     s_x = float(np.float32(0.05))
