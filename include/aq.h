@@ -67,7 +67,10 @@ extern "C" {
 typedef enum aq_dtype {
   AQ_DTYPE_F16 = 0,   /* output fp16, round to nearest even */
   AQ_DTYPE_F32 = 1,   /* output fp32                        */
-  AQ_DTYPE_I8 = 2     /* output int8, quantized (the _q8 entry points only) */
+  AQ_DTYPE_I8 = 2,    /* int8 codes of the 8-bit activation rule: output of the _q8 and
+                         _ex calls (quantized with s_out); input of the _ex calls */
+  AQ_DTYPE_F16_CODES = 3  /* the same codes held as fp16 values (exact): output and input
+                             of the _ex calls; the layout the shared-memory A form reads */
 } aq_dtype;
 
 typedef enum aq_path {
@@ -401,6 +404,42 @@ AQ_API int aq_conv2d_nhwc_f16(const void* x, float s_x, const void* codes_packed
                               void* y, int out_dtype, int Nb, int H, int W, int Cin, int Cout,
                               int kh, int kw, int stride, int pad, int g, int M, int B,
                               void* workspace, size_t workspace_bytes, int path, void* stream);
+
+/* ---- layer calls with the activation and output kinds as arguments ----------
+ * The linear layer / 3x3 convolution above, with
+ *   act_dtype  AQ_DTYPE_I8: act holds int8 codes (as aq_linear / aq_conv2d_nhwc), or
+ *              AQ_DTYPE_F16_CODES: act holds the codes as fp16 values (as aq_linear_a16); the
+ *              tensor cores then read them from shared memory, on a dense path (AUTO means
+ *              AQ_PATH_DENSE; AQ_PATH_FUSED, _LUT, _FEW_TOKENS: AQ_ERR_UNSUPPORTED);
+ *   out_dtype  AQ_DTYPE_F16 or AQ_DTYPE_F32 (s_out unused), or AQ_DTYPE_I8 /
+ *              AQ_DTYPE_F16_CODES: the next layer's codes under the activation rule with
+ *              scale s_out applied to the fp16-rounded output (as aq_linear_q8), stored as
+ *              int8 (N % 16 == 0) or as their fp16 values.
+ * A chain of layers can so hand each layer its activations in the form its own plan reads
+ * (aq_linear_f16_plan / aq_conv2d_f16_plan report, in info[6], whether the shared-memory A
+ * form is the faster one for a shape).  The codes as fp16 values and as int8 give the same
+ * bits when both run the same plan (N tile and K split).  Shapes, paths, workspace and
+ * errors otherwise as for the calls above; act_dtype other than the two: AQ_ERR_UNSUPPORTED. */
+AQ_API int aq_linear_ex_workspace_size(int act_dtype, int T, int K, int N, int g, int M, int B,
+                                       int path, size_t* bytes);
+AQ_API int aq_linear_ex_plan(int act_dtype, int T, int K, int N, int g, int M, int B, int path,
+                             int* info, int n_info);
+AQ_API int aq_linear_ex(const void* act, int act_dtype, float s_x, const void* codes_packed,
+                        const void* codebooks, const void* scale, const void* bias, void* y,
+                        int out_dtype, float s_out, int T, int K, int N, int g, int M, int B,
+                        void* workspace, size_t workspace_bytes, int path, void* stream);
+AQ_API int aq_conv2d_ex_workspace_size(int act_dtype, int Nb, int H, int W, int Cin, int Cout,
+                                       int kh, int kw, int stride, int pad, int g, int M, int B,
+                                       int path, size_t* bytes);
+AQ_API int aq_conv2d_ex_plan(int act_dtype, int Nb, int H, int W, int Cin, int Cout, int kh,
+                             int kw, int stride, int pad, int g, int M, int B, int path,
+                             int* info, int n_info);
+AQ_API int aq_conv2d_nhwc_ex(const void* act, int act_dtype, float s_x,
+                             const void* codes_packed, const void* codebooks, const void* scale,
+                             const void* bias, void* y, int out_dtype, float s_out, int Nb, int H,
+                             int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
+                             int M, int B, void* workspace, size_t workspace_bytes, int path,
+                             void* stream);
 
 #ifdef __cplusplus
 }

@@ -14,7 +14,7 @@ import os
 _PKG = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_PKG, "lib", "libaq_gb300.so")
 
-AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_DTYPE_I8 = 0, 1, 2
+AQ_DTYPE_F16, AQ_DTYPE_F32, AQ_DTYPE_I8, AQ_DTYPE_F16_CODES = 0, 1, 2, 3
 AQ_PATH_AUTO, AQ_PATH_DENSE, AQ_PATH_FUSED, AQ_PATH_LUT, AQ_PATH_FEW_TOKENS = 0, 1, 2, 3, 4
 AQ_PATH_PREDECODED = 5
 
@@ -68,6 +68,15 @@ _SIGNATURES = {
                        + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_nhwc_q8": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_float]
                           + [_c_int] * 12 + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_linear_ex_workspace_size": (_c_int, [_c_int] * 8 + [ctypes.POINTER(_c_size_t)]),
+    "aq_linear_ex_plan": (_c_int, [_c_int] * 8 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_linear_ex": (_c_int, [_c_void_p, _c_int, _c_float] + [_c_void_p] * 5 + [_c_int, _c_float]
+                     + [_c_int] * 6 + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
+    "aq_conv2d_ex_workspace_size": (_c_int, [_c_int] * 14 + [ctypes.POINTER(_c_size_t)]),
+    "aq_conv2d_ex_plan": (_c_int, [_c_int] * 14 + [ctypes.POINTER(_c_int), _c_int]),
+    "aq_conv2d_nhwc_ex": (_c_int, [_c_void_p, _c_int, _c_float] + [_c_void_p] * 5
+                          + [_c_int, _c_float] + [_c_int] * 12
+                          + [_c_void_p, _c_size_t, _c_int, _c_void_p]),
     "aq_conv2d_f16_workspace_size": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_size_t)]),
     "aq_conv2d_f16_plan": (_c_int, [_c_int] * 13 + [ctypes.POINTER(_c_int), _c_int]),
     "aq_conv2d_nhwc_f16": (_c_int, [_c_void_p, _c_float] + [_c_void_p] * 5 + [_c_int] * 13
@@ -378,3 +387,56 @@ def aq_conv2d_nhwc_f16(x, s_x, codes_packed, codebooks, scale, bias, y, out_dtyp
         _ptr(x), float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale), _ptr(bias),
         _ptr(y), out_dtype, Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, _ptr(workspace),
         int(workspace_bytes), path, _stream(stream)), "aq_conv2d_nhwc_f16")
+
+
+def aq_linear_ex_workspace_size(act_dtype, T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_linear_ex_workspace_size(act_dtype, T, K, N, g, M, B, path,
+                                                      ctypes.byref(out)),
+           "aq_linear_ex_workspace_size")
+    return out.value
+
+
+def aq_linear_ex_plan(act_dtype, T, K, N, g=8, M=2, B=8, path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_linear_ex runs for these shapes and activation kind (no device access)."""
+    return _plan(load_library().aq_linear_ex_plan, "aq_linear_ex_plan", act_dtype, T, K, N, g,
+                 M, B, path)
+
+
+def aq_linear_ex(act, act_dtype, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, s_out,
+                 T, K, N, g=8, M=2, B=8, workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO,
+                 stream=None) -> None:
+    """The linear layer with the activation kind (int8 or fp16 codes) and the output kind
+    (fp16, fp32, int8 codes or fp16 codes with scale s_out) as arguments."""
+    _check(load_library().aq_linear_ex(
+        _ptr(act), act_dtype, float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale),
+        _ptr(bias), _ptr(y), out_dtype, float(s_out), T, K, N, g, M, B, _ptr(workspace),
+        int(workspace_bytes), path, _stream(stream)), "aq_linear_ex")
+
+
+def aq_conv2d_ex_workspace_size(act_dtype, Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1,
+                                g=8, M=4, B=8, path=AQ_PATH_AUTO) -> int:
+    out = _c_size_t(0)
+    _check(load_library().aq_conv2d_ex_workspace_size(act_dtype, Nb, H, W, Cin, Cout, kh, kw,
+                                                      stride, pad, g, M, B, path,
+                                                      ctypes.byref(out)),
+           "aq_conv2d_ex_workspace_size")
+    return out.value
+
+
+def aq_conv2d_ex_plan(act_dtype, Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4,
+                      B=8, path=AQ_PATH_AUTO) -> dict:
+    """The plan aq_conv2d_nhwc_ex runs for these shapes and activation kind (no device access)."""
+    return _plan(load_library().aq_conv2d_ex_plan, "aq_conv2d_ex_plan", act_dtype, Nb, H, W, Cin,
+                 Cout, kh, kw, stride, pad, g, M, B, path)
+
+
+def aq_conv2d_nhwc_ex(act, act_dtype, s_x, codes_packed, codebooks, scale, bias, y, out_dtype,
+                      s_out, Nb, H, W, Cin, Cout, kh=3, kw=3, stride=1, pad=1, g=8, M=4, B=8,
+                      workspace=None, workspace_bytes=0, path=AQ_PATH_AUTO, stream=None) -> None:
+    """The 3x3 NHWC convolution with the activation and output kinds as arguments."""
+    _check(load_library().aq_conv2d_nhwc_ex(
+        _ptr(act), act_dtype, float(s_x), _ptr(codes_packed), _ptr(codebooks), _ptr(scale),
+        _ptr(bias), _ptr(y), out_dtype, float(s_out), Nb, H, W, Cin, Cout, kh, kw, stride, pad,
+        g, M, B, _ptr(workspace), int(workspace_bytes), path, _stream(stream)),
+           "aq_conv2d_nhwc_ex")

@@ -616,7 +616,7 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
     cuuint32_t box[3] = {32, 32, 1};
     r = encode(&mapY, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, p.partial, dims, strides, box,
                CU_TENSOR_MAP_SWIZZLE_128B);
-  } else if (p.out_q8) {
+  } else if (p.out_q8 == aq::kOutCodesI8) {
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(T)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(N)};
     cuuint32_t box[2] = {32, 32};
@@ -749,14 +749,21 @@ int encode_linear_a16(CUtensorMap* mapA, const void* xh, int T, int K) {
                 CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
+// GemmParams::out_q8 / SkinnyParams::out_q8 of an output dtype.
+int out_codes(int out_dtype) {
+  return out_dtype == AQ_DTYPE_I8 ? aq::kOutCodesI8
+                                  : (out_dtype == AQ_DTYPE_F16_CODES ? aq::kOutCodesF16 : 0);
+}
+
 // Output kinds of the layer entry points: AQ_DTYPE_F16 / AQ_DTYPE_F32 through
 // aq_linear / aq_conv2d_nhwc, AQ_DTYPE_I8 (quantized with s_out) through the _q8
 // variants.  int8 rows need N % 16 == 0 (16-byte TMA row stride).
 int check_output(int out_dtype, float s_out, int N) {
-  if (out_dtype == AQ_DTYPE_I8) {
+  if (out_dtype == AQ_DTYPE_I8 || out_dtype == AQ_DTYPE_F16_CODES) {
     if (!(s_out > 0.0f) || s_out == __builtin_inff())
       return set_error(AQ_ERR_SHAPE, "s_out must be finite and > 0");
-    if (N % 16 != 0) return set_error(AQ_ERR_SHAPE, "int8 output needs N %% 16 == 0");
+    if (out_dtype == AQ_DTYPE_I8 && N % 16 != 0)
+      return set_error(AQ_ERR_SHAPE, "int8 output needs N %% 16 == 0");
     return AQ_OK;
   }
   if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
@@ -780,9 +787,9 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
               int B, void* workspace, size_t workspace_bytes, int path, void* stream,
-              const void* x16 = nullptr);
+              const void* x16 = nullptr, const void* xh = nullptr);
 int conv_ws(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
-            int M, int B, int path, bool a16, size_t* bytes);
+            int M, int B, int path, ActKind act, size_t* bytes);
 
 }  // namespace
 
@@ -1001,7 +1008,8 @@ int aq_linear(const int8_t* xq, float s_x, const void* codes_packed, const void*
               const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
               int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
               void* stream) {
-  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d: F16 or F32 (int8: aq_linear_q8; codes: aq_linear_ex)", out_dtype);
   return linear_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, T, K, N,
                      g, M, B, workspace, workspace_bytes, path, stream);
 }
@@ -1039,7 +1047,8 @@ int aq_linear_a16(const void* xh, float s_x, const void* codes_packed, const voi
                   const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
                   int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
                   void* stream) {
-  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d: F16 or F32 (int8: aq_linear_q8; codes: aq_linear_ex)", out_dtype);
   const int rp = resolve_a16_path(path);
   if (rp < 0) return path_error(-2, path);
   if (T > 0 && !xh) return set_error(AQ_ERR_NULL, "xh is NULL");
@@ -1052,7 +1061,8 @@ int aq_linear_f16(const void* x, float s_x, const void* codes_packed, const void
                   const void* scale, const void* bias, void* y, int out_dtype, int T, int K, int N,
                   int g, int M, int B, void* workspace, size_t workspace_bytes, int path,
                   void* stream) {
-  if (out_dtype == AQ_DTYPE_I8) return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_linear_q8");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED, "out_dtype %d: F16 or F32 (int8: aq_linear_q8; codes: aq_linear_ex)", out_dtype);
   if (!(s_x > 0.0f) || s_x == __builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite and > 0");
   if (T < 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and K > 0");
@@ -1135,7 +1145,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     sp.bias = static_cast<const __half*>(bias);
     sp.y = y;
     sp.out_f32 = out_dtype == AQ_DTYPE_F32;
-    sp.out_q8 = out_dtype == AQ_DTYPE_I8;
+    sp.out_q8 = out_codes(out_dtype);
     sp.s_x = s_x;
     sp.s_out = s_out;
     sp.T = T;
@@ -1182,7 +1192,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     rpar.bias = static_cast<const __half*>(bias);
     rpar.y = y;
     rpar.out_f32 = out_dtype == AQ_DTYPE_F32;
-    rpar.out_q8 = out_dtype == AQ_DTYPE_I8;
+    rpar.out_q8 = out_codes(out_dtype);
     rpar.s_out = s_out;
     rpar.partial = lpar.partial;
     {
@@ -1217,7 +1227,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  p.out_q8 = out_dtype == AQ_DTYPE_I8;
+  p.out_q8 = out_codes(out_dtype);
   p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st, false, x16,
                   const_cast<int8_t*>(xq), rt.predecoded);
@@ -1229,12 +1239,12 @@ extern "C" {
 
 int aq_conv2d_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
                              int pad, int g, int M, int B, int path, size_t* bytes) {
-  return conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, false, bytes);
+  return conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, kActInt8, bytes);
 }
 
 namespace {
 int conv_plan_impl(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
-                   int g, int M, int B, int path, bool a16, int* info, int n_info) {
+                   int g, int M, int B, int path, ActKind act, int* info, int n_info) {
   int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
@@ -1242,23 +1252,23 @@ int conv_plan_impl(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int 
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles, g);
+  const int rp = act == kActF16Codes ? resolve_a16_path(path) : resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
   const Route rt = route_layer(rp, Nb * cg.Ho * cg.Wo, Cout, kh * kw * Cin, cg.m_tiles, false, M,
-                               B, a16 ? kActF16 : kActInt8);
+                               B, act);
   return fill_plan_info(rp, &rt.pl, info, n_info);
 }
 }  // namespace
 
 int aq_conv2d_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
                    int g, int M, int B, int path, int* info, int n_info) {
-  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, false, info,
+  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, kActInt8, info,
                         n_info);
 }
 
 int aq_conv2d_f16_plan(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
                        int pad, int g, int M, int B, int path, int* info, int n_info) {
-  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, true, info,
+  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, kActF16, info,
                         n_info);
 }
 
@@ -1266,7 +1276,7 @@ int aq_conv2d_f16_workspace_size(int Nb, int H, int W, int Cin, int Cout, int kh
                                  int stride, int pad, int g, int M, int B, int path,
                                  size_t* bytes) {
   size_t rest = 0;
-  const int r = conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, true, &rest);
+  const int r = conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, kActF16, &rest);
   if (r) return r;
   *bytes = f16_act_bytes(Nb * H * W, Cin) + rest;
   return ok();
@@ -1277,8 +1287,10 @@ int aq_conv2d_nhwc_f16(const void* x, float s_x, const void* codes_packed, const
                        int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
                        int M, int B, void* workspace, size_t workspace_bytes, int path,
                        void* stream) {
-  if (out_dtype == AQ_DTYPE_I8)
-    return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_conv2d_nhwc_q8");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED,
+                     "out_dtype %d: F16 or F32 (int8: aq_conv2d_nhwc_q8; codes: aq_conv2d_nhwc_ex)",
+                     out_dtype);
   if (!(s_x > 0.0f) || s_x == __builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite and > 0");
   if (Nb < 0 || H <= 0 || W <= 0 || Cin <= 0)
@@ -1304,8 +1316,10 @@ int aq_conv2d_nhwc(const int8_t* xq, float s_x, const void* codes_packed, const 
                    const void* scale, const void* bias, void* y, int out_dtype, int Nb, int H,
                    int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
                    int B, void* workspace, size_t workspace_bytes, int path, void* stream) {
-  if (out_dtype == AQ_DTYPE_I8)
-    return set_error(AQ_ERR_UNSUPPORTED, "int8 output: aq_conv2d_nhwc_q8");
+  if (out_dtype != AQ_DTYPE_F16 && out_dtype != AQ_DTYPE_F32)
+    return set_error(AQ_ERR_UNSUPPORTED,
+                     "out_dtype %d: F16 or F32 (int8: aq_conv2d_nhwc_q8; codes: aq_conv2d_nhwc_ex)",
+                     out_dtype);
   return conv_impl(xq, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, 0.0f, Nb, H, W,
                    Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes, path,
                    stream);
@@ -1321,18 +1335,117 @@ int aq_conv2d_nhwc_q8(const int8_t* xq, float s_x, const void* codes_packed,
                    stream);
 }
 
+// ---- layer calls with the activation and output kinds as arguments: int8 codes or the codes
+// held as fp16 values in; fp16, fp32, int8 codes or fp16 codes out (so a chain of layers can
+// hand each layer its activations in the form its tensor-core plan reads).
+namespace {
+int act_kind(int act_dtype, ActKind* act) {
+  if (act_dtype == AQ_DTYPE_I8) {
+    *act = kActInt8;
+    return AQ_OK;
+  }
+  if (act_dtype == AQ_DTYPE_F16_CODES) {
+    *act = kActF16Codes;
+    return AQ_OK;
+  }
+  return set_error(AQ_ERR_UNSUPPORTED, "act_dtype %d: AQ_DTYPE_I8 or AQ_DTYPE_F16_CODES",
+                   act_dtype);
+}
+}  // namespace
+
+int aq_linear_ex_workspace_size(int act_dtype, int T, int K, int N, int g, int M, int B, int path,
+                                size_t* bytes) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  if (act == kActInt8) return linear_ws(T, K, N, g, M, B, path, kActInt8, bytes);
+  const int rp = resolve_a16_path(path);
+  if (rp < 0) return path_error(-2, path);
+  return linear_ws(T, K, N, g, M, B, rp, kActF16Codes, bytes);
+}
+
+int aq_linear_ex_plan(int act_dtype, int T, int K, int N, int g, int M, int B, int path, int* info,
+                      int n_info) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  return linear_plan_impl(T, K, N, g, M, B, path, act == kActF16Codes, act == kActF16Codes, info,
+                          n_info);
+}
+
+int aq_linear_ex(const void* act_in, int act_dtype, float s_x, const void* codes_packed,
+                 const void* codebooks, const void* scale, const void* bias, void* y,
+                 int out_dtype, float s_out, int T, int K, int N, int g, int M, int B,
+                 void* workspace, size_t workspace_bytes, int path, void* stream) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  if (act == kActInt8)
+    return linear_impl(static_cast<const int8_t*>(act_in), s_x, codes_packed, codebooks, scale,
+                       bias, y, out_dtype, s_out, T, K, N, g, M, B, workspace, workspace_bytes,
+                       path, stream);
+  const int rp = resolve_a16_path(path);
+  if (rp < 0) return path_error(-2, path);
+  if (T > 0 && !act_in) return set_error(AQ_ERR_NULL, "activations are NULL");
+  return linear_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, s_out, T,
+                     K, N, g, M, B, workspace, workspace_bytes, rp, stream, nullptr,
+                     T > 0 ? act_in : nullptr);
+}
+
+int aq_conv2d_ex_workspace_size(int act_dtype, int Nb, int H, int W, int Cin, int Cout, int kh,
+                                int kw, int stride, int pad, int g, int M, int B, int path,
+                                size_t* bytes) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  return conv_ws(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, act, bytes);
+}
+
+int aq_conv2d_ex_plan(int act_dtype, int Nb, int H, int W, int Cin, int Cout, int kh, int kw,
+                      int stride, int pad, int g, int M, int B, int path, int* info, int n_info) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  return conv_plan_impl(Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, path, act, info,
+                        n_info);
+}
+
+int aq_conv2d_nhwc_ex(const void* act_in, int act_dtype, float s_x, const void* codes_packed,
+                      const void* codebooks, const void* scale, const void* bias, void* y,
+                      int out_dtype, float s_out, int Nb, int H, int W, int Cin, int Cout, int kh,
+                      int kw, int stride, int pad, int g, int M, int B, void* workspace,
+                      size_t workspace_bytes, int path, void* stream) {
+  ActKind act;
+  int r = act_kind(act_dtype, &act);
+  if (r) return r;
+  if (act == kActInt8)
+    return conv_impl(static_cast<const int8_t*>(act_in), s_x, codes_packed, codebooks, scale, bias,
+                     y, out_dtype, s_out, Nb, H, W, Cin, Cout, kh, kw, stride, pad, g, M, B,
+                     workspace, workspace_bytes, path, stream);
+  if (Nb > 0 && !act_in) return set_error(AQ_ERR_NULL, "activations are NULL");
+  if (Nb == 0)  // argument checks only (the int8 form's, on a dense path)
+    return conv_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, s_out, 0,
+                     H, W, Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes,
+                     path == AQ_PATH_AUTO ? AQ_PATH_DENSE : path, stream);
+  return conv_impl(nullptr, s_x, codes_packed, codebooks, scale, bias, y, out_dtype, s_out, Nb, H,
+                   W, Cin, Cout, kh, kw, stride, pad, g, M, B, workspace, workspace_bytes, path,
+                   stream, nullptr, act_in);
+}
+
 }  // extern "C"
 
 namespace {
 
 // x16 != nullptr (aq_conv2d_nhwc_f16): the fp16 NHWC activations, quantized into xq by this
-// call -- on the dense paths as the codes' fp16 values (the region holds Nb*H*W*Cin*2 bytes)
-// read by the shared-memory A form of the GEMM, else as int8 codes.
+// call -- as the codes' fp16 values (the region holds Nb*H*W*Cin*2 bytes) when the
+// shared-memory A form runs (route_layer), else as int8 codes.
+// xh != nullptr (aq_conv2d_nhwc_ex with AQ_DTYPE_F16_CODES): the codes already held as fp16
+// values; the path resolves to a dense one and xq is unused.
 int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void* codebooks,
               const void* scale, const void* bias, void* y, int out_dtype, float s_out, int Nb,
               int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g, int M,
               int B, void* workspace, size_t workspace_bytes, int path, void* stream,
-              const void* x16) {
+              const void* x16, const void* xh) {
   int r = check_format(g, M, B, true);
   if (r) return r;
   r = check_conv_args(Nb, H, W, Cin, Cout, kh, kw, stride, pad);
@@ -1344,18 +1457,20 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles, g);
+  const int rp = xh ? resolve_a16_path(path) : resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
   if (Nb == 0) return ok();
-  if (!xq || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
-  if (!aligned16(xq) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
+  const void* act = xh ? xh : static_cast<const void*>(xq);
+  if (!act || !codes_packed || !codebooks || !scale || !y) return set_error(AQ_ERR_NULL, "NULL argument");
+  if (!aligned16(act) || !aligned16(codes_packed) || !aligned16(codebooks) || !aligned16(scale) ||
       !aligned16(y) || (bias && !aligned16(bias)))
     return set_error(AQ_ERR_ALIGN, "buffers must be 16-byte aligned");
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  // fp16 activations quantized by this call may run the shared-memory A form (route_layer)
+  // fp16 activations (given as codes, or quantized by this call) may run the shared-memory A
+  // form (route_layer)
   const Route rt = route_layer(rp, T, Cout, K, cg.m_tiles, out_dtype == AQ_DTYPE_F32, M, B,
-                               x16 ? kActF16 : kActInt8);
+                               xh ? kActF16Codes : (x16 ? kActF16 : kActInt8));
   const bool a16 = rt.pl.a16 != 0;
   r = check_workspace(workspace, workspace_bytes, rt.ws);
   if (r) return r;
@@ -1375,9 +1490,9 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
     cuuint32_t box[4] = {static_cast<cuuint32_t>(aq::kBK), static_cast<cuuint32_t>(stride * cg.bw),
                          static_cast<cuuint32_t>(stride * cg.bh), static_cast<cuuint32_t>(cg.bn)};
     cuuint32_t es[4] = {1, static_cast<cuuint32_t>(stride), static_cast<cuuint32_t>(stride), 1};
-    r = encode(&mapA, a16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, xq,
-               dims, strides, box, a16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
-               es);
+    r = encode(&mapA, a16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4,
+               act, dims, strides, box,
+               a16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, es);
     if (r) return r;
   }
   aq::GemmParams p{};
@@ -1396,7 +1511,7 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
   p.bias = static_cast<const __half*>(bias);
   p.y = y;
   p.out_f32 = out_dtype == AQ_DTYPE_F32;
-  p.out_q8 = out_dtype == AQ_DTYPE_I8;
+  p.out_q8 = out_codes(out_dtype);
   p.s_out = s_out;
   return run_gemm(mapA, p, rt.pl, codes_packed, codebooks, M, B, Wdec, partial, st,
                   g == kKaqGroup, x16, const_cast<int8_t*>(xq), rt.predecoded,
@@ -1404,7 +1519,7 @@ int conv_impl(const int8_t* xq, float s_x, const void* codes_packed, const void*
 }
 
 int conv_ws(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int g,
-            int M, int B, int path, bool a16, size_t* bytes) {
+            int M, int B, int path, ActKind act, size_t* bytes) {
   if (!bytes) return set_error(AQ_ERR_NULL, "bytes is NULL");
   int r = check_format(g, M, B, true);
   if (r) return r;
@@ -1413,11 +1528,11 @@ int conv_ws(int Nb, int H, int W, int Cin, int Cout, int kh, int kw, int stride,
   ConvGeom cg;
   r = conv_geometry(Nb, H, W, kh, kw, stride, pad, &cg);
   if (r) return r;
-  const int rp = resolve_conv_path(path, cg.m_tiles, g);
+  const int rp = act == kActF16Codes ? resolve_a16_path(path) : resolve_conv_path(path, cg.m_tiles, g);
   if (rp < 0) return path_error(rp, path);
   const int K = kh * kw * Cin;
   const int T = Nb * cg.Ho * cg.Wo;
-  *bytes = route_layer(rp, T, Cout, K, cg.m_tiles, false, M, B, a16 ? kActF16 : kActInt8).ws;
+  *bytes = route_layer(rp, T, Cout, K, cg.m_tiles, false, M, B, act).ws;
   return ok();
 }
 

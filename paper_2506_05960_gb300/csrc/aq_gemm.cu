@@ -314,7 +314,13 @@ __device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n
     for (int e = 0; e < 4; ++e)
       b |= static_cast<uint32_t>(static_cast<uint8_t>(quant_one(__float2half_rn(o[e]), p.s_out, rs)))
            << (8 * e);
-    *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(p.y) + t * p.N + n) = b;
+    if (p.out_q8 == kOutCodesF16) {
+      uint32_t lo, hi;
+      i8x4_to_f16x4(b, lo, hi);
+      *reinterpret_cast<uint2*>(static_cast<__half*>(p.y) + t * p.N + n) = make_uint2(lo, hi);
+    } else {
+      *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(p.y) + t * p.N + n) = b;
+    }
   } else {
     __half2 a = __floats2half2_rn(o[0], o[1]);
     __half2 b = __floats2half2_rn(o[2], o[3]);
@@ -784,9 +790,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int jj = 0; jj < 4; ++jj)
               wq[4 * hf + jj] = pack_low_bytes(qb[4 * jj], qb[4 * jj + 1], qb[4 * jj + 2], qb[4 * jj + 3]);
           }
-          uint4* row = reinterpret_cast<uint4*>(dst + lane * 32);
-          row[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
-          row[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
+          if (p.out_q8 == kOutCodesF16) {
+            // the codes as fp16 values (exact), staged like the fp16 output: 16-byte piece j
+            // holds columns 8j .. 8j+7
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              uint32_t f0, f1, f2, f3;
+              i8x4_to_f16x4(wq[2 * j], f0, f1);
+              i8x4_to_f16x4(wq[2 * j + 1], f2, f3);
+              *reinterpret_cast<uint4*>(dst + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                  make_uint4(f0, f1, f2, f3);
+            }
+          } else {
+            uint4* row = reinterpret_cast<uint4*>(dst + lane * 32);
+            row[0] = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+            row[1] = make_uint4(wq[4], wq[5], wq[6], wq[7]);
+          }
         } else {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {

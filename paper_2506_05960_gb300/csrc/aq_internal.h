@@ -17,6 +17,10 @@ constexpr int kBK = 64;         // K per TMA box / swizzle row (128 bytes of fp1
 constexpr int kStageBlocks = 2; // 64-wide K blocks per pipeline stage (8 MMAs of K = 16)
 constexpr int kMaxBN = 256;     // widest N tile: 2 fp32 accumulators in TMEM
 constexpr int kA8MaxBN = 192;   // the TMEM-A form also needs >= 2 A slots beside them
+// GemmParams::out_q8 / SkinnyParams::out_q8: 0 (fp16 or fp32 output), or the 8-bit activation
+// rule applied to the fp16-rounded output and stored as int8 codes or as their fp16 values
+constexpr int kOutCodesI8 = 1;
+constexpr int kOutCodesF16 = 2;
 constexpr int kMaxStages = 8;   // pipeline ring depth bound
 constexpr int kMaxClusterSplits = 8;  // K splits summed inside one cluster (portable size)
 
@@ -52,7 +56,8 @@ struct GemmParams {
   const __half* bias;           // may be null
   void* y;
   int out_f32;
-  int out_q8;                   // int8 output: the next layer's activations, quantized with s_out
+  int out_q8;                   // the next layer's activations, quantized with s_out: int8
+                                // codes (kOutCodesI8) or the codes as fp16 values (kOutCodesF16)
   float s_out;
   float* partial;               // split-K partial sums [splits][T][N] (null: fused epilogue)
   int epi_warps;                // epilogue warps: 4, or 8 on the dense path (BN >= 64)
@@ -90,7 +95,7 @@ struct SkinnyParams {
   const __half* scale;
   const __half* bias;           // may be null
   void* y;                      // [T][N]
-  int out_f32, out_q8;
+  int out_f32, out_q8;          // out_q8: as GemmParams::out_q8
   float s_x, s_out;
   int T, K, N, M, B;
   int sms;                      // SMs of the device (the caller's count; sizes the grid)

@@ -193,6 +193,9 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
       const int64_t off = static_cast<int64_t>(t) * N + nn;
       if (p.out_f32)
         static_cast<float*>(p.y)[off] = v;
+      else if (p.out_q8 == kOutCodesF16)
+        static_cast<__half*>(p.y)[off] =
+            __short2half_rn(quant_one(__float2half_rn(v), p.s_out, rs_out));
       else if (p.out_q8)
         static_cast<int8_t*>(p.y)[off] = quant_one(__float2half_rn(v), p.s_out, rs_out);
       else
@@ -302,6 +305,9 @@ __global__ void __launch_bounds__(256, 2) skinny_gather_kernel(const SkinnyParam
     const int64_t off = static_cast<int64_t>(t) * p.N + n;
     if (p.out_f32)
       static_cast<float*>(p.y)[off] = v;
+    else if (p.out_q8 == kOutCodesF16)
+      static_cast<__half*>(p.y)[off] =
+          __short2half_rn(quant_one(__float2half_rn(v), p.s_out, rs_out));
     else if (p.out_q8)
       static_cast<int8_t*>(p.y)[off] = quant_one(__float2half_rn(v), p.s_out, rs_out);
     else
