@@ -410,6 +410,24 @@ class Dev:
                             self.yq, s_out, self.T, self.K, self.N, 8, self.M, self.B, ws_t,
                             ws_t.numel(), path, stream=st)
 
+    def layer_ex(self, st, path=None, ws=None, s_out=0.02):
+        """The layer through aq_*_ex: activations in self.in_kind (int8 codes self.xq, or fp16
+        codes self.xh), output in self.out_kind (the next layer's codes, scale s_out) into
+        self.yc; `ws` replaces the layer's workspace (e.g. one holding decoded weights)."""
+        aq, s = self.aq, self.spec
+        path = self.path if path is None else path
+        ws_t = self.ws if ws is None else ws
+        act = self.xh if self.in_kind == aq.AQ_DTYPE_F16_CODES else self.xq
+        if self.conv:
+            aq.aq_conv2d_nhwc_ex(act, self.in_kind, self.s_x, self.packed, self.books, self.scale,
+                                 self.bias, self.yc, self.out_kind, s_out, s.Nb, s.H, s.W, s.Cin,
+                                 s.Cout, 3, 3, s.stride, 1, 8, self.M, self.B, ws_t, ws_t.numel(),
+                                 path, stream=st)
+        else:
+            aq.aq_linear_ex(act, self.in_kind, self.s_x, self.packed, self.books, self.scale,
+                            self.bias, self.yc, self.out_kind, s_out, self.T, self.K, self.N, 8,
+                            self.M, self.B, ws_t, ws_t.numel(), path, stream=st)
+
     def gemm_a16(self, st, xh, ws):
         """The tensor-core GEMM alone: fp16 activations xh (the 8-bit codes as fp16 values) and
         weights decoded beforehand into ws (AQ_PATH_PREDECODED)."""
@@ -456,13 +474,16 @@ def replay_ms(torch, stream, g, reps):
 
 
 def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
-                 decode_ahead=False):
+                 decode_ahead=False, mixed=False):
     """One UNet-shaped forward: every AQ layer of the LDM-4-like sweep, captured as one
     graph.  Each layer is preceded by its activation quantizer (aq_quant_act), or, with
     fused_quant, writes int8 output through its _q8 epilogue instead (the chain of
-    layers then has no separate quantizer pass).  Above batch 2 the int8 activations
-    are drawn on the device (seeded torch generator) and the host arrays only supply
-    the weights.  Returns (ms, GFLOP, layers)."""
+    layers then has no separate quantizer pass).  With mixed (and fused_quant), each layer
+    takes its activations in the form its own plan reads faster -- the codes as fp16 values
+    where the shared-memory A form wins (aq_*_f16_plan), else int8 -- and the layer before it
+    writes that form (aq_*_ex).  Above batch 2 the int8 activations are drawn on the device
+    (seeded torch generator) and the host arrays only supply the weights.
+    Returns (ms, GFLOP, layers)."""
     from aq_synth import ConvSpec, LinearSpec, make_conv, make_linear, unet_sweep_layers
     layers = []
     seed = 4000 + 100 * M
@@ -509,6 +530,29 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
     # Every weight is still decoded once per forward; each such layer then needs its decoded
     # weights resident until it runs (here: one workspace per layer).
     side = torch.cuda.Stream(device=dev) if decode_ahead else None
+    F16C, I8 = aq.AQ_DTYPE_F16_CODES, aq.AQ_DTYPE_I8
+    for i, L in enumerate(layers):
+        L.in_kind = I8
+        if mixed:
+            s = L.spec
+            pf = (aq.aq_conv2d_f16_plan(s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3, s.stride, 1, 8, L.M,
+                                        L.B, L.path) if L.conv
+                  else aq.aq_linear_f16_plan(L.T, L.K, L.N, 8, L.M, L.B, L.path))
+            L.in_kind = F16C if pf["a16"] else I8
+    for i, L in enumerate(layers):
+        L.out_kind = layers[i + 1].in_kind if i + 1 < len(layers) else I8
+        if mixed:
+            L.yc = torch.empty(tuple(L.y.shape),
+                               dtype=torch.float16 if L.out_kind == F16C else torch.int8,
+                               device=dev)
+            if L.in_kind == F16C:
+                s = L.spec
+                nb = (aq.aq_conv2d_ex_workspace_size(F16C, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
+                                                     s.stride, 1, 8, L.M, L.B, L.path)
+                      if L.conv else
+                      aq.aq_linear_ex_workspace_size(F16C, L.T, L.K, L.N, 8, L.M, L.B, L.path))
+                if nb > L.ws.numel():
+                    L.ws = torch.empty(nb, dtype=torch.uint8, device=dev)
     for L in layers:
         L.dense = False
         L.ws_pre = L.ws
@@ -526,6 +570,16 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
                       aq.aq_linear_workspace_size(L.T, L.K, L.N, 8, L.M, L.B,
                                                   aq.AQ_PATH_PREDECODED))
                 L.ws_pre = torch.empty(nb, dtype=torch.uint8, device=dev)
+            if L.dense and L.in_kind == F16C:
+                # the fp16-code form's plan may split K differently: room for its partials too
+                nb16 = (aq.aq_conv2d_ex_workspace_size(F16C, s.Nb, s.H, s.W, s.Cin, s.Cout, 3, 3,
+                                                       s.stride, 1, 8, L.M, L.B,
+                                                       aq.AQ_PATH_PREDECODED)
+                        if L.conv else
+                        aq.aq_linear_ex_workspace_size(F16C, L.T, L.K, L.N, 8, L.M, L.B,
+                                                       aq.AQ_PATH_PREDECODED))
+                if nb16 > L.ws_pre.numel():
+                    L.ws_pre = torch.empty(nb16, dtype=torch.uint8, device=dev)
 
     def fwd():
         if decode_ahead:
@@ -544,11 +598,17 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
             for L, e in zip(layers, ready):
                 if e is not None:
                     stream.wait_event(e)
-                L.layer_q8(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None,
-                           ws=L.ws_pre)
+                if mixed:
+                    L.layer_ex(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None,
+                               ws=L.ws_pre)
+                else:
+                    L.layer_q8(stream, path=aq.AQ_PATH_PREDECODED if L.dense else None,
+                               ws=L.ws_pre)
             return
         for L in layers:
-            if fused_quant:
+            if mixed:
+                L.layer_ex(stream)
+            elif fused_quant:
                 L.layer_q8(stream)
             else:
                 L.step(stream)
@@ -556,6 +616,8 @@ def unet_forward(aq, torch, dev, stream, M, batch=2, reps=20, fused_quant=False,
     with torch.cuda.stream(stream):
         for L in layers:
             L.quant(stream)          # int8 inputs for the fused-quantizer chain
+            if L.in_kind == F16C:
+                L.xh = L.xq.to(torch.float16)   # the same codes as fp16 values
         for _ in range(2):
             fwd()
     stream.synchronize()
@@ -1082,15 +1144,21 @@ def main():
         unet = {}
         for Mu, label in ((2, "W2A8"), (4, "W4A8")):
             for batch in [int(b) for b in args.unet_batches.split(",") if b]:
-                for fq, ahead in ((False, False), (True, False), (True, True)):
+                for fq, ahead, mixed in ((False, False, False), (True, False, False),
+                                         (True, True, False), (True, True, True)):
                     ms, gflop, nl = unet_forward(aq, torch, dev, stream, Mu, batch=batch,
                                                  reps=20 if batch <= 2 else 5, fused_quant=fq,
-                                                 decode_ahead=ahead)
+                                                 decode_ahead=ahead, mixed=mixed)
                     key = (f"{label} batch {batch}" + (" quantizer in epilogue" if fq else "")
-                           + (", decode ahead" if ahead else ""))
+                           + (", decode ahead" if ahead else "")
+                           + (", fp16 codes into the layers whose plan prefers them"
+                              if mixed else ""))
                     unet[key] = {"ms_per_forward": ms, "gflop": gflop, "tflops": gflop / ms,
                                  "layers": nl, "batch": batch,
-                                 "step": ("each layer writes the next layer's int8 activations"
+                                 "step": ("each layer writes the next layer's activation codes "
+                                          "(int8, or fp16 values where that layer's plan reads "
+                                          "them faster)" if mixed else
+                                          "each layer writes the next layer's int8 activations"
                                           if fq else "each layer preceded by aq_quant_act")
                                          + ("; dense-path layers decoded on a second stream "
                                             "ahead of the chain (AQ_PATH_PREDECODED)"
