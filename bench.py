@@ -59,12 +59,11 @@ NSETS = 8
 # DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from
 # `ncu --set full` capture of one launch (dram__bytes_read.sum + dram__bytes_write.sum;
 # summary in profiles/aq_gemm_kernel_a16_qkv_T4096_K960_N2880.md); reported only while the
-# kernel sources are the ones it was measured on (the key was refreshed after changes -- a
-# header declaration, a named constant -- that left the GEMM's compiled code byte-identical
-# apart from line information).
+# kernel sources are the ones it was measured on (re-captured with the fp16-code epilogue
+# branch: dram__bytes_read.sum + dram__bytes_write.sum of one launch).
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 13475584, "sources_sha": "43ab19d5b4821bef"}
+TRAFFIC = {"bytes": 13476096, "sources_sha": "eca79d81de8e5887"}
 
 
 def sources_sha() -> str:
