@@ -99,6 +99,7 @@ struct SkinnyParams {
   float s_x, s_out;
   int T, K, N, M, B;
   int sms;                      // SMs of the device (the caller's count; sizes the grid)
+  int x_smem;                   // set by the launcher: activations staged in shared memory
 };
 
 // Launch with programmatic stream serialization (the kernel must call

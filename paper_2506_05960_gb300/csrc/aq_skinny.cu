@@ -34,6 +34,7 @@ namespace aq {
 constexpr int kSkinnyRows = 8;    // output rows per row block (lane / 4)
 constexpr int kSkinnyWarps = 8;   // warps per CTA; they split the K blocks
 constexpr int kSkinnyUnroll = 4;  // K blocks per warp whose code loads are in flight together
+constexpr int kSkinnyXsBytes = 32 * 1024;  // activations staged in shared memory up to this size
 
 // 16 int8 (one uint4) -> 16 floats
 __device__ __forceinline__ void i8x16_to_f32(uint4 v, float (&x)[16]) {
@@ -113,6 +114,10 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
   const int R = fused_book_copies(M);
   uint4* sbook = reinterpret_cast<uint4*>(skinny_smem4);                   // [M*256][R]
   float* wred = reinterpret_cast<float*>(skinny_smem4) + M * 256 * R * 4;
+  // the activations as fp16 (exact for |x| <= 127), [T][K], when p.x_smem: every lane of a
+  // row block reads them with broadcast loads instead of converting the same int8 values
+  __half* xs = p.x_smem ? reinterpret_cast<__half*>(wred + kSkinnyWarps * kSkinnyRows * TT)
+                        : nullptr;
   grid_dependency_wait();
   allow_dependents();
   const uint4* gbook = static_cast<const uint4*>(p.books);
@@ -120,6 +125,17 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
   for (int i = threadIdx.x; i < M * 256; i += blockDim.x) {
     const uint4 v = gbook[i];
     for (int r = 0; r < R; ++r) sbook[i * R + ((r + i) & (R - 1))] = v;
+  }
+  if (xs) {
+    // 8 activations (8 bytes, K % 16 == 0 keeps them inside one row) per thread and step
+    const int n8 = p.T * p.K / 8;
+    for (int i = threadIdx.x; i < n8; i += blockDim.x) {
+      const uint2 v = reinterpret_cast<const uint2*>(p.xq)[i];
+      uint32_t h0, h1, h2, h3;
+      i8x4_to_f16x4(v.x, h0, h1);
+      i8x4_to_f16x4(v.y, h2, h3);
+      reinterpret_cast<uint4*>(xs)[i] = make_uint4(h0, h1, h2, h3);
+    }
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -165,7 +181,23 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
           for (int t = 0; t < TT; ++t) {
             if (t < T) {
               float x[16];
-              i8x16_to_f32(__ldg(reinterpret_cast<const uint4*>(p.xq + static_cast<int64_t>(t) * K + k0)), x);
+              if (xs) {
+                const uint4* xp = reinterpret_cast<const uint4*>(xs + t * K + k0);
+                const uint4 a = xp[0], b = xp[1];
+                const __half2* ha = reinterpret_cast<const __half2*>(&a);
+                const __half2* hb = reinterpret_cast<const __half2*>(&b);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  const float2 fa = __half22float2(ha[i]);
+                  const float2 fb = __half22float2(hb[i]);
+                  x[2 * i] = fa.x;
+                  x[2 * i + 1] = fa.y;
+                  x[8 + 2 * i] = fb.x;
+                  x[8 + 2 * i + 1] = fb.y;
+                }
+              } else {
+                i8x16_to_f32(__ldg(reinterpret_cast<const uint4*>(p.xq + static_cast<int64_t>(t) * K + k0)), x);
+              }
 #pragma unroll
               for (int e = 0; e < 16; ++e) acc[t] = fmaf(w[e], x[e], acc[t]);
             }
@@ -317,10 +349,20 @@ __global__ void __launch_bounds__(256, 2) skinny_gather_kernel(const SkinnyParam
 
 static int skinny_tt(int T) { return T <= 1 ? 1 : T <= 2 ? 2 : T <= 4 ? 4 : T <= 8 ? 8 : 16; }
 
-// 8-bit codes (the row-block kernel): codebook copies + the warps' partial sums
-size_t skinny_smem_bytes(int M, int T) {
+// Activations staged in shared memory as fp16 from two tokens on, when T * K * 2 bytes fit
+// kSkinnyXsBytes.  Measured on GB300 (K = 8192, N = 16384, 2x8): T = 2 77.3 -> 62.4 us; at
+// T = 1 the conversions it saves are fewer than the occupancy it costs (45.2 -> 50.2 us:
+// 2 instead of 3 CTAs per SM), so one token keeps converting from global memory.
+static bool skinny_x_smem(int T, int K) {
+  return T >= 2 && static_cast<size_t>(T) * K * 2 <= static_cast<size_t>(kSkinnyXsBytes);
+}
+
+// 8-bit codes (the row-block kernel): codebook copies + the warps' partial sums (+ the
+// activations as fp16)
+size_t skinny_smem_bytes(int M, int T, int K) {
   return static_cast<size_t>(M) * 256 * 16 * fused_book_copies(M) +
-         static_cast<size_t>(kSkinnyWarps) * kSkinnyRows * skinny_tt(T) * 4;
+         static_cast<size_t>(kSkinnyWarps) * kSkinnyRows * skinny_tt(T) * 4 +
+         (skinny_x_smem(T, K) ? static_cast<size_t>(T) * K * 2 : 0);
 }
 
 template <int MM>
@@ -369,7 +411,8 @@ cudaError_t launch_skinny_gather(const SkinnyParams& p, cudaStream_t st) {
 
 cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st) {
   if (p.B == 16) return launch_skinny_gather(p, st);
-  const size_t smem = skinny_smem_bytes(p.M, p.T);
+  p.x_smem = skinny_x_smem(p.T, p.K) ? 1 : 0;
+  const size_t smem = skinny_smem_bytes(p.M, p.T, p.K);
   if (p.M == 1) return launch_skinny_m<1>(p, smem, st);
   if (p.M == 2) return launch_skinny_m<2>(p, smem, st);
   return launch_skinny_m<0>(p, smem, st);
