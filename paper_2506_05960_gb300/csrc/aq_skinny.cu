@@ -116,8 +116,10 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
   float* wred = reinterpret_cast<float*>(skinny_smem4) + M * 256 * R * 4;
   // the activations as fp16 (exact for |x| <= 127), [T][K], when p.x_smem: every lane of a
   // row block reads them with broadcast loads instead of converting the same int8 values
-  __half* xs = p.x_smem ? reinterpret_cast<__half*>(wred + kSkinnyWarps * kSkinnyRows * TT)
-                        : nullptr;
+  // (one token never stages them: TT == 1 compiles the branch out of the inner loop)
+  __half* xs = (TT >= 2 && p.x_smem)
+                   ? reinterpret_cast<__half*>(wred + kSkinnyWarps * kSkinnyRows * TT)
+                   : nullptr;
   grid_dependency_wait();
   allow_dependents();
   const uint4* gbook = static_cast<const uint4*>(p.books);
@@ -126,7 +128,7 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
     const uint4 v = gbook[i];
     for (int r = 0; r < R; ++r) sbook[i * R + ((r + i) & (R - 1))] = v;
   }
-  if (xs) {
+  if (TT >= 2 && xs) {
     // 8 activations (8 bytes, K % 16 == 0 keeps them inside one row) per thread and step
     const int n8 = p.T * p.K / 8;
     for (int i = threadIdx.x; i < n8; i += blockDim.x) {
@@ -181,7 +183,7 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) skinny_kernel(const SkinnyP
           for (int t = 0; t < TT; ++t) {
             if (t < T) {
               float x[16];
-              if (xs) {
+              if (TT >= 2 && xs) {
                 const uint4* xp = reinterpret_cast<const uint4*>(xs + t * K + k0);
                 const uint4 a = xp[0], b = xp[1];
                 const __half2* ha = reinterpret_cast<const __half2*>(&a);
