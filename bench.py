@@ -1122,11 +1122,13 @@ def main():
                                   "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
                                   "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
                     del gs, Ls
-        # the few-token path on a layer large enough to amortise its launch: how fast it
-        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes)
-        for Ts in (1, 4):
+        # few tokens on a layer large enough to amortise the launches: how fast each path
+        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes); AUTO takes the one-token
+        # table kernel at T = 1
+        for Ts, pth in ((1, aq.AQ_PATH_FEW_TOKENS), (1, aq.AQ_PATH_AUTO), (4, aq.AQ_PATH_FEW_TOKENS),
+                        (4, aq.AQ_PATH_FUSED)):
             inp_s = _mlin(LinearSpec(T=Ts, K=8192, N=16384, M=2, B=8), seed=90 + Ts)
-            Ls = [Dev(aq, torch, inp_s, dev, path=aq.AQ_PATH_FEW_TOKENS) for _ in range(4)]
+            Ls = [Dev(aq, torch, inp_s, dev, path=pth) for _ in range(4)]
             with torch.cuda.stream(stream):
                 for L in Ls:
                     L.step(stream)
@@ -1134,7 +1136,9 @@ def main():
             gs = capture(torch, stream, lambda: [L.layer(stream) for L in Ls])
             ms = replay_ms(torch, stream, gs, 10) / len(Ls)
             wbytes = alg_bytes(Ts, 8192, 16384, 2, 8)
-            sweep[f"K=8192 N=16384 2x8 T={Ts} FEW (layer only, 4 rotating buffer sets)"] = {
+            pname = {aq.AQ_PATH_FEW_TOKENS: "FEW", aq.AQ_PATH_AUTO: "AUTO (table)",
+                     aq.AQ_PATH_FUSED: "FUSED"}[pth]
+            sweep[f"K=8192 N=16384 2x8 T={Ts} {pname} (layer only, 4 rotating buffer sets)"] = {
                 "us_per_step": ms * 1e3, "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
                 "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
             del gs, Ls

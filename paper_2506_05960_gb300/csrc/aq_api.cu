@@ -356,6 +356,22 @@ struct LutPlan {
 
 LutPlan plan_lut(int T, int K, int N, int M) {
   LutPlan lp{};
+  if (T == 1) {
+    // one token: one fp32 per table entry, chunks of whole packed K blocks with tables of at
+    // most 64 KB (8 K blocks for one codebook, 4 for two, 2 for three or four, else 1), over
+    // (chunk, row slice) CTAs
+    lp.Tp = 1;
+    lp.J = 8 * (M == 1 ? 8 : (M == 2 ? 4 : (M <= 4 ? 2 : 1)));
+    const int G = K / 8;
+    lp.chunks = (G + lp.J - 1) / lp.J;
+    // (as many row slices as keep chunks x slices within one wave of three CTAs per SM: a
+    // second, nearly empty wave would double the time)
+    int n_slices = 3 * kPlanSMs / lp.chunks;
+    if (n_slices < 1) n_slices = 1;
+    lp.rows_per_cta = ((N + n_slices - 1) / n_slices + 31) / 32 * 32;
+    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * N * 4, 1024);
+    return lp;
+  }
   lp.Tp = T <= 4 ? 4 : (T <= 8 ? 8 : 16);
   lp.J = 8;
   while (lp.J > 1 && static_cast<size_t>(lp.J) * M * 256 * lp.Tp * 4 > 160 * 1024) lp.J >>= 1;
@@ -375,10 +391,18 @@ constexpr int kFewTokensMaxT = 16;
 constexpr int kFewTokensAutoMaxT = 4;
 
 // AUTO / explicit path of a linear layer: -1 unknown path, -2 path cannot run this layer.
-int resolve_linear_path(int path, int T, int B) {
+// AUTO takes the one-token table kernel (lut1_kernel) from this many bytes of 8-bit codes:
+// measured on GB300 against the few-token kernel (2x8 codebooks, us, few-token / table):
+// 8.4 MB 12.3 / 16.4, 16.8 MB (1x8) 33.4 / 20.3, 33.6 MB 45.0 / 29.2, 67.1 MB (4x8) 198 / 48.
+constexpr size_t kLut1AutoMinCodeBytes = 12u << 20;
+
+int resolve_linear_path(int path, int T, int B, int N = 0, int K = 0, int M = 0) {
   const int m_tiles = (T + aq::kBM - 1) / aq::kBM;
   switch (path) {
     case AQ_PATH_AUTO:
+      if (T == 1 && B == 8 &&
+          static_cast<size_t>(N) * (K / 8) * M >= kLut1AutoMinCodeBytes)
+        return AQ_PATH_LUT;
       if (T <= kFewTokensAutoMaxT) return AQ_PATH_FEW_TOKENS;
       return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
     case AQ_PATH_FEW_TOKENS:
@@ -976,7 +1000,7 @@ int linear_plan_impl(int T, int K, int N, int g, int M, int B, int path, bool a1
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  const int rp = a16_only ? resolve_a16_path(path) : resolve_linear_path(path, T, B);
+  const int rp = a16_only ? resolve_a16_path(path) : resolve_linear_path(path, T, B, N, K, M);
   if (rp < 0) return path_error(rp, path);
   if (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT) return fill_plan_info(rp, nullptr, info, n_info);
   const Route rt = route_layer(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B,
@@ -1091,7 +1115,7 @@ int linear_ws(int T, int K, int N, int g, int M, int B, int path, ActKind act, s
   if (r) return r;
   if (T < 0 || N <= 0 || K <= 0) return set_error(AQ_ERR_SHAPE, "need T >= 0 and N, K > 0");
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
-  const int rp = resolve_linear_path(path, T, B);
+  const int rp = resolve_linear_path(path, T, B, N, K, M);
   if (rp < 0) return path_error(rp, path);
   if (rp == AQ_PATH_FEW_TOKENS) {
     *bytes = 0;
@@ -1121,7 +1145,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
   if (r) return r;
   if (!(s_x == s_x) || s_x == __builtin_inff() || s_x == -__builtin_inff())
     return set_error(AQ_ERR_SHAPE, "s_x must be finite");
-  const int rp = resolve_linear_path(path, T, B);
+  const int rp = resolve_linear_path(path, T, B, N, K, M);
   if (rp < 0) return path_error(rp, path);
   if (T == 0) return ok();
   const void* act = xh ? xh : static_cast<const void*>(xq);

@@ -81,8 +81,9 @@ struct LutParams {
   const __half* books;          // [M][256][8]
   float* partial;               // [chunks][T][N] partial sums
   int T, K, N, M;
-  int Tp;                       // T rounded up to 4, 8 or 16 (floats per table entry)
-  int J;                        // groups per chunk (divides 8)
+  int Tp;                       // floats per table entry: 1 (one token: lut1_kernel), or T
+                                // rounded up to 4, 8 or 16
+  int J;                        // groups per chunk (divides 8; Tp == 1: whole K blocks)
   int G;                        // K / 8
   int chunks, rows_per_cta;
 };

@@ -113,11 +113,132 @@ __global__ void __launch_bounds__(256) lut_kernel(const LutParams p) {
   }
 }
 
+// One token (Tp == 1): the same order with one fp32 per table entry.  A chunk is J groups =
+// J / 8 whole packed K blocks, its tables J * M * 256 floats (<= 64 KB).  One thread per output
+// row: per K block it reads the row's 8 * M codes as M contiguous 8-byte pieces (consecutive
+// rows consecutive, so a warp's loads are coalesced) and adds one table entry per code, in
+// the fixed order (K block, group, codebook).  MM: M when 1, 2 or 4 (index arithmetic known
+// at compile time), else 0.
+template <int MM>
+__global__ void __launch_bounds__(256) lut1_kernel(const LutParams p) {
+  extern __shared__ float4 lut_smem4[];
+  float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256]
+  const int J = p.J, M = MM > 0 ? MM : p.M;
+  float* xs = L + static_cast<size_t>(J) * M * 256;            // [J * 8]
+  grid_dependency_wait();
+  allow_dependents();
+  const int chunk = blockIdx.x;
+  const int g0 = chunk * J;
+  const int nj = min(J, p.G - g0);
+  for (int i = threadIdx.x; i < J * 8; i += blockDim.x)
+    xs[i] = (i < nj * 8) ? static_cast<float>(p.xq[g0 * 8 + i]) : 0.0f;
+  __syncthreads();
+  // build: L[j][m][c] = sum_e x[g0 + j][e] * C^(m)[c][e], ascending e (zero past the last group)
+  const int entries = J * M * 256;
+  for (int ent = threadIdx.x; ent < entries; ent += blockDim.x) {
+    const int j = ent / (M * 256);
+    const int r = ent - j * (M * 256);
+    const uint4 raw = reinterpret_cast<const uint4*>(p.books)[r];
+    const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+    const float* xr = xs + j * 8;
+    float s = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __half22float2(h2[i]);
+      s = fmaf(xr[2 * i], f.x, s);
+      s = fmaf(xr[2 * i + 1], f.y, s);
+    }
+    L[ent] = s;
+  }
+  __syncthreads();
+  const int kb0 = g0 >> 3;
+  const int nkb = (nj + 7) >> 3;                  // packed K blocks holding this chunk's groups
+  const int n_begin = blockIdx.y * p.rows_per_cta;
+  const int n_end = min(p.N, n_begin + p.rows_per_cta);
+  if constexpr (MM > 0) {
+    // one, two or four codebooks: a chunk is 8 / MM K blocks, so a row's codes in it are always
+    // eight 8-byte pieces; all eight are loaded at once, and the next row's while this row's
+    // entries are summed (the code stream's latency overlaps the lookups)
+    constexpr int kBlocks = 8 / MM;
+    auto load = [&](int n, uint2 (&v)[8]) {
+#pragma unroll
+      for (int b = 0; b < kBlocks; ++b) {
+        const uint2* rec = reinterpret_cast<const uint2*>(
+            p.packed + (static_cast<int64_t>(kb0 + b) * p.N + n) * 8 * MM);
+#pragma unroll
+        for (int pc = 0; pc < MM; ++pc)
+          v[b * MM + pc] = b < nkb ? __ldcs(rec + pc) : make_uint2(0u, 0u);
+      }
+    };
+    uint2 cur[8], nxt[8];
+    int n = n_begin + threadIdx.x;
+    if (n < n_end) load(n, cur);
+    for (; n < n_end; n += blockDim.x) {
+      if (n + static_cast<int>(blockDim.x) < n_end) load(n + blockDim.x, nxt);
+      float acc = 0.0f;
+#pragma unroll
+      for (int b = 0; b < kBlocks; ++b) {
+        if (b < nkb) {
+          const float* Lb = L + b * 8 * MM * 256;
+#pragma unroll
+          for (int pc = 0; pc < MM; ++pc) {
+            const uint2 v = cur[b * MM + pc];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
+              acc += Lb[(pc * 8 + k) * 256 + code];
+            }
+          }
+        }
+      }
+      p.partial[static_cast<int64_t>(chunk) * p.N + n] = acc;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
+    }
+  } else {
+    for (int n = n_begin + threadIdx.x; n < n_end; n += blockDim.x) {
+      float acc = 0.0f;
+      for (int b = 0; b < nkb; ++b) {
+        const uint2* rec = reinterpret_cast<const uint2*>(
+            p.packed + (static_cast<int64_t>(kb0 + b) * p.N + n) * 8 * M);
+        const float* Lb = L + b * 8 * M * 256;      // tables of this K block's 8 groups
+        for (int pc = 0; pc < M; ++pc) {
+          const uint2 v = __ldcs(rec + pc);         // streamed once: no reuse in L1
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
+            // byte pc*8 + k of the record is group (pc*8 + k) / M, codebook (pc*8 + k) % M,
+            // and its table is entry ((pc*8 + k) * 256 + code) of this K block's [8][M][256]
+            acc += Lb[(pc * 8 + k) * 256 + code];
+          }
+        }
+      }
+      p.partial[static_cast<int64_t>(chunk) * p.N + n] = acc;
+    }
+  }
+}
+
 size_t lut_smem_bytes(int J, int M, int Tp, int T) {
   return static_cast<size_t>(J) * M * 256 * Tp * 4 + static_cast<size_t>(T) * J * 8 * 4;
 }
 
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
+  if (p.Tp == 1) {
+    static std::atomic<int> configured1[64] = {}, configured2[64] = {}, configured4[64] = {},
+        configured0[64] = {};
+    const size_t bytes = static_cast<size_t>(p.J) * p.M * 256 * 4 + static_cast<size_t>(p.J) * 8 * 4;
+    const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
+    const dim3 grid(p.chunks, n_slices);
+    auto go = [&](auto kernel, std::atomic<int> (&conf)[64]) -> cudaError_t {
+      const cudaError_t se = ensure_dynamic_smem(kernel, bytes, conf);
+      if (se != cudaSuccess) return se;
+      return launch_pdl(kernel, grid, dim3(256), bytes, st, p);
+    };
+    if (p.M == 1) return go(lut1_kernel<1>, configured1);
+    if (p.M == 2) return go(lut1_kernel<2>, configured2);
+    if (p.M == 4) return go(lut1_kernel<4>, configured4);
+    return go(lut1_kernel<0>, configured0);
+  }
   static std::atomic<int> configured[64] = {};
   const size_t bytes = lut_smem_bytes(p.J, p.M, p.Tp, p.T);
   const cudaError_t se = ensure_dynamic_smem(lut_kernel, bytes, configured);

@@ -277,3 +277,28 @@ def test_noalloc_argument_checks_before_any_cuda_call(lib):
     assert lib.aq_linear_noalloc(*args(4, 4096, 2048, out=2)) == -3  # int8 output not offered
     assert lib.aq_linear_noalloc(*args(4, 4096, 2048, s=float("nan"))) == -2
     assert lib.aq_linear_noalloc(*args(4, 4100, 2048)) == -2        # K % 16
+
+
+def test_auto_path_rules(lib):
+    """AUTO's choices for a linear layer (no device access): one token on a layer with at least
+    12 MB of 8-bit codes takes the one-token table kernel; few tokens otherwise the few-token
+    kernel; one row tile the fused decode; more the dense path.  fp16 activations choose the
+    shared-memory A form only where its plan has no K split and a wider N tile."""
+    import paper_2506_05960_gb300 as aq
+    LUT, FEW, FUSED, DENSE = 3, 4, 2, 1
+    assert aq.aq_linear_plan(1, 8192, 16384, 8, 2, 8)["path"] == LUT       # 33.6 MB of codes
+    assert aq.aq_linear_plan(1, 8192, 16384, 8, 1, 8)["path"] == LUT       # 16.8 MB
+    assert aq.aq_linear_plan(1, 4096, 8192, 8, 2, 8)["path"] == FEW        # 8.4 MB
+    assert aq.aq_linear_plan(1, 8192, 16384, 8, 1, 16)["path"] == FEW      # 16-bit codes
+    assert aq.aq_linear_plan(2, 8192, 16384, 8, 2, 8)["path"] == FEW       # two tokens
+    assert aq.aq_linear_plan(1, 960, 2880, 8, 2, 8)["path"] == FEW
+    assert aq.aq_linear_plan(100, 960, 2880, 8, 2, 8)["path"] == FUSED
+    assert aq.aq_linear_plan(4096, 960, 2880, 8, 2, 8)["path"] == DENSE
+    # the one-token table path needs a workspace for its per-chunk partial sums
+    assert aq.aq_linear_workspace_size(1, 8192, 16384, 8, 2, 8) == \
+        aq.aq_linear_workspace_size(1, 8192, 16384, 8, 2, 8, LUT) > 0
+    for (T, K, N) in ((4096, 960, 2880), (16384, 192, 576), (2048, 960, 960)):
+        p16, p8 = aq.aq_linear_f16_plan(T, K, N), aq.aq_linear_plan(T, K, N)
+        wider = aq.aq_linear_a16_plan(T, K, N)
+        want = wider["splits"] == 1 and wider["BN"] > p8["BN"]
+        assert p16["a16"] == (1 if want else 0), (T, K, N, p16, p8, wider)

@@ -67,3 +67,29 @@ def test_lut_path_selection():
     with pytest.raises(aq.AQError) as e:
         aq.aq_linear_workspace_size(17, 960, 960, 8, 2, 8, LUT)      # too many tokens
     assert e.value.status == -3
+
+
+@pytest.mark.parametrize("K,N,M", [
+    (960, 2880, 2),       # the qkv projection
+    (208, 40, 2),         # 26 groups: the last packed K block half empty; N not a warp multiple
+    (4096, 4096, 2),      # many chunks and row slices
+    (576, 1728, 1),       # one codebook: 8 K blocks per chunk
+    (576, 1736, 3),       # three codebooks (general index arithmetic)
+    (1024, 512, 4),
+    (512, 264, 5),
+    (640, 96, 8),         # one K block per chunk
+])
+def test_lut_one_token(K, N, M):
+    """One token: one fp32 per table entry (lut1_kernel), every output kind."""
+    import paper_2506_05960_gb300 as aq
+    inp = make_linear(LinearSpec(T=1, K=K, N=N, M=M, B=8, cb_std=0.05 / M ** 0.5),
+                      seed=300 + K + N + M)
+    ref = O.layer_f64(inp)
+    assert_close(run_linear(inp, path=LUT), ref, (K, N, M))
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    y32 = run_linear(inp, path=LUT, out_f32=True, with_bias=False)
+    assert_close(y32, O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], None), (K, N, M))
+    y_lut = O.lut_linear_f64(inp["xq"], inp["s_x"], inp["codes"], inp["codebooks"],
+                             inp["scale"], inp["bias"])
+    assert_close(run_linear(inp, path=LUT), y_lut, "table order")
+    assert aq.aq_linear_workspace_size(1, K, N, 8, M, 8, LUT) > 0
