@@ -638,6 +638,8 @@ KERNEL_WORKLOADS = {
     "fused128": "aq_linear, T=128 K=960 N=2880 2x8 (fused decode, K split in cluster)",
     "few4": "aq_linear, T=4 K=960 N=2880 2x8 (few-token kernel)",
     "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
+    "lut1": ("aq_linear, T=1 K=8192 N=65536 2x8 (134 MB of codes, more than L2), AUTO: the "
+             "one-token table kernel"),
     "grad": "aq_codebook_grad of the qkv layer (fp32 G)",
     "search": "aq_code_update of the qkv layer, both codebooks, unweighted",
 }
@@ -648,9 +650,10 @@ def run_kernel_workload(args, aq, torch, dev, stream):
     (no graph), for ncu captures; returns the mean time per call (CUDA events)."""
     from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_linear
     w = args.workload
-    if w in ("fused128", "few4", "lut8"):
-        T = {"fused128": 128, "few4": 4, "lut8": 8}[w]
-        spec = LinearSpec(T=T, K=960, N=2880, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02)
+    if w in ("fused128", "few4", "lut8", "lut1"):
+        T = {"fused128": 128, "few4": 4, "lut8": 8, "lut1": 1}[w]
+        K, N = (8192, 65536) if w == "lut1" else (960, 2880)
+        spec = LinearSpec(T=T, K=K, N=N, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02)
         L = Dev(aq, torch, make_linear(spec, seed=7), dev, path=3 if w == "lut8" else 0)
         call = lambda: L.layer(stream)
     else:
