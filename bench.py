@@ -1128,10 +1128,11 @@ def main():
                                   "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
                     del gs, Ls
         # few tokens on a layer large enough to amortise the launches: how fast each path
-        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes); AUTO takes the one-token
-        # table kernel at T = 1
-        for Ts, pth in ((1, aq.AQ_PATH_FEW_TOKENS), (1, aq.AQ_PATH_AUTO), (4, aq.AQ_PATH_FEW_TOKENS),
-                        (4, aq.AQ_PATH_FUSED)):
+        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes); AUTO takes the
+        # vector-table kernel up to four tokens here
+        for Ts, pth in ((1, aq.AQ_PATH_FEW_TOKENS), (1, aq.AQ_PATH_AUTO),
+                        (2, aq.AQ_PATH_FEW_TOKENS), (2, aq.AQ_PATH_AUTO),
+                        (4, aq.AQ_PATH_FEW_TOKENS), (4, aq.AQ_PATH_FUSED), (4, aq.AQ_PATH_AUTO)):
             inp_s = _mlin(LinearSpec(T=Ts, K=8192, N=16384, M=2, B=8), seed=90 + Ts)
             Ls = [Dev(aq, torch, inp_s, dev, path=pth) for _ in range(4)]
             with torch.cuda.stream(stream):

@@ -350,26 +350,31 @@ int resolve_conv_path(int path, int m_tiles, int g) {
 constexpr int kLutMaxT = 16;       // tokens per call the LUT kernel handles
 
 struct LutPlan {
-  int J, Tp, chunks, rows_per_cta;
+  int vec, J, Tp, chunks, rows_per_cta;
   size_t ws_bytes;
 };
 
 LutPlan plan_lut(int T, int K, int N, int M) {
   LutPlan lp{};
-  if (T == 1) {
-    // one token: one fp32 per table entry, chunks of whole packed K blocks with tables of at
-    // most 64 KB (8 K blocks for one codebook, 4 for two, 2 for three or four, else 1), over
-    // (chunk, row slice) CTAs
-    lp.Tp = 1;
-    lp.J = 8 * (M == 1 ? 8 : (M == 2 ? 4 : (M <= 4 ? 2 : 1)));
+  const bool mm = M == 1 || M == 2 || M == 4;
+  if (T == 1 || (T <= 4 && mm)) {
+    // lutv_kernel: TP = 1, 2 or 4 floats per entry; chunks of whole packed K blocks with at
+    // most 64 KB of tables (8 / (M * TP) K blocks, at least one: four codebooks at four
+    // tokens take 128 KB), over (chunk, row slice) CTAs -- as many row slices as keep them
+    // within one wave (a second, nearly empty wave would double the time)
+    lp.vec = 1;
+    lp.Tp = T == 1 ? 1 : (T == 2 ? 2 : 4);
+    const int kb = mm ? std::max(1, 8 / (M * lp.Tp)) : (M <= 4 ? 2 : 1);
+    lp.J = 8 * kb;
     const int G = K / 8;
     lp.chunks = (G + lp.J - 1) / lp.J;
-    // (as many row slices as keep chunks x slices within one wave of three CTAs per SM: a
-    // second, nearly empty wave would double the time)
-    int n_slices = 3 * kPlanSMs / lp.chunks;
+    const size_t smem = static_cast<size_t>(lp.J) * M * 256 * lp.Tp * 4 +
+                        static_cast<size_t>(lp.Tp) * lp.J * 8 * 4;
+    const int per_sm = std::max(1, std::min(3, static_cast<int>(232448 / (smem + 1024))));
+    int n_slices = per_sm * kPlanSMs / lp.chunks;
     if (n_slices < 1) n_slices = 1;
     lp.rows_per_cta = ((N + n_slices - 1) / n_slices + 31) / 32 * 32;
-    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * N * 4, 1024);
+    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * T * N * 4, 1024);
     return lp;
   }
   lp.Tp = T <= 4 ? 4 : (T <= 8 ? 8 : 16);
@@ -391,17 +396,20 @@ constexpr int kFewTokensMaxT = 16;
 constexpr int kFewTokensAutoMaxT = 4;
 
 // AUTO / explicit path of a linear layer: -1 unknown path, -2 path cannot run this layer.
-// AUTO takes the one-token table kernel (lut1_kernel) from this many bytes of 8-bit codes:
-// measured on GB300 against the few-token kernel (2x8 codebooks, us, few-token / table):
-// 8.4 MB 12.3 / 16.4, 16.8 MB (1x8) 33.4 / 20.3, 33.6 MB 45.0 / 29.2, 67.1 MB (4x8) 198 / 48.
-constexpr size_t kLut1AutoMinCodeBytes = 12u << 20;
+// AUTO takes the vector-table kernel (lutv_kernel: one token with any M, up to four tokens with
+// M = 1, 2 or 4) from this many bytes of 8-bit codes.  Measured on GB300 (layer only, us,
+// few-token / table / fused GEMM): T=1 2x8 8.4 MB 12.3 / 16.4, 33.6 MB 45.0 / 29.2; T=1 1x8
+// 16.8 MB 33.4 / 20.3; T=1 4x8 67.1 MB 198 / 48; T=2 2x8 8.4 MB 17.4 / 18.5 / 28.2, 33.6 MB
+// 62.5 / 39.0 / 81.4; T=4 2x8 8.4 MB 24.1 / 24.6 / 28.2, 33.6 MB 127.8 / 67.8 / 82.7; T=4 1x8
+// 16.8 MB 92.4 / 36.4 / 61.3; T=4 4x8 67.1 MB 285 / 116 / 163.
+constexpr size_t kLutAutoMinCodeBytes = 12u << 20;
 
 int resolve_linear_path(int path, int T, int B, int N = 0, int K = 0, int M = 0) {
   const int m_tiles = (T + aq::kBM - 1) / aq::kBM;
   switch (path) {
     case AQ_PATH_AUTO:
-      if (T == 1 && B == 8 &&
-          static_cast<size_t>(N) * (K / 8) * M >= kLut1AutoMinCodeBytes)
+      if (T <= kFewTokensAutoMaxT && B == 8 && (T == 1 || M == 1 || M == 2 || M == 4) &&
+          static_cast<size_t>(N) * (K / 8) * M >= kLutAutoMinCodeBytes)
         return AQ_PATH_LUT;
       if (T <= kFewTokensAutoMaxT) return AQ_PATH_FEW_TOKENS;
       return m_tiles <= kFusedAutoMaxMTiles ? AQ_PATH_FUSED : AQ_PATH_DENSE;
@@ -1197,6 +1205,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     lpar.K = K;
     lpar.N = N;
     lpar.M = M;
+    lpar.vec = lp.vec;
     lpar.Tp = lp.Tp;
     lpar.J = lp.J;
     lpar.G = K / 8;

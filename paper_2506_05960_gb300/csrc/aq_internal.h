@@ -81,9 +81,11 @@ struct LutParams {
   const __half* books;          // [M][256][8]
   float* partial;               // [chunks][T][N] partial sums
   int T, K, N, M;
-  int Tp;                       // floats per table entry: 1 (one token: lut1_kernel), or T
+  int vec;                      // 1: lutv_kernel (whole K blocks per chunk, Tp = 1, 2 or 4
+                                // floats per entry); 0: lut_kernel
+  int Tp;                       // floats per table entry: vec: 1, 2 or 4 (>= T); else T
                                 // rounded up to 4, 8 or 16
-  int J;                        // groups per chunk (divides 8; Tp == 1: whole K blocks)
+  int J;                        // groups per chunk (vec: whole K blocks; else divides 8)
   int G;                        // K / 8
   int chunks, rows_per_cta;
 };

@@ -113,42 +113,65 @@ __global__ void __launch_bounds__(256) lut_kernel(const LutParams p) {
   }
 }
 
-// One token (Tp == 1): the same order with one fp32 per table entry.  A chunk is J groups =
-// J / 8 whole packed K blocks, its tables J * M * 256 floats (<= 64 KB).  One thread per output
-// row: per K block it reads the row's 8 * M codes as M contiguous 8-byte pieces (consecutive
-// rows consecutive, so a warp's loads are coalesced) and adds one table entry per code, in
-// the fixed order (K block, group, codebook).  MM: M when 1, 2 or 4 (index arithmetic known
-// at compile time), else 0.
-template <int MM>
-__global__ void __launch_bounds__(256) lut1_kernel(const LutParams p) {
+// Up to four tokens (TP = 1, 2 or 4 floats per table entry; T <= TP): the same order with
+// chunks of whole packed K blocks and at most 64 KB of tables, and one thread per output row:
+// per K block it reads the row's 8 * M codes as M contiguous 8-byte pieces (consecutive rows
+// consecutive, so a warp's loads are coalesced) and adds, per code, the entry's TP floats with
+// one vector load, in the fixed order (K block, group, codebook).  MM: M when 1, 2 or 4 (index
+// arithmetic known at compile time; then a chunk is 8 / (MM * TP) K blocks, at least one, and
+// the row's code pieces are loaded together, the next row's while this row's entries are
+// summed), or 0: any M, one token.
+template <int MM, int TP>
+__global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
   extern __shared__ float4 lut_smem4[];
-  float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256]
-  const int J = p.J, M = MM > 0 ? MM : p.M;
-  float* xs = L + static_cast<size_t>(J) * M * 256;            // [J * 8]
+  float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256][TP]
+  const int J = p.J, M = MM > 0 ? MM : p.M, T = p.T;
+  float* xs = L + static_cast<size_t>(J) * M * 256 * TP;       // [TP][J * 8]
   grid_dependency_wait();
   allow_dependents();
   const int chunk = blockIdx.x;
   const int g0 = chunk * J;
   const int nj = min(J, p.G - g0);
-  for (int i = threadIdx.x; i < J * 8; i += blockDim.x)
-    xs[i] = (i < nj * 8) ? static_cast<float>(p.xq[g0 * 8 + i]) : 0.0f;
+  const int width = J * 8;
+  for (int i = threadIdx.x; i < TP * width; i += blockDim.x) {
+    const int t = i / width;
+    const int e = i - t * width;
+    xs[i] = (t < T && e < nj * 8)
+                ? static_cast<float>(p.xq[static_cast<int64_t>(t) * p.K + g0 * 8 + e])
+                : 0.0f;
+  }
   __syncthreads();
-  // build: L[j][m][c] = sum_e x[g0 + j][e] * C^(m)[c][e], ascending e (zero past the last group)
+  // build: L[j][m][c][t] = sum_e x[t][g0 + j][e] * C^(m)[c][e], ascending e (zero past the last
+  // group and past the last token)
   const int entries = J * M * 256;
   for (int ent = threadIdx.x; ent < entries; ent += blockDim.x) {
     const int j = ent / (M * 256);
     const int r = ent - j * (M * 256);
     const uint4 raw = reinterpret_cast<const uint4*>(p.books)[r];
     const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
-    const float* xr = xs + j * 8;
-    float s = 0.0f;
+    float cw[8];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const float2 f = __half22float2(h2[i]);
-      s = fmaf(xr[2 * i], f.x, s);
-      s = fmaf(xr[2 * i + 1], f.y, s);
+      cw[2 * i] = f.x;
+      cw[2 * i + 1] = f.y;
     }
-    L[ent] = s;
+    float o[TP];
+#pragma unroll
+    for (int t = 0; t < TP; ++t) {
+      const float* xr = xs + t * width + j * 8;
+      float s = 0.0f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s = fmaf(xr[e], cw[e], s);
+      o[t] = s;
+    }
+    if constexpr (TP == 1) {
+      L[ent] = o[0];
+    } else if constexpr (TP == 2) {
+      reinterpret_cast<float2*>(L)[ent] = make_float2(o[0], o[1]);
+    } else {
+      reinterpret_cast<float4*>(L)[ent] = make_float4(o[0], o[1], o[2], o[3]);
+    }
   }
   __syncthreads();
   const int kb0 = g0 >> 3;
@@ -156,11 +179,9 @@ __global__ void __launch_bounds__(256) lut1_kernel(const LutParams p) {
   const int n_begin = blockIdx.y * p.rows_per_cta;
   const int n_end = min(p.N, n_begin + p.rows_per_cta);
   if constexpr (MM > 0) {
-    // one, two or four codebooks: a chunk is 8 / MM K blocks, so a row's codes in it are always
-    // eight 8-byte pieces; all eight are loaded at once, and the next row's while this row's
-    // entries are summed (the code stream's latency overlaps the lookups)
-    constexpr int kBlocks = 8 / MM;
-    auto load = [&](int n, uint2 (&v)[8]) {
+    constexpr int kBlocks = (MM * TP >= 8) ? 1 : 8 / (MM * TP);
+    constexpr int kPieces = kBlocks * MM;         // 8-byte code pieces of a row in a chunk
+    auto load = [&](int n, uint2 (&v)[kPieces]) {
 #pragma unroll
       for (int b = 0; b < kBlocks; ++b) {
         const uint2* rec = reinterpret_cast<const uint2*>(
@@ -170,32 +191,52 @@ __global__ void __launch_bounds__(256) lut1_kernel(const LutParams p) {
           v[b * MM + pc] = b < nkb ? __ldcs(rec + pc) : make_uint2(0u, 0u);
       }
     };
-    uint2 cur[8], nxt[8];
+    uint2 cur[kPieces], nxt[kPieces];
     int n = n_begin + threadIdx.x;
     if (n < n_end) load(n, cur);
     for (; n < n_end; n += blockDim.x) {
       if (n + static_cast<int>(blockDim.x) < n_end) load(n + blockDim.x, nxt);
-      float acc = 0.0f;
+      float acc[TP];
+#pragma unroll
+      for (int t = 0; t < TP; ++t) acc[t] = 0.0f;
 #pragma unroll
       for (int b = 0; b < kBlocks; ++b) {
         if (b < nkb) {
-          const float* Lb = L + b * 8 * MM * 256;
+          const float* Lb = L + b * 8 * MM * 256 * TP;   // tables of this K block's 8 groups
 #pragma unroll
           for (int pc = 0; pc < MM; ++pc) {
             const uint2 v = cur[b * MM + pc];
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
+              // byte pc*8 + k of the record is group (pc*8 + k) / MM, codebook (pc*8 + k) % MM,
+              // and its entry is ((pc*8 + k) * 256 + code) of this K block's [8][MM][256]
               const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
-              acc += Lb[(pc * 8 + k) * 256 + code];
+              const float* e = Lb + ((pc * 8 + k) * 256 + code) * TP;
+              if constexpr (TP == 1) {
+                acc[0] += e[0];
+              } else if constexpr (TP == 2) {
+                const float2 w = *reinterpret_cast<const float2*>(e);
+                acc[0] += w.x;
+                acc[1] += w.y;
+              } else {
+                const float4 w = *reinterpret_cast<const float4*>(e);
+                acc[0] += w.x;
+                acc[1] += w.y;
+                acc[2] += w.z;
+                acc[3] += w.w;
+              }
             }
           }
         }
       }
-      p.partial[static_cast<int64_t>(chunk) * p.N + n] = acc;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
+      for (int t = 0; t < TP; ++t)
+        if (t < T) p.partial[(static_cast<int64_t>(chunk) * T + t) * p.N + n] = acc[t];
+#pragma unroll
+      for (int i = 0; i < kPieces; ++i) cur[i] = nxt[i];
     }
   } else {
+    static_assert(MM > 0 || TP == 1, "any M: one token only");
     for (int n = n_begin + threadIdx.x; n < n_end; n += blockDim.x) {
       float acc = 0.0f;
       for (int b = 0; b < nkb; ++b) {
@@ -207,8 +248,6 @@ __global__ void __launch_bounds__(256) lut1_kernel(const LutParams p) {
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
-            // byte pc*8 + k of the record is group (pc*8 + k) / M, codebook (pc*8 + k) % M,
-            // and its table is entry ((pc*8 + k) * 256 + code) of this K block's [8][M][256]
             acc += Lb[(pc * 8 + k) * 256 + code];
           }
         }
@@ -223,10 +262,12 @@ size_t lut_smem_bytes(int J, int M, int Tp, int T) {
 }
 
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
-  if (p.Tp == 1) {
-    static std::atomic<int> configured1[64] = {}, configured2[64] = {}, configured4[64] = {},
-        configured0[64] = {};
-    const size_t bytes = static_cast<size_t>(p.J) * p.M * 256 * 4 + static_cast<size_t>(p.J) * 8 * 4;
+  if (p.vec) {
+    // lutv_kernel: whole K blocks per chunk, TP = p.Tp floats per entry
+    static std::atomic<int> c11[64] = {}, c21[64] = {}, c41[64] = {}, c01[64] = {}, c12[64] = {},
+                            c22[64] = {}, c42[64] = {}, c14[64] = {}, c24[64] = {}, c44[64] = {};
+    const size_t bytes = static_cast<size_t>(p.J) * p.M * 256 * p.Tp * 4 +
+                         static_cast<size_t>(p.Tp) * p.J * 8 * 4;
     const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
     const dim3 grid(p.chunks, n_slices);
     auto go = [&](auto kernel, std::atomic<int> (&conf)[64]) -> cudaError_t {
@@ -234,10 +275,20 @@ cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
       if (se != cudaSuccess) return se;
       return launch_pdl(kernel, grid, dim3(256), bytes, st, p);
     };
-    if (p.M == 1) return go(lut1_kernel<1>, configured1);
-    if (p.M == 2) return go(lut1_kernel<2>, configured2);
-    if (p.M == 4) return go(lut1_kernel<4>, configured4);
-    return go(lut1_kernel<0>, configured0);
+    const int mm = (p.M == 1 || p.M == 2 || p.M == 4) ? p.M : 0;
+    switch (p.Tp * 16 + mm) {
+      case 16 + 1: return go(lutv_kernel<1, 1>, c11);
+      case 16 + 2: return go(lutv_kernel<2, 1>, c21);
+      case 16 + 4: return go(lutv_kernel<4, 1>, c41);
+      case 16 + 0: return go(lutv_kernel<0, 1>, c01);
+      case 32 + 1: return go(lutv_kernel<1, 2>, c12);
+      case 32 + 2: return go(lutv_kernel<2, 2>, c22);
+      case 32 + 4: return go(lutv_kernel<4, 2>, c42);
+      case 64 + 1: return go(lutv_kernel<1, 4>, c14);
+      case 64 + 2: return go(lutv_kernel<2, 4>, c24);
+      case 64 + 4: return go(lutv_kernel<4, 4>, c44);
+      default: return cudaErrorInvalidConfiguration;
+    }
   }
   static std::atomic<int> configured[64] = {};
   const size_t bytes = lut_smem_bytes(p.J, p.M, p.Tp, p.T);

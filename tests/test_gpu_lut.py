@@ -69,21 +69,29 @@ def test_lut_path_selection():
     assert e.value.status == -3
 
 
-@pytest.mark.parametrize("K,N,M", [
-    (960, 2880, 2),       # the qkv projection
-    (208, 40, 2),         # 26 groups: the last packed K block half empty; N not a warp multiple
-    (4096, 4096, 2),      # many chunks and row slices
-    (576, 1728, 1),       # one codebook: 8 K blocks per chunk
-    (576, 1736, 3),       # three codebooks (general index arithmetic)
-    (1024, 512, 4),
-    (512, 264, 5),
-    (640, 96, 8),         # one K block per chunk
+@pytest.mark.parametrize("T,K,N,M", [
+    (1, 960, 2880, 2),       # the qkv projection
+    (1, 208, 40, 2),         # 26 groups: the last packed K block half empty; N not a warp multiple
+    (1, 4096, 4096, 2),      # many chunks and row slices
+    (1, 576, 1728, 1),       # one codebook: 8 K blocks per chunk
+    (1, 576, 1736, 3),       # three codebooks (general index arithmetic)
+    (1, 1024, 512, 4),
+    (1, 512, 264, 5),
+    (1, 640, 96, 8),         # one K block per chunk
+    (2, 960, 2880, 2),       # two floats per entry
+    (2, 208, 40, 1),
+    (2, 1024, 520, 4),
+    (3, 960, 2880, 2),       # four floats per entry, one token unused
+    (4, 4096, 4096, 2),
+    (4, 208, 264, 1),
+    (4, 1024, 512, 4),       # 128 KB of tables: one CTA per SM
 ])
-def test_lut_one_token(K, N, M):
-    """One token: one fp32 per table entry (lut1_kernel), every output kind."""
+def test_lut_vector_tables(T, K, N, M):
+    """Up to four tokens with whole K blocks per chunk and 1, 2 or 4 floats per table entry
+    (lutv_kernel), against the oracle's decode order and table order, fp16 and fp32 outputs."""
     import paper_2506_05960_gb300 as aq
-    inp = make_linear(LinearSpec(T=1, K=K, N=N, M=M, B=8, cb_std=0.05 / M ** 0.5),
-                      seed=300 + K + N + M)
+    inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=8, cb_std=0.05 / M ** 0.5),
+                      seed=300 + T + K + N + M)
     ref = O.layer_f64(inp)
     assert_close(run_linear(inp, path=LUT), ref, (K, N, M))
     W = O.decode_f64(inp["codes"], inp["codebooks"])
@@ -92,4 +100,4 @@ def test_lut_one_token(K, N, M):
     y_lut = O.lut_linear_f64(inp["xq"], inp["s_x"], inp["codes"], inp["codebooks"],
                              inp["scale"], inp["bias"])
     assert_close(run_linear(inp, path=LUT), y_lut, "table order")
-    assert aq.aq_linear_workspace_size(1, K, N, 8, M, 8, LUT) > 0
+    assert aq.aq_linear_workspace_size(T, K, N, 8, M, 8, LUT) > 0
