@@ -639,7 +639,7 @@ KERNEL_WORKLOADS = {
     "few4": "aq_linear, T=4 K=960 N=2880 2x8 (few-token kernel)",
     "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
     "lut1": ("aq_linear, T=1 K=8192 N=65536 2x8 (134 MB of codes, more than L2), AUTO: the "
-             "one-token table kernel"),
+             "vector-table kernel with one fp32 per entry"),
     "grad": "aq_codebook_grad of the qkv layer (fp32 G)",
     "search": "aq_code_update of the qkv layer, both codebooks, unweighted",
 }
