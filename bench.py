@@ -640,6 +640,9 @@ KERNEL_WORKLOADS = {
     "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
     "lut1": ("aq_linear, T=1 K=8192 N=65536 2x8 (134 MB of codes, more than L2), AUTO: the "
              "vector-table kernel with one fp32 per entry"),
+    "book16_decode": "aq_decode of the 2^16-codebook conv weight (960 x 8640, 1x16)",
+    "book16_gemm": ("aq_conv2d_nhwc 2x8x8x960->960 1x16, weights decoded beforehand (the "
+                    "tensor-core GEMM alone)"),
     "grad": "aq_codebook_grad of the qkv layer (fp32 G)",
     "search": "aq_code_update of the qkv layer, both codebooks, unweighted",
 }
@@ -648,9 +651,19 @@ KERNEL_WORKLOADS = {
 def run_kernel_workload(args, aq, torch, dev, stream):
     """One kernel's call on the seeded qkv-shaped layer, --warmup + --steps plain launches
     (no graph), for ncu captures; returns the mean time per call (CUDA events)."""
-    from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_linear
+    from aq_synth import SEEDS, WORKLOADS, LinearSpec, make_conv, make_linear
     w = args.workload
-    if w in ("fused128", "few4", "lut8", "lut1"):
+    if w.startswith("book16"):
+        L = Dev(aq, torch, make_conv(WORKLOADS["conv8_book16"], seed=SEEDS["conv8_book16"]), dev,
+                path=aq.AQ_PATH_PREDECODED)
+        L.quant(stream)
+        if w == "book16_decode":
+            wdec = torch.empty((L.N, L.K), dtype=torch.float16, device=dev)
+            call = lambda: L.decode_only(stream, wdec)
+        else:
+            L.decode_only(stream, L.ws)
+            call = lambda: L.layer(stream)
+    elif w in ("fused128", "few4", "lut8", "lut1"):
         T = {"fused128": 128, "few4": 4, "lut8": 8, "lut1": 1}[w]
         K, N = (8192, 65536) if w == "lut1" else (960, 2880)
         spec = LinearSpec(T=T, K=K, N=N, M=2, B=8, cb_std=0.05, act="uniform", s_x=0.02)

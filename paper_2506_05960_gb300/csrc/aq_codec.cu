@@ -411,15 +411,17 @@ cudaError_t launch_decode_kaq(const void* codes, const void* books, void* W, int
 // where G[n][k] = sum_t dY[t][n] * xq[t][k] is the gradient with respect to the
 // unscaled weight (a plain GEMM the caller runs).  dC is accumulated (+=) in fp32:
 // 8-bit codebooks in shared memory per CTA, flushed with global atomics; 16-bit
-// codebooks with global atomics directly.  One thread per group; g = 8 reads the
-// packed layout, g = 9 (one group per 3x3 filter) the canonical [N][Cin][M] codes
-// with G in the convolution's OHWI order.
+// codebooks with global atomics directly.  One thread per group (its G row piece and
+// its M codes are loaded before the first add); g = 8 reads the packed layout, g = 9
+// (one group per 3x3 filter) the canonical [N][Cin][M] codes with G in the
+// convolution's OHWI order.
 template <int EB, bool kKaq>
-__global__ void __launch_bounds__(256) codebook_grad_kernel(
+__global__ void __launch_bounds__(256, 2) codebook_grad_kernel(
     const uint8_t* __restrict__ codes, const float* __restrict__ G,
     const __half* __restrict__ scale, float s_x, float* __restrict__ dC, int N, int K, int M,
     int KB) {
   constexpr int g = kKaq ? 9 : 8;
+  constexpr int kMaxM = EB == 1 ? 8 : 2;
   // 8-bit codes: the CTA's table in shared memory, element-major [g][M*256] so that
   // the adds of a warp (random codewords, same element) spread over all banks
   extern __shared__ float sdc[];
@@ -461,15 +463,21 @@ __global__ void __launch_bounds__(256) codebook_grad_kernel(
       v[0] = f * a.x; v[1] = f * a.y; v[2] = f * a.z; v[3] = f * a.w;
       v[4] = f * b.x; v[5] = f * b.y; v[6] = f * b.z; v[7] = f * b.w;
     }
-    for (int m = 0; m < M; ++m) {
-      const int c = EB == 1 ? codes[idx * M + m]
-                            : reinterpret_cast<const uint16_t*>(codes)[idx * M + m];
+    int cw[kMaxM];
+#pragma unroll
+    for (int m = 0; m < kMaxM; ++m)
+      if (m < M)
+        cw[m] = EB == 1 ? codes[idx * M + m]
+                        : reinterpret_cast<const uint16_t*>(codes)[idx * M + m];
+#pragma unroll
+    for (int m = 0; m < kMaxM; ++m) {
+      if (m >= M) break;
       if constexpr (EB == 1) {
-        float* dst = sdc + m * 256 + c;
+        float* dst = sdc + m * 256 + cw[m];
 #pragma unroll
         for (int e = 0; e < g; ++e) atomicAdd(dst + e * (M * 256), v[e]);
       } else {
-        float* dst = dC + ((static_cast<int64_t>(m) << 16) + c) * g;
+        float* dst = dC + ((static_cast<int64_t>(m) << 16) + cw[m]) * g;
 #pragma unroll
         for (int e = 0; e < g; ++e) atomicAdd(dst + e, v[e]);
       }
@@ -501,30 +509,23 @@ cudaError_t launch_codebook_grad(const void* codes, const float* G, const __half
   const bool kaq = g == 9;
   const int KB = (K + 63) / 64;
   const int64_t total = kaq ? static_cast<int64_t>(N) * (K / 9) : static_cast<int64_t>(KB) * N * 8;
-  int64_t blocks = (total + 255) / 256;
   // 8-bit: two blocks per SM, each flushes its table once (more threads per SM only
-  // add shared-memory atomic contention)
-  const int64_t cap = B == 8 ? 152 * 2 : 152 * 8;
+  // add shared-memory atomic contention; a flush summed first over a cluster's tables
+  // through distributed shared memory measured slower)
   const int threads = 256;
-  blocks = (total + threads - 1) / threads;
+  const int64_t cap = B == 8 ? 152 * 2 : 152 * 8;
+  int64_t blocks = (total + threads - 1) / threads;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   const dim3 grid(static_cast<unsigned>(blocks)), block(static_cast<unsigned>(threads));
   const uint8_t* c = static_cast<const uint8_t*>(codes);
   const size_t smem = B == 8 ? static_cast<size_t>(M) * 256 * g * 4 : 0;
   if (B == 8) {
-    if (kaq) {
-      if (smem > 48 * 1024)
-        cudaFuncSetAttribute(codebook_grad_kernel<1, true>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-      return launch_pdl(codebook_grad_kernel<1, true>, grid, block, smem, st, c, G, scale, s_x, dC,
-                        N, K, M, KB);
-    }
+    auto kernel = kaq ? codebook_grad_kernel<1, true> : codebook_grad_kernel<1, false>;
     if (smem > 48 * 1024)
-      cudaFuncSetAttribute(codebook_grad_kernel<1, false>,
-                           cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    return launch_pdl(codebook_grad_kernel<1, false>, grid, block, smem, st, c, G, scale, s_x, dC,
-                      N, K, M, KB);
+      cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem));
+    return launch_pdl(kernel, grid, block, smem, st, c, G, scale, s_x, dC, N, K, M, KB);
   }
   if (kaq)
     return launch_pdl(codebook_grad_kernel<2, true>, grid, block, 0, st, c, G, scale, s_x, dC, N,
