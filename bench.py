@@ -713,6 +713,59 @@ def run_kernel_workload(args, aq, torch, dev, stream):
     return e0.elapsed_time(e1) / max(1, args.steps)
 
 
+def small_t_sweep(aq, torch, dev, stream, reps=50):
+    """Layer time against the token count T in {1, 2, 4, ..., 64} on the attention-projection
+    shape (K=960, N=2880, 2x8) and on the 2^16-codebook conv's GEMM shape taken as a linear
+    layer (K=8640, N=960, 1x16), on every path that runs the shape.  Per path: the step
+    (quantizer + layer, fp16 output) with warm L2 (a graph of 8 launches replayed) and cold L2
+    (a 256 MB buffer written before each launch: a graph of 8 x (write, step) minus a graph of
+    the 8 writes).  The roofline is
+    max(flops / tensor peak, algorithmic bytes / HBM bandwidth), the bytes being codes,
+    codebooks, int8 activations, fp16 output, scale and bias."""
+    from aq_synth import LinearSpec, make_linear
+    peaks = measured_peaks()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    names = {aq.AQ_PATH_AUTO: "auto", aq.AQ_PATH_DENSE: "dense", aq.AQ_PATH_FUSED: "fused",
+             aq.AQ_PATH_LUT: "lut", aq.AQ_PATH_FEW_TOKENS: "few"}
+    rows = []
+    for shape, K, N, M, B in (("attention qkv K=960 N=2880 2x8", 960, 2880, 2, 8),
+                              ("2^16-codebook K=8640 N=960 1x16", 8640, 960, 1, 16)):
+        for T in (1, 2, 4, 8, 16, 32, 64):
+            spec = LinearSpec(T=T, K=K, N=N, M=M, B=B, cb_std=0.05, act="uniform", s_x=0.02)
+            inp = make_linear(spec, seed=11 + T)
+            fl = 2.0 * T * N * K
+            by = N * K * M * B // 64 + M * (1 << B) * 16 + T * K + 2 * T * N + 4 * N
+            roof = max(fl / (peaks["bf16_tflops"] * 1e12), by / (peaks["hbm_gbs"] * 1e9)) * 1e6
+            row = {"shape": shape, "T": T, "roofline_us": round(roof, 3),
+                   "bound": "hbm" if by / peaks["hbm_gbs"] > fl / (peaks["bf16_tflops"] * 1e3)
+                   else "tensor",
+                   "auto_path": names[aq.aq_linear_plan(T, K, N, 8, M, B, 0)["path"]]}
+            for path, pname in names.items():
+                try:
+                    aq.aq_linear_plan(T, K, N, 8, M, B, path)
+                except aq.AQError:
+                    continue
+                L = Dev(aq, torch, inp, dev, path=path)
+                with torch.cuda.stream(stream):
+                    for _ in range(3):
+                        L.step(stream)
+                stream.synchronize()
+                g = capture(torch, stream, lambda: [L.step(stream) for _ in range(8)])
+                warm = replay_ms(torch, stream, g, reps) / 8 * 1e3
+                # cold: 8 x (flush, step) minus 8 x flush, both graphs replayed
+                gc = capture(torch, stream, lambda: [(flush.fill_(1), L.step(stream))
+                                                     for _ in range(8)])
+                gf = capture(torch, stream, lambda: [flush.fill_(1) for _ in range(8)])
+                cold = (replay_ms(torch, stream, gc, 10) - replay_ms(torch, stream, gf, 10)) / 8
+                del g, gc, gf
+                assert aq.aq_device_error() == 0
+                row[pname] = {"warm_us": round(warm, 2), "cold_us": round(cold * 1e3, 2)}
+                del L
+            rows.append(row)
+            print(json.dumps(row), flush=True)
+    return rows
+
+
 def run_single(args):
     """One non-headline workload on one GPU (profiling aid): prints its timing."""
     import torch
@@ -725,6 +778,9 @@ def run_single(args):
         ms = run_kernel_workload(args, aq, torch, dev, stream)
         out = {"workload": KERNEL_WORKLOADS[args.workload], "us_per_call": ms * 1e3,
                "timing": "plain launches, CUDA events (no graph)"}
+    elif args.workload == "tsweep":
+        small_t_sweep(aq, torch, dev, stream)
+        return 0
     elif args.workload == "unet":
         ms, gflop, nl = unet_forward(aq, torch, dev, stream, 2, reps=max(1, args.steps // 100))
         out = {"workload": "UNet-shaped forward W2A8 batch 2", "ms_per_forward": ms,
@@ -764,7 +820,7 @@ def main():
     ap.add_argument("--no-cpu-baselines", action="store_true",
                     help="skip the per-workload CPU oracle timings")
     ap.add_argument("--workload", default="qkv",
-                    choices=["qkv", "conv64", "conv8", "unet"] + list(KERNEL_WORKLOADS),
+                    choices=["qkv", "conv64", "conv8", "unet", "tsweep"] + list(KERNEL_WORKLOADS),
                     help="qkv: the headline line (default); the others run only that workload "
                          "and print its timing (for profiling)")
     args = ap.parse_args()
