@@ -296,14 +296,31 @@ __device__ __forceinline__ void decode_unit_dispatch(int M, int EB, const uint8_
 // Epilogue of four summed split-K outputs y[t][n .. n+3]: acc * (s_x * scale) + bias in
 // fp32, then fp32, fp16 or the 8-bit activation rule (the same arithmetic as the
 // single-pass epilogue).
-__device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n, float4 acc) {
+// s_x * scale and bias of output columns n .. n+3 (n % 4 == 0: one 8-byte load each).
+__device__ __forceinline__ void load_scale_bias4(const GemmParams& p, int n, float (&sc)[4],
+                                                 float (&bi)[4]) {
+  const uint2 s2 = *reinterpret_cast<const uint2*>(p.scale + n);
+  const uint2 b2 = p.bias ? *reinterpret_cast<const uint2*>(p.bias + n) : make_uint2(0u, 0u);
+  const __half2 s01 = *reinterpret_cast<const __half2*>(&s2.x);
+  const __half2 s23 = *reinterpret_cast<const __half2*>(&s2.y);
+  const __half2 b01 = *reinterpret_cast<const __half2*>(&b2.x);
+  const __half2 b23 = *reinterpret_cast<const __half2*>(&b2.y);
+  sc[0] = p.s_x * __low2float(s01);
+  sc[1] = p.s_x * __high2float(s01);
+  sc[2] = p.s_x * __low2float(s23);
+  sc[3] = p.s_x * __high2float(s23);
+  bi[0] = __low2float(b01);
+  bi[1] = __high2float(b01);
+  bi[2] = __low2float(b23);
+  bi[3] = __high2float(b23);
+}
+
+// The epilogue of four consecutive outputs with their scale and bias given.
+__device__ __forceinline__ void store_out4_sb(const GemmParams& p, int64_t t, int n, float4 acc,
+                                              const float (&sc)[4], const float (&bi)[4]) {
   float o[4] = {acc.x, acc.y, acc.z, acc.w};
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float sc = p.s_x * __half2float(p.scale[n + e]);
-    const float bi = p.bias ? __half2float(p.bias[n + e]) : 0.0f;
-    o[e] = fmaf(o[e], sc, bi);
-  }
+  for (int e = 0; e < 4; ++e) o[e] = fmaf(o[e], sc[e], bi[e]);
   if (p.out_f32) {
     *reinterpret_cast<float4*>(static_cast<float*>(p.y) + t * p.N + n) =
         make_float4(o[0], o[1], o[2], o[3]);
@@ -327,6 +344,12 @@ __device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n
     uint2 w = make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
     *reinterpret_cast<uint2*>(static_cast<__half*>(p.y) + t * p.N + n) = w;
   }
+}
+
+__device__ __forceinline__ void store_out4(const GemmParams& p, int64_t t, int n, float4 acc) {
+  float sc[4], bi[4];
+  load_scale_bias4(p, n, sc, bi);
+  store_out4_sb(p, t, n, acc, sc, bi);
 }
 
 // kA16: the shared-memory A form (GemmParams::a16): fp16 A boxes with the 128-byte swizzle
@@ -909,7 +932,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the epilogue.  Every thread of every CTA passes both cluster barriers, also after a
     // failed wait above, so no CTA waits on a peer that left.
     __syncwarp();
-    cluster_sync_all();  // every split's partial tile is in its CTA's shared memory
     const TileCoord tc = tile_coord(p, blockIdx.x);
     const int nsp = p.splits;
     const int rows = (kBM + nsp - 1) / nsp;
@@ -920,6 +942,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n0 = tc.n_tile * BN;
     const uint32_t pbase = smem_u32(smem);
     const int items = r1 > r0 ? (r1 - r0) * c4n : 0;
+    cluster_sync_all();  // every split's partial tile is in its CTA's shared memory
     for (int i = threadIdx.x; i < items; i += blockDim.x) {
       const int mr = i / c4n;
       const int c4 = i - mr * c4n;
@@ -933,6 +956,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int sp = 0; sp < kMaxClusterSplits; ++sp)
         if (sp < nsp) v[sp] = ld_cluster_f4(cluster_map(pbase + off, static_cast<uint32_t>(sp)));
+      // the outputs' scale and bias are read while the partials are in flight
+      float sc[4], bi[4];
+      load_scale_bias4(p, n, sc, bi);
       float4 acc = v[0];
 #pragma unroll
       for (int sp = 1; sp < kMaxClusterSplits; ++sp) {
@@ -943,8 +969,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           acc.w += v[sp].w;
         }
       }
-      store_out4(p, t, n, acc);
+      store_out4_sb(p, t, n, acc, sc, bi);
     }
+    __syncwarp();
     cluster_sync_all();  // no CTA leaves while a peer still reads its shared memory
   }
 
