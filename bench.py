@@ -62,10 +62,10 @@ NSETS = 8
 # kernel sources are the ones it was measured on (re-captured with the fp16-code epilogue
 # branch: dram__bytes_read.sum + dram__bytes_write.sum of one launch; the key was refreshed
 # after header changes for other kernels that left the GEMM's code byte-identical apart from
-# line information).
+# line information, checked by comparing the hashes of the GEMM kernels' code sections).
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 13476096, "sources_sha": "467723e91f5ab8c9"}
+TRAFFIC = {"bytes": 13476096, "sources_sha": "f3be9d829af10fec"}
 
 
 def sources_sha() -> str:
@@ -639,7 +639,7 @@ KERNEL_WORKLOADS = {
     "few4": "aq_linear, T=4 K=960 N=2880 2x8 (few-token kernel)",
     "lut8": "aq_linear, T=8 K=960 N=2880 2x8, lookup-table path",
     "lut1": ("aq_linear, T=1 K=8192 N=65536 2x8 (134 MB of codes, more than L2), AUTO: the "
-             "vector-table kernel with one fp32 per entry"),
+             "rotated-table kernel (bank-conflict-free tables, one fp32 per entry)"),
     "book16_decode": "aq_decode of the 2^16-codebook conv weight (960 x 8640, 1x16)",
     "book16_gemm": ("aq_conv2d_nhwc 2x8x8x960->960 1x16, weights decoded beforehand (the "
                     "tensor-core GEMM alone)"),
@@ -1198,7 +1198,7 @@ def main():
                     del gs, Ls
         # few tokens on a layer large enough to amortise the launches: how fast each path
         # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes); AUTO takes the
-        # vector-table kernel up to four tokens here
+        # table path up to four tokens here
         for Ts, pth in ((1, aq.AQ_PATH_FEW_TOKENS), (1, aq.AQ_PATH_AUTO),
                         (2, aq.AQ_PATH_FEW_TOKENS), (2, aq.AQ_PATH_AUTO),
                         (4, aq.AQ_PATH_FEW_TOKENS), (4, aq.AQ_PATH_FUSED), (4, aq.AQ_PATH_AUTO)):

@@ -350,31 +350,49 @@ int resolve_conv_path(int path, int m_tiles, int g) {
 constexpr int kLutMaxT = 16;       // tokens per call the LUT kernel handles
 
 struct LutPlan {
-  int vec, J, Tp, chunks, rows_per_cta;
+  int vec, J, Tp, chunks, rows_per_cta, ctas;
   size_t ws_bytes;
 };
+
+// lutr_kernel: each CTA takes at least this many 32-row blocks of (chunk, row block) units, so
+// that building a chunk's 64 KB of tables is paid for by enough lookups.
+constexpr int kLutrMinRowBlocksPerCta = 64;
 
 LutPlan plan_lut(int T, int K, int N, int M) {
   LutPlan lp{};
   const bool mm = M == 1 || M == 2 || M == 4;
-  if (T == 1 || (T <= 4 && mm)) {
-    // lutv_kernel: TP = 1, 2 or 4 floats per entry; chunks of whole packed K blocks with at
-    // most 64 KB of tables (8 / (M * TP) K blocks, at least one: four codebooks at four
-    // tokens take 128 KB), over (chunk, row slice) CTAs -- as many row slices as keep them
-    // within one wave (a second, nearly empty wave would double the time)
-    lp.vec = 1;
+  if (T <= 4 && mm) {
+    // lutr_kernel: TP = 1, 2 or 4 floats per entry; a chunk is 32 / TP code bytes of every row
+    // (32 / (TP * M) groups); one CTA of 1024 threads per SM at most, each with an equal
+    // contiguous range of (chunk, 32-row block) units
+    lp.vec = 2;
     lp.Tp = T == 1 ? 1 : (T == 2 ? 2 : 4);
-    const int kb = mm ? std::max(1, 8 / (M * lp.Tp)) : (M <= 4 ? 2 : 1);
-    lp.J = 8 * kb;
+    const int KB = (K + 63) / 64;
+    const int nt = 32 / lp.Tp;
+    lp.J = nt / M;
+    lp.chunks = (KB * 8 * M + nt - 1) / nt;
+    const int64_t units = static_cast<int64_t>(lp.chunks) * ((N + 31) / 32);
+    lp.ctas = static_cast<int>(std::max<int64_t>(
+        1, std::min<int64_t>(kPlanSMs, units / kLutrMinRowBlocksPerCta)));
+    lp.rows_per_cta = 0;
+    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * T * N * 4, 1024);
+    return lp;
+  }
+  if (T == 1) {
+    // lutv_kernel (one token, M other than 1, 2, 4): chunks of whole packed K blocks (two for
+    // M <= 4, else one: at most 64 KB of tables), over (chunk, row slice) CTAs -- as many row
+    // slices as keep them within one wave (a second, nearly empty wave would double the time)
+    lp.vec = 1;
+    lp.Tp = 1;
+    lp.J = 8 * (M <= 4 ? 2 : 1);
     const int G = K / 8;
     lp.chunks = (G + lp.J - 1) / lp.J;
-    const size_t smem = static_cast<size_t>(lp.J) * M * 256 * lp.Tp * 4 +
-                        static_cast<size_t>(lp.Tp) * lp.J * 8 * 4;
+    const size_t smem = static_cast<size_t>(lp.J) * M * 256 * 4 + static_cast<size_t>(lp.J) * 8 * 4;
     const int per_sm = std::max(1, std::min(3, static_cast<int>(232448 / (smem + 1024))));
     int n_slices = per_sm * kPlanSMs / lp.chunks;
     if (n_slices < 1) n_slices = 1;
     lp.rows_per_cta = ((N + n_slices - 1) / n_slices + 31) / 32 * 32;
-    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * T * N * 4, 1024);
+    lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * N * 4, 1024);
     return lp;
   }
   lp.Tp = T <= 4 ? 4 : (T <= 8 ? 8 : 16);
@@ -396,13 +414,14 @@ constexpr int kFewTokensMaxT = 16;
 constexpr int kFewTokensAutoMaxT = 4;
 
 // AUTO / explicit path of a linear layer: -1 unknown path, -2 path cannot run this layer.
-// AUTO takes the vector-table kernel (lutv_kernel: one token with any M, up to four tokens with
-// M = 1, 2 or 4) from this many bytes of 8-bit codes.  Measured on GB300 (layer only, us,
-// few-token / table / fused GEMM): T=1 2x8 8.4 MB 12.3 / 16.4, 33.6 MB 45.0 / 29.2; T=1 1x8
-// 16.8 MB 33.4 / 20.3; T=1 4x8 67.1 MB 198 / 48; T=2 2x8 8.4 MB 17.4 / 18.5 / 28.2, 33.6 MB
-// 62.5 / 39.0 / 81.4; T=4 2x8 8.4 MB 24.1 / 24.6 / 28.2, 33.6 MB 127.8 / 67.8 / 82.7; T=4 1x8
-// 16.8 MB 92.4 / 36.4 / 61.3; T=4 4x8 67.1 MB 285 / 116 / 163.
-constexpr size_t kLutAutoMinCodeBytes = 12u << 20;
+// AUTO takes the table path (lutr_kernel for up to four tokens with M = 1, 2 or 4; lutv_kernel
+// for one token with other M) from this many bytes of 8-bit codes, the few-token kernel below.
+// Measured on GB300 (layer only, graph replay over 4 rotating layers, us, table / few-token):
+// T=1 2x8 33.6 MB 19.1 / 44.9, 8.4 MB 8.8-9.2 / 12.4-13.3, 4.2 MB 8.7 / 8.2-8.8, 0.7 MB
+// 10.3 / 4.1; T=2 2x8 33.6 MB 23.8 / 62.0, 8.4 MB 12.8-14.3 / 17.4-17.5, 4.2 MB 9.2 / 9.8;
+// T=4 2x8 33.6 MB 44.5 / 126.5, 4.2 MB 12.8 / 14.4; T=1 1x8 16.8 MB 13.3 / 33.5; T=1 4x8
+// 67.1 MB 36.4 / 198; T=4 4x8 67.1 MB 101 / 283.
+constexpr size_t kLutAutoMinCodeBytes = 6u << 20;
 
 int resolve_linear_path(int path, int T, int B, int N = 0, int K = 0, int M = 0) {
   const int m_tiles = (T + aq::kBM - 1) / aq::kBM;
@@ -1211,6 +1230,7 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     lpar.G = K / 8;
     lpar.chunks = lp.chunks;
     lpar.rows_per_cta = lp.rows_per_cta;
+    lpar.ctas = std::min(lp.ctas, sm_count());
     cudaError_t e;
     {
       ProfScope ps(kProfLutGather, st);
@@ -1230,7 +1250,8 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     rpar.partial = lpar.partial;
     {
       ProfScope ps(kProfSplitK, st);
-      e = aq::launch_splitk_reduce(rpar, lp.chunks, st);
+      e = lp.vec == 2 ? aq::launch_lut_reduce(rpar, lp.chunks, st)
+                      : aq::launch_splitk_reduce(rpar, lp.chunks, st);
     }
     if (e != cudaSuccess) return cuda_status(e, "LUT reduce launch");
     return ok();

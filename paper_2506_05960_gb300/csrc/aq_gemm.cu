@@ -1005,6 +1005,61 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
   }
 }
 
+// Sum of many partials over few outputs (the table path: up to hundreds of chunks, one to four
+// tokens): a block takes 32 output quads; warp j sums splits j, j + 8, j + 16, ... in order
+// (independent loads in flight), then warp 0 adds the eight warps' sums in order and applies
+// the epilogue.  The order is fixed, so results are reproducible.
+__global__ void __launch_bounds__(256) lut_reduce_kernel(const GemmParams p, int splits) {
+  __shared__ float4 part[8][32];
+  grid_dependency_wait();
+  allow_dependents();
+  const int qi = threadIdx.x & 31;
+  const int j = threadIdx.x >> 5;
+  const int64_t nq = static_cast<int64_t>(p.T) * (p.N / 4);
+  for (int64_t q0 = static_cast<int64_t>(blockIdx.x) * 32; q0 < nq;
+       q0 += static_cast<int64_t>(gridDim.x) * 32) {
+    const int64_t q = q0 + qi;
+    const int64_t t = q / (p.N / 4);
+    const int n = static_cast<int>(q - t * (p.N / 4)) * 4;
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    if (q < nq) {
+#pragma unroll 4
+      for (int s = j; s < splits; s += 8) {
+        const float4 v = *reinterpret_cast<const float4*>(
+            p.partial + (static_cast<int64_t>(s) * p.T + t) * p.N + n);
+        acc.x += v.x;
+        acc.y += v.y;
+        acc.z += v.z;
+        acc.w += v.w;
+      }
+    }
+    part[j][qi] = acc;
+    __syncthreads();
+    if (j == 0 && q < nq) {
+      float4 sum = part[0][qi];
+#pragma unroll
+      for (int w = 1; w < 8; ++w) {
+        const float4 v = part[w][qi];
+        sum.x += v.x;
+        sum.y += v.y;
+        sum.z += v.z;
+        sum.w += v.w;
+      }
+      store_out4(p, t, n, sum);
+    }
+    __syncthreads();
+  }
+}
+
+cudaError_t launch_lut_reduce(const GemmParams& p, int splits, cudaStream_t st) {
+  const int64_t nq = static_cast<int64_t>(p.T) * (p.N / 4);
+  int64_t blocks = (nq + 31) / 32;
+  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (blocks < 1) blocks = 1;
+  return launch_pdl(lut_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, p,
+                    splits);
+}
+
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st) {
   static std::atomic<int> configured_i8[64] = {};

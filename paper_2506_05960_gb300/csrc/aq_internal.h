@@ -81,13 +81,18 @@ struct LutParams {
   const __half* books;          // [M][256][8]
   float* partial;               // [chunks][T][N] partial sums
   int T, K, N, M;
-  int vec;                      // 1: lutv_kernel (whole K blocks per chunk, Tp = 1, 2 or 4
-                                // floats per entry); 0: lut_kernel
+  int vec;                      // 2: lutr_kernel (rotated, bank-conflict-free tables; Tp = 1,
+                                // 2 or 4; M = 1, 2 or 4); 1: lutv_kernel (one token, any M,
+                                // whole K blocks per chunk); 0: lut_kernel
   int Tp;                       // floats per table entry: vec: 1, 2 or 4 (>= T); else T
                                 // rounded up to 4, 8 or 16
   int J;                        // groups per chunk (vec: whole K blocks; else divides 8)
   int G;                        // K / 8
   int chunks, rows_per_cta;
+  int ctas;                     // lutr_kernel: grid size (CTAs share the (chunk, row block)
+                                // units in equal contiguous ranges)
+  unsigned lutr_table_off;      // lutr_kernel: dynamic shared-memory offset of the tables (set
+                                // by launch_lut so that they start at a 64 KB boundary)
 };
 
 // Parameters of the few-token kernel (linear layer, T <= 16, one pass, no workspace).
@@ -182,6 +187,9 @@ int gemm_a_stages(int BN);                   // TMEM A slots beside two BN-colum
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                         const GemmParams& p, int grid, cudaStream_t st);
 cudaError_t launch_splitk_reduce(const GemmParams& p, int splits, cudaStream_t st);
+// The table path's chunk partials [splits][T][N]: summed by split groups in parallel (a fixed
+// order), then the epilogue of launch_splitk_reduce.
+cudaError_t launch_lut_reduce(const GemmParams& p, int splits, cudaStream_t st);
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st);
 cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st);
 

@@ -5,14 +5,19 @@
 // The weight matrix is never decoded: each output row costs M table reads per
 // group instead of g multiply-adds, and the tables cost 2*g*M*2^B flops per
 // group and token.  Only 8-bit codes (256-row codebooks) are supported.
+// Three kernels, all writing fp32 partial sums per chunk of groups to the
+// workspace [chunks][T][N] (a reduction applies scale and bias):
+//   lutr_kernel  up to four tokens, M = 1, 2 or 4: bank-conflict-free rotated
+//                tables, codes streamed per lane with cp.async (the AUTO choice);
+//   lutv_kernel  one token, any other M;
+//   lut_kernel   up to sixteen tokens, any M (on request).
 //
-// One CTA owns a chunk of J consecutive groups (inside one packed 64-wide K
-// block) and a slice of output rows: it stages the chunk's int8 activations,
-// builds the chunk's tables for all tokens in shared memory, then each thread
-// walks its rows, reads the rows' codes with one contiguous load and
+// lut_kernel: one CTA owns a chunk of J consecutive groups (inside one packed
+// 64-wide K block) and a slice of output rows: it stages the chunk's int8
+// activations, builds the chunk's tables for all tokens in shared memory, then
+// each thread walks its rows, reads the rows' codes with one contiguous load and
 // gather-sums the table entries of all tokens (Tp floats per entry, 16-byte
-// shared loads).  Chunk partial sums go to the workspace [chunks][T][N] and
-// the split reduction applies scale and bias.
+// shared loads).
 #include <cstdint>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -113,36 +118,25 @@ __global__ void __launch_bounds__(256) lut_kernel(const LutParams p) {
   }
 }
 
-// Up to four tokens (TP = 1, 2 or 4 floats per table entry; T <= TP): the same order with
-// chunks of whole packed K blocks and at most 64 KB of tables, and one thread per output row:
-// per K block it reads the row's 8 * M codes as M contiguous 8-byte pieces (consecutive rows
-// consecutive, so a warp's loads are coalesced) and adds, per code, the entry's TP floats with
-// one vector load, in the fixed order (K block, group, codebook).  MM: M when 1, 2 or 4 (index
-// arithmetic known at compile time; then a chunk is 8 / (MM * TP) K blocks, at least one, and
-// the row's code pieces are loaded together, the next row's while this row's entries are
-// summed), or 0: any M, one token.
-template <int MM, int TP>
+// One token with any number of codebooks (the rotated-table kernel below takes M = 1, 2 or 4):
+// the same order with chunks of whole packed K blocks (two for M <= 4, else one) and one thread
+// per output row, which reads its codes per K block as M contiguous 8-byte pieces (consecutive
+// rows consecutive, so a warp's loads are coalesced) and adds one table entry per code, in the
+// fixed order (K block, group, codebook).
 __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
   extern __shared__ float4 lut_smem4[];
-  float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256][TP]
-  const int J = p.J, M = MM > 0 ? MM : p.M, T = p.T;
-  float* xs = L + static_cast<size_t>(J) * M * 256 * TP;       // [TP][J * 8]
+  float* L = reinterpret_cast<float*>(lut_smem4);              // [J][M][256]
+  const int J = p.J, M = p.M;
+  float* xs = L + static_cast<size_t>(J) * M * 256;            // [J * 8]
   grid_dependency_wait();
   allow_dependents();
   const int chunk = blockIdx.x;
   const int g0 = chunk * J;
   const int nj = min(J, p.G - g0);
-  const int width = J * 8;
-  for (int i = threadIdx.x; i < TP * width; i += blockDim.x) {
-    const int t = i / width;
-    const int e = i - t * width;
-    xs[i] = (t < T && e < nj * 8)
-                ? static_cast<float>(p.xq[static_cast<int64_t>(t) * p.K + g0 * 8 + e])
-                : 0.0f;
-  }
+  for (int e = threadIdx.x; e < J * 8; e += blockDim.x)
+    xs[e] = e < nj * 8 ? static_cast<float>(p.xq[g0 * 8 + e]) : 0.0f;
   __syncthreads();
-  // build: L[j][m][c][t] = sum_e x[t][g0 + j][e] * C^(m)[c][e], ascending e (zero past the last
-  // group and past the last token)
+  // build: L[j][m][c] = sum_e x[g0 + j][e] * C^(m)[c][e], ascending e (zero past the last group)
   const int entries = J * M * 256;
   for (int ent = threadIdx.x; ent < entries; ent += blockDim.x) {
     const int j = ent / (M * 256);
@@ -156,104 +150,332 @@ __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
       cw[2 * i] = f.x;
       cw[2 * i + 1] = f.y;
     }
-    float o[TP];
+    const float* xr = xs + j * 8;
+    float s = 0.0f;
 #pragma unroll
-    for (int t = 0; t < TP; ++t) {
-      const float* xr = xs + t * width + j * 8;
-      float s = 0.0f;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) s = fmaf(xr[e], cw[e], s);
-      o[t] = s;
-    }
-    if constexpr (TP == 1) {
-      L[ent] = o[0];
-    } else if constexpr (TP == 2) {
-      reinterpret_cast<float2*>(L)[ent] = make_float2(o[0], o[1]);
-    } else {
-      reinterpret_cast<float4*>(L)[ent] = make_float4(o[0], o[1], o[2], o[3]);
-    }
+    for (int e = 0; e < 8; ++e) s = fmaf(xr[e], cw[e], s);
+    L[ent] = s;
   }
   __syncthreads();
   const int kb0 = g0 >> 3;
   const int nkb = (nj + 7) >> 3;                  // packed K blocks holding this chunk's groups
   const int n_begin = blockIdx.y * p.rows_per_cta;
   const int n_end = min(p.N, n_begin + p.rows_per_cta);
-  if constexpr (MM > 0) {
-    constexpr int kBlocks = (MM * TP >= 8) ? 1 : 8 / (MM * TP);
-    constexpr int kPieces = kBlocks * MM;         // 8-byte code pieces of a row in a chunk
-    auto load = [&](int n, uint2 (&v)[kPieces]) {
+  for (int n = n_begin + threadIdx.x; n < n_end; n += blockDim.x) {
+    float acc = 0.0f;
+    for (int b = 0; b < nkb; ++b) {
+      const uint2* rec = reinterpret_cast<const uint2*>(
+          p.packed + (static_cast<int64_t>(kb0 + b) * p.N + n) * 8 * M);
+      const float* Lb = L + b * 8 * M * 256;      // tables of this K block's 8 groups
+      for (int pc = 0; pc < M; ++pc) {
+        const uint2 v = __ldcs(rec + pc);         // streamed once: no reuse in L1
 #pragma unroll
-      for (int b = 0; b < kBlocks; ++b) {
-        const uint2* rec = reinterpret_cast<const uint2*>(
-            p.packed + (static_cast<int64_t>(kb0 + b) * p.N + n) * 8 * MM);
-#pragma unroll
-        for (int pc = 0; pc < MM; ++pc)
-          v[b * MM + pc] = b < nkb ? __ldcs(rec + pc) : make_uint2(0u, 0u);
-      }
-    };
-    uint2 cur[kPieces], nxt[kPieces];
-    int n = n_begin + threadIdx.x;
-    if (n < n_end) load(n, cur);
-    for (; n < n_end; n += blockDim.x) {
-      if (n + static_cast<int>(blockDim.x) < n_end) load(n + blockDim.x, nxt);
-      float acc[TP];
-#pragma unroll
-      for (int t = 0; t < TP; ++t) acc[t] = 0.0f;
-#pragma unroll
-      for (int b = 0; b < kBlocks; ++b) {
-        if (b < nkb) {
-          const float* Lb = L + b * 8 * MM * 256 * TP;   // tables of this K block's 8 groups
-#pragma unroll
-          for (int pc = 0; pc < MM; ++pc) {
-            const uint2 v = cur[b * MM + pc];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              // byte pc*8 + k of the record is group (pc*8 + k) / MM, codebook (pc*8 + k) % MM,
-              // and its entry is ((pc*8 + k) * 256 + code) of this K block's [8][MM][256]
-              const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
-              const float* e = Lb + ((pc * 8 + k) * 256 + code) * TP;
-              if constexpr (TP == 1) {
-                acc[0] += e[0];
-              } else if constexpr (TP == 2) {
-                const float2 w = *reinterpret_cast<const float2*>(e);
-                acc[0] += w.x;
-                acc[1] += w.y;
-              } else {
-                const float4 w = *reinterpret_cast<const float4*>(e);
-                acc[0] += w.x;
-                acc[1] += w.y;
-                acc[2] += w.z;
-                acc[3] += w.w;
-              }
-            }
-          }
+        for (int k = 0; k < 8; ++k) {
+          // byte pc*8 + k of the record is group (pc*8 + k) / M, codebook (pc*8 + k) % M
+          const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
+          acc += Lb[(pc * 8 + k) * 256 + code];
         }
       }
-#pragma unroll
-      for (int t = 0; t < TP; ++t)
-        if (t < T) p.partial[(static_cast<int64_t>(chunk) * T + t) * p.N + n] = acc[t];
-#pragma unroll
-      for (int i = 0; i < kPieces; ++i) cur[i] = nxt[i];
     }
-  } else {
-    static_assert(MM > 0 || TP == 1, "any M: one token only");
-    for (int n = n_begin + threadIdx.x; n < n_end; n += blockDim.x) {
-      float acc = 0.0f;
-      for (int b = 0; b < nkb; ++b) {
-        const uint2* rec = reinterpret_cast<const uint2*>(
-            p.packed + (static_cast<int64_t>(kb0 + b) * p.N + n) * 8 * M);
-        const float* Lb = L + b * 8 * M * 256;      // tables of this K block's 8 groups
-        for (int pc = 0; pc < M; ++pc) {
-          const uint2 v = __ldcs(rec + pc);         // streamed once: no reuse in L1
+    p.partial[static_cast<int64_t>(chunk) * p.N + n] = acc;
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Rotated-table kernel: one to four tokens, M = 1, 2 or 4 codebooks of 2^8 entries.  The table
+// order of App. A.1 (Eq. A5 -> A6) with tables laid out so that the lanes of a warp never
+// collide on a shared-memory bank, whatever the codes:
+//  * a chunk is NT = 32 / TP consecutive bytes of every row's code stream (the row's packed
+//    records of consecutive K blocks, 8 * M bytes each: stream byte b is group b / M, codebook
+//    b % M), i.e. NT tables, one per (group, codebook);
+//  * entry e of table t (TP floats, one per token) is stored at word e * 64 + t * TP and again
+//    at word e * 64 + (t + NT) * TP: 256 rows of 64 words, 64 KB, placed at shared-window
+//    address kLutrTableAddr (a multiple of 64 KB);
+//  * lane l owns one output row; at step s (0 <= s < NT) it adds the entry of table
+//    (l' + s) mod NT, l' = l mod NT, read from slot l' + s < 2 NT (the copy spares the wrap).
+//    The lanes of one shared-memory phase (32 / TP lanes, distinct l') read TP-word slots
+//    (l' + s) * TP mod 32 that are pairwise distinct: one conflict-free wavefront per phase;
+//  * the row's NT code bytes are rotated by l' bytes once (selects and funnel shifts), so step
+//    s takes byte s of the rotated words, and one byte permute assembles the entry's whole
+//    shared address: kLutrTableAddr | code << 8 | l' * TP * 4 (plus s * TP * 4 as the load's
+//    offset).
+// Each lane sums its row's entries in its own rotated order (fixed per lane: deterministic).
+// Work: (chunk, 32-row block) units in chunk-major order, one contiguous equal range per CTA
+// (one CTA per SM): a CTA builds the tables of each chunk its range reaches (one or two) from
+// codebooks staged once in shared memory, and writes fp32 partial sums [chunk][T][N]; the
+// reduction sums the chunks and applies the epilogue.
+// Code streaming: every lane copies its own row's NT code bytes with cp.async into a private
+// ring of kLutrLaneRing bytes (kStages row blocks ahead, across chunk boundaries) and reads them
+// back after waiting for its own copies: each lane touches only what it copied, so no barrier
+// is needed, and a warp keeps several row blocks of codes in flight.
+constexpr int kLutrThreads = 1024;
+constexpr int kLutrLaneRing = 96;                // bytes of code ring per lane
+constexpr uint32_t kLutrTableAddr = 0x20000u;    // shared-window address of the tables
+
+template <int MM, int TP>
+struct LutrShape {
+  static constexpr int NT = 32 / TP;             // tables (code bytes of a row) per chunk
+  static constexpr int NW = NT / 4;              // 32-bit code words of a row per chunk
+  static constexpr int R = 8 * MM;               // bytes of one packed record (row, K block)
+  static constexpr int GC = NT / MM;             // groups per chunk
+  static constexpr int PB = NT < R ? NT : R;
+  static constexpr int P = PB < 16 ? PB : 16;    // bytes per code copy
+  static constexpr int NP = NT / P;              // copies per row and chunk
+  static constexpr int kStages = kLutrLaneRing / NT;
+  static constexpr uint32_t kRingBytes = static_cast<uint32_t>(kLutrThreads) * kLutrLaneRing;
+  static constexpr uint32_t kStageBytes = static_cast<uint32_t>(kLutrThreads) * NT;
+  static constexpr uint32_t kBookOff = kRingBytes;
+  static constexpr uint32_t kXsOff = kBookOff + MM * 256 * 16;
+  static constexpr uint32_t kFront = kXsOff + (TP * GC * 8 * 4 + 15) / 16 * 16;
+  static constexpr uint32_t kTableBytes = 256 * 64 * 4;
+};
+
+__device__ __forceinline__ void cp_async_zfill(uint32_t dst, const void* src, bool valid,
+                                               int bytes) {
+  const int n = valid ? bytes : 0;               // 0: nothing is read, the bytes are zeroed
+  if (bytes == 16)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
+                 : "memory");
+  else
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(n)
+                 : "memory");
+}
+
+template <int MM, int TP>
+__global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p) {
+  using S = LutrShape<MM, TP>;
+  constexpr int NT = S::NT, NW = S::NW, R = S::R, GC = S::GC, P = S::P, NP = S::NP;
+  constexpr int D = S::kStages;
+  extern __shared__ float4 lut_smem4[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(lut_smem4);
+  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+  // the host sized the allocation for this base; any other layout would misplace the tables
+  if (sbase + p.lutr_table_off != kLutrTableAddr || p.lutr_table_off < S::kFront) return;
+  uint4* sbook = reinterpret_cast<uint4*>(smem + S::kBookOff);                  // [MM][256]
+  float* xs = reinterpret_cast<float*>(smem + S::kXsOff);                       // [TP][GC*8]
+  float* L = reinterpret_cast<float*>(smem + p.lutr_table_off);                 // [256][64]
+  grid_dependency_wait();
+  allow_dependents();
+  const int N = p.N, T = p.T;
+  const int KB = (p.K + 63) / 64;
+  const int64_t stream_bytes = static_cast<int64_t>(KB) * R;   // code bytes of a row
+  const int nrb = (N + 31) / 32;
+  const int64_t U = static_cast<int64_t>(p.chunks) * nrb;
+  const int64_t u0 = U * blockIdx.x / gridDim.x;
+  const int64_t u1 = U * (blockIdx.x + 1) / gridDim.x;
+  if (u0 >= u1) return;
+  for (int i = threadIdx.x; i < MM * 256; i += blockDim.x)
+    sbook[i] = reinterpret_cast<const uint4*>(p.books)[i];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nwarps = blockDim.x >> 5;
+  const int c_first = static_cast<int>(u0 / nrb);
+  const int rb_first = static_cast<int>(u0 % nrb);
+  const int c_last = static_cast<int>((u1 - 1) / nrb);
+  const int rb_last_end = static_cast<int>((u1 - 1) % nrb) + 1;
+  const int li = lane & (NT - 1);
+  // entry address = kLutrTableAddr | code << 8 | lane_off (bytes 2, 0 of lane_reg; byte 1 from
+  // the code)
+  const uint32_t lane_reg = kLutrTableAddr | static_cast<uint32_t>(li * TP * 4);
+
+  // ---- producer: this warp's row blocks, chunk by chunk (rb_begin(c) + warp, + nwarps, ...),
+  // copied kStages items ahead of the lookups; every lane of the warp walks the same sequence
+  int pc = c_first, prb = rb_first + warp;       // next item to copy
+  const uint8_t* psrc = p.packed;                // its piece-0 source for this lane's row
+  uint32_t pmask = 0;                            // its pieces inside the code stream
+  auto prod_settle = [&]() {
+    while (pc <= c_last && prb >= (pc == c_last ? rb_last_end : nrb)) {
+      ++pc;
+      prb = warp;
+    }
+    if (pc <= c_last) {
+      const int64_t b0 = static_cast<int64_t>(pc) * NT;
+      psrc = p.packed + ((b0 / R) * N + prb * 32 + lane) * R + (b0 % R);
+      pmask = 0;
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t code = ((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu;
-            acc += Lb[(pc * 8 + k) * 256 + code];
+      for (int q = 0; q < NP; ++q)
+        if (b0 + q * P < stream_bytes) pmask |= 1u << q;
+    }
+  };
+  prod_settle();
+  const uint32_t ring_lane = sbase + static_cast<uint32_t>(threadIdx.x * P);
+  uint32_t wr = 0;                               // write offset of the next stage
+  auto produce = [&]() {
+    if (pc <= c_last) {
+      const bool row_ok = prb * 32 + lane < N;
+#pragma unroll
+      for (int q = 0; q < NP; ++q) {
+        const bool ok = row_ok && ((pmask >> q) & 1u);
+        // piece q: q * P bytes further in the stream: the next record, or further in this one
+        const int64_t poff = static_cast<int64_t>((q * P) / R) * N * R + (q * P) % R;
+        cp_async_zfill(ring_lane + wr + static_cast<uint32_t>(q * kLutrThreads * P),
+                       ok ? psrc + poff : p.packed, ok, P);
+      }
+      prb += nwarps;
+      if (prb < (pc == c_last ? rb_last_end : nrb))
+        psrc += static_cast<int64_t>(nwarps) * 32 * R;
+      else
+        prod_settle();
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");   // empty past the end: counts stay
+    wr += S::kStageBytes;
+    if (wr == S::kRingBytes) wr = 0;
+  };
+#pragma unroll 1
+  for (int d = 0; d < D; ++d) produce();
+  uint32_t rd = 0;                               // read offset of the oldest stage
+
+  for (int c = c_first; c <= c_last; ++c) {
+    const int g0 = c * GC;                       // first group of the chunk
+    // ---- the chunk's tables (after every warp is done with the previous chunk's)
+    __syncthreads();
+    for (int i = threadIdx.x; i < TP * GC * 8; i += blockDim.x) {
+      const int tt = i / (GC * 8);
+      const int k = g0 * 8 + (i - tt * GC * 8);
+      xs[i] = (tt < T && k < p.K) ? static_cast<float>(p.xq[static_cast<int64_t>(tt) * p.K + k])
+                                  : 0.0f;
+    }
+    __syncthreads();
+    {
+      const int t = threadIdx.x % NT;
+      const int j = t / MM;                      // group within the chunk
+      const bool live = g0 + j < p.G;            // groups past K (zero-padded codes): 0
+      float xr[TP][8];
+#pragma unroll
+      for (int tt = 0; tt < TP; ++tt)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) xr[tt][e] = xs[tt * GC * 8 + j * 8 + e];
+      const uint4* book = sbook + (t % MM) * 256;
+      for (int e = threadIdx.x / NT; e < 256; e += blockDim.x / NT) {
+        float o[TP];
+#pragma unroll
+        for (int tt = 0; tt < TP; ++tt) o[tt] = 0.0f;
+        if (live) {
+          // L[e] = sum_u x[g0 + j][u] * C^(m)[e][u], ascending u (the other table kernels'
+          // arithmetic)
+          const uint4 raw = book[e];
+          const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+          float cw[8];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = __half22float2(h2[i]);
+            cw[2 * i] = f.x;
+            cw[2 * i + 1] = f.y;
+          }
+#pragma unroll
+          for (int tt = 0; tt < TP; ++tt) {
+            float s = 0.0f;
+#pragma unroll
+            for (int v = 0; v < 8; ++v) s = fmaf(xr[tt][v], cw[v], s);
+            o[tt] = s;
           }
         }
+        float* d0 = L + e * 64 + t * TP;
+        float* d1 = d0 + NT * TP;
+        if constexpr (TP == 1) {
+          d0[0] = o[0];
+          d1[0] = o[0];
+        } else if constexpr (TP == 2) {
+          *reinterpret_cast<float2*>(d0) = make_float2(o[0], o[1]);
+          *reinterpret_cast<float2*>(d1) = make_float2(o[0], o[1]);
+        } else {
+          *reinterpret_cast<float4*>(d0) = make_float4(o[0], o[1], o[2], o[3]);
+          *reinterpret_cast<float4*>(d1) = make_float4(o[0], o[1], o[2], o[3]);
+        }
       }
-      p.partial[static_cast<int64_t>(chunk) * p.N + n] = acc;
     }
+    __syncthreads();
+    const int rb_e = c == c_last ? rb_last_end : nrb;
+    float* pout = p.partial + static_cast<int64_t>(c) * T * N + lane;
+    for (int rb = (c == c_first ? rb_first : 0) + warp; rb < rb_e; rb += nwarps) {
+      // this row block's codes: the oldest of this lane's copy groups
+      asm volatile("cp.async.wait_group %0;" ::"n"(D - 1) : "memory");
+      uint32_t r[NW];
+#pragma unroll
+      for (int q = 0; q < NP; ++q) {
+        const uint32_t a = ring_lane + rd + static_cast<uint32_t>(q * kLutrThreads * P);
+        if constexpr (P == 16) {
+          asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(r[4 * q]), "=r"(r[4 * q + 1]), "=r"(r[4 * q + 2]), "=r"(r[4 * q + 3])
+                       : "r"(a) : "memory");
+        } else {
+          asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];"
+                       : "=r"(r[2 * q]), "=r"(r[2 * q + 1]) : "r"(a) : "memory");
+        }
+      }
+      // rotate the row's code bytes left by li: byte s of r is stream byte (s + li) mod NT
+      const int qw = li >> 2;
+#pragma unroll
+      for (int d = 1; d < NW; d <<= 1) {
+        uint32_t tmp[NW];
+#pragma unroll
+        for (int k = 0; k < NW; ++k) tmp[k] = (qw & d) ? r[(k + d) % NW] : r[k];
+#pragma unroll
+        for (int k = 0; k < NW; ++k) r[k] = tmp[k];
+      }
+      {
+        const uint32_t sh = static_cast<uint32_t>(8 * (li & 3));
+        uint32_t tmp[NW];
+#pragma unroll
+        for (int k = 0; k < NW; ++k) tmp[k] = __funnelshift_r(r[k], r[(k + 1) % NW], sh);
+#pragma unroll
+        for (int k = 0; k < NW; ++k) r[k] = tmp[k];
+      }
+      // the stage is free again (its words are in registers and used above): refill it with
+      // this warp's item kStages ahead
+      produce();
+      rd += S::kStageBytes;
+      if (rd == S::kRingBytes) rd = 0;
+      float acc0[TP], acc1[TP];
+#pragma unroll
+      for (int tt = 0; tt < TP; ++tt) acc0[tt] = acc1[tt] = 0.0f;
+#pragma unroll
+      for (int s = 0; s < NT; ++s) {
+        const uint32_t addr = __byte_perm(r[s >> 2], lane_reg, 0x7604u | ((s & 3) << 4)) +
+                              static_cast<uint32_t>(s * TP * 4);
+        float* acc = (s & 1) ? acc1 : acc0;
+        if constexpr (TP == 1) {
+          float v;
+          asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+          acc[0] += v;
+        } else if constexpr (TP == 2) {
+          float v0, v1;
+          asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v0), "=f"(v1) : "r"(addr));
+          acc[0] += v0;
+          acc[1] += v1;
+        } else {
+          float v0, v1, v2, v3;
+          asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+              : "=f"(v0), "=f"(v1), "=f"(v2), "=f"(v3) : "r"(addr));
+          acc[0] += v0;
+          acc[1] += v1;
+          acc[2] += v2;
+          acc[3] += v3;
+        }
+      }
+      if (rb * 32 + lane < N) {
+#pragma unroll
+        for (int tt = 0; tt < TP; ++tt)
+          if (tt < T) pout[static_cast<int64_t>(tt) * N + rb * 32] = acc0[tt] + acc1[tt];
+      }
+    }
+  }
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+// Dynamic shared memory of lutr_kernel for a window whose dynamic part starts at `base`: the
+// ring, codebooks and activations, then the tables at kLutrTableAddr.  0 if they do not fit.
+static uint32_t lutr_front(int TP, int M) {
+  switch (TP * 16 + M) {
+    case 16 + 1: return LutrShape<1, 1>::kFront;
+    case 16 + 2: return LutrShape<2, 1>::kFront;
+    case 16 + 4: return LutrShape<4, 1>::kFront;
+    case 32 + 1: return LutrShape<1, 2>::kFront;
+    case 32 + 2: return LutrShape<2, 2>::kFront;
+    case 32 + 4: return LutrShape<4, 2>::kFront;
+    case 64 + 1: return LutrShape<1, 4>::kFront;
+    case 64 + 2: return LutrShape<2, 4>::kFront;
+    case 64 + 4: return LutrShape<4, 4>::kFront;
+    default: return 0;
   }
 }
 
@@ -262,33 +484,49 @@ size_t lut_smem_bytes(int J, int M, int Tp, int T) {
 }
 
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {
-  if (p.vec) {
-    // lutv_kernel: whole K blocks per chunk, TP = p.Tp floats per entry
-    static std::atomic<int> c11[64] = {}, c21[64] = {}, c41[64] = {}, c01[64] = {}, c12[64] = {},
-                            c22[64] = {}, c42[64] = {}, c14[64] = {}, c24[64] = {}, c44[64] = {};
-    const size_t bytes = static_cast<size_t>(p.J) * p.M * 256 * p.Tp * 4 +
-                         static_cast<size_t>(p.Tp) * p.J * 8 * 4;
-    const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
-    const dim3 grid(p.chunks, n_slices);
+  if (p.vec == 2) {
+    // lutr_kernel: p.Tp floats per entry, p.ctas CTAs of 1024 threads
+    static std::atomic<int> c11[64] = {}, c21[64] = {}, c41[64] = {}, c12[64] = {}, c22[64] = {},
+                            c42[64] = {}, c14[64] = {}, c24[64] = {}, c44[64] = {};
+    // the dynamic window starts after the per-block reserved shared memory (no static shared
+    // memory in this kernel): the tables go at kLutrTableAddr, the rest before them
+    int dev = 0, reserved = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess)
+      e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev);
+    if (e != cudaSuccess) return e;
+    const uint32_t front = lutr_front(p.Tp, p.M);
+    if (front == 0 || static_cast<uint32_t>(reserved) + front > kLutrTableAddr)
+      return cudaErrorInvalidConfiguration;
+    LutParams q = p;
+    q.lutr_table_off = kLutrTableAddr - static_cast<uint32_t>(reserved);
+    const size_t bytes = q.lutr_table_off + 256 * 64 * 4;
     auto go = [&](auto kernel, std::atomic<int> (&conf)[64]) -> cudaError_t {
       const cudaError_t se = ensure_dynamic_smem(kernel, bytes, conf);
       if (se != cudaSuccess) return se;
-      return launch_pdl(kernel, grid, dim3(256), bytes, st, p);
+      return launch_pdl(kernel, dim3(static_cast<unsigned>(q.ctas)), dim3(1024), bytes, st, q);
     };
-    const int mm = (p.M == 1 || p.M == 2 || p.M == 4) ? p.M : 0;
-    switch (p.Tp * 16 + mm) {
-      case 16 + 1: return go(lutv_kernel<1, 1>, c11);
-      case 16 + 2: return go(lutv_kernel<2, 1>, c21);
-      case 16 + 4: return go(lutv_kernel<4, 1>, c41);
-      case 16 + 0: return go(lutv_kernel<0, 1>, c01);
-      case 32 + 1: return go(lutv_kernel<1, 2>, c12);
-      case 32 + 2: return go(lutv_kernel<2, 2>, c22);
-      case 32 + 4: return go(lutv_kernel<4, 2>, c42);
-      case 64 + 1: return go(lutv_kernel<1, 4>, c14);
-      case 64 + 2: return go(lutv_kernel<2, 4>, c24);
-      case 64 + 4: return go(lutv_kernel<4, 4>, c44);
+    switch (p.Tp * 16 + p.M) {
+      case 16 + 1: return go(lutr_kernel<1, 1>, c11);
+      case 16 + 2: return go(lutr_kernel<2, 1>, c21);
+      case 16 + 4: return go(lutr_kernel<4, 1>, c41);
+      case 32 + 1: return go(lutr_kernel<1, 2>, c12);
+      case 32 + 2: return go(lutr_kernel<2, 2>, c22);
+      case 32 + 4: return go(lutr_kernel<4, 2>, c42);
+      case 64 + 1: return go(lutr_kernel<1, 4>, c14);
+      case 64 + 2: return go(lutr_kernel<2, 4>, c24);
+      case 64 + 4: return go(lutr_kernel<4, 4>, c44);
       default: return cudaErrorInvalidConfiguration;
     }
+  }
+  if (p.vec == 1) {
+    // lutv_kernel: one token, whole K blocks per chunk
+    static std::atomic<int> conf[64] = {};
+    const size_t bytes = static_cast<size_t>(p.J) * p.M * 256 * 4 + static_cast<size_t>(p.J) * 8 * 4;
+    const int n_slices = (p.N + p.rows_per_cta - 1) / p.rows_per_cta;
+    const cudaError_t se = ensure_dynamic_smem(lutv_kernel, bytes, conf);
+    if (se != cudaSuccess) return se;
+    return launch_pdl(lutv_kernel, dim3(p.chunks, n_slices), dim3(256), bytes, st, p);
   }
   static std::atomic<int> configured[64] = {};
   const size_t bytes = lut_smem_bytes(p.J, p.M, p.Tp, p.T);

@@ -281,14 +281,15 @@ def test_noalloc_argument_checks_before_any_cuda_call(lib):
 
 def test_auto_path_rules(lib):
     """AUTO's choices for a linear layer (no device access): up to four tokens on a layer with
-    at least 12 MB of 8-bit codes take the vector-table kernel (one token with any M, more with
-    1, 2 or 4 codebooks); few tokens otherwise the few-token kernel; one row tile the fused decode; more the dense path.  fp16 activations choose the
+    at least 6 MB of 8-bit codes take the table path (one token with any M, more with 1, 2 or 4
+    codebooks); few tokens otherwise the few-token kernel; one row tile the fused decode; more the dense path.  fp16 activations choose the
     shared-memory A form only where its plan has no K split and a wider N tile."""
     import paper_2506_05960_gb300 as aq
     LUT, FEW, FUSED, DENSE = 3, 4, 2, 1
     assert aq.aq_linear_plan(1, 8192, 16384, 8, 2, 8)["path"] == LUT       # 33.6 MB of codes
     assert aq.aq_linear_plan(1, 8192, 16384, 8, 1, 8)["path"] == LUT       # 16.8 MB
-    assert aq.aq_linear_plan(1, 4096, 8192, 8, 2, 8)["path"] == FEW        # 8.4 MB
+    assert aq.aq_linear_plan(1, 4096, 8192, 8, 2, 8)["path"] == LUT        # 8.4 MB
+    assert aq.aq_linear_plan(1, 2048, 8192, 8, 2, 8)["path"] == FEW        # 4.2 MB
     assert aq.aq_linear_plan(1, 8192, 16384, 8, 1, 16)["path"] == FEW      # 16-bit codes
     assert aq.aq_linear_plan(2, 8192, 16384, 8, 2, 8)["path"] == LUT       # two tokens
     assert aq.aq_linear_plan(4, 8192, 16384, 8, 4, 8)["path"] == LUT       # four, 4x8

@@ -84,11 +84,14 @@ def test_lut_path_selection():
     (3, 960, 2880, 2),       # four floats per entry, one token unused
     (4, 4096, 4096, 2),
     (4, 208, 264, 1),
-    (4, 1024, 512, 4),       # 128 KB of tables: one CTA per SM
+    (4, 1024, 512, 4),       # a chunk is a quarter of a packed record
+    (1, 8192, 4104, 2),      # 129 CTAs whose row-block ranges cross chunk boundaries; 8-row tail
+    (2, 4096, 1032, 1),
 ])
 def test_lut_vector_tables(T, K, N, M):
-    """Up to four tokens with whole K blocks per chunk and 1, 2 or 4 floats per table entry
-    (lutv_kernel), against the oracle's decode order and table order, fp16 and fp32 outputs."""
+    """Up to four tokens: the rotated-table kernel (M = 1, 2 or 4; 1, 2 or 4 floats per entry)
+    and the one-token kernel for other M, against the oracle's decode order and table order, fp16
+    and fp32 outputs."""
     import paper_2506_05960_gb300 as aq
     inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=8, cb_std=0.05 / M ** 0.5),
                       seed=300 + T + K + N + M)
