@@ -75,7 +75,7 @@ typedef enum aq_dtype {
 
 typedef enum aq_path {
   AQ_PATH_AUTO  = 0,  /* library picks from (T, N, K, M, B): linear layers with T <= 4 take
-                         AQ_PATH_LUT when B = 8, the codes fill at least 12 MB and (T == 1
+                         AQ_PATH_LUT when B = 8, the codes fill at least 6 MB and (T == 1
                          or M is 1, 2 or 4), else AQ_PATH_FEW_TOKENS; one 128-row tile of
                          tokens AQ_PATH_FUSED; more AQ_PATH_DENSE (a convolution: FUSED for
                          one tile with g = 8, else DENSE)                                  */
@@ -84,9 +84,10 @@ typedef enum aq_path {
   AQ_PATH_FUSED = 2,  /* decode inside the GEMM into shared memory (codebooks in shared
                          memory, or in L2 for 2^16-entry books); W-hat never touches HBM  */
   AQ_PATH_LUT   = 3,  /* lookup-table order of App. A.1 (Eq. A5-A6): per token and group,
-                         the dot product with every codeword, then a gather-sum by code;
-                         linear layers with T <= 16 and B = 8; needs a workspace for the
-                         per-chunk partial sums                                            */
+                         the dot product with every codeword, then a gather-sum by code
+                         (up to four tokens with M = 1, 2 or 4: bank-conflict-free rotated
+                         tables); linear layers with T <= 16 and B = 8; needs a workspace
+                         for the per-chunk partial sums                                    */
   AQ_PATH_FEW_TOKENS = 4, /* linear layers with T <= 16: one kernel streams each row's codes
                          once, decodes in registers and dots with every token on CUDA
                          cores; no workspace                                              */
