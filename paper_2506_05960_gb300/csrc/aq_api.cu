@@ -647,6 +647,17 @@ int run_gemm(const CUtensorMap& mapA, aq::GemmParams p, const Plan& pl, const vo
   p.a_col = pl.a_col;
   p.cluster = pl.cluster;
   p.epi_warps = pl.epi_warps;
+  // The shared-memory A form takes 12 epilogue warps (three per TMEM lane quarter) where the
+  // epilogue, not the mainloop, bounds a tile -- the 8-bit activation rule of the _q8 / _ex
+  // code outputs costs about four times the fp16 epilogue's instructions per value, and a tile
+  // of at most 8 K blocks has a shorter mainloop than its epilogue -- when the extra staging
+  // costs no pipeline stage.  Measured on GB300 (T=65536, K=384, N=1152, N tile 256, 8 warps):
+  // fp16 output 66 us, int8 codes 110 us.
+  // (8 epilogue warps imply fp16 / int8 staging: no fp32 output, no partials)
+  if (pl.a16 && !fused && !pl.cluster && pl.epi_warps == 8 &&
+      (p.out_q8 || pl.kb_per_split <= 8) &&
+      aq::gemm_max_stages(pl.BN, false, 0, 0, 12, true, pl.sb) >= pl.stages)
+    p.epi_warps = 12;
   p.partial = (pl.splits > 1 && !pl.cluster) ? partial : nullptr;
   const int T = p.T, N = p.N, K = p.K;
   int r;

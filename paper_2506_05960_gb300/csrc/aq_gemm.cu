@@ -56,9 +56,9 @@ constexpr int kASlotCols = kStageBlocks * 32;   // TMEM columns of one fp16 A sl
 constexpr int kEpiBuf32 = 4096;                 // one 32 x 32 fp32 output box (128-byte rows)
 constexpr int kEpiBuf16 = 2048;                 // one 32 x 32 fp16 output box (64-byte rows)
 // Epilogue staging per warp: 4 warps keep two output boxes and the scale/bias of all BN
-// columns each; 8 warps (two per lane quarter, alternate 32-column chunks) keep one box
-// and the scale/bias of their own columns, so both take the same shared memory.
-__host__ __device__ constexpr int epi_out_bufs(int epi_warps) { return epi_warps == 8 ? 1 : 2; }
+// columns each; 8 or 12 warps (two or three per lane quarter, taking its 32-column chunks in
+// turn) keep one box and the scale/bias of their own columns.
+__host__ __device__ constexpr int epi_out_bufs(int epi_warps) { return epi_warps >= 8 ? 1 : 2; }
 // Columns of scale/bias a warp keeps: its 32-column chunks of a BN-wide tile, compacted.
 __host__ __device__ constexpr int epi_scale_cols(int epi_warps, int BN) {
   return ((BN + 31) / 32 + epi_warps / 4 - 1) / (epi_warps / 4) * 32;
@@ -377,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* bring = smem;
   uint8_t* aring = bring + S * b_stage;
   uint8_t* epi = aring + S * a_stage;
-  const int EW = p.epi_warps;                  // 4, or 8 (two per TMEM lane quarter)
+  const int EW = p.epi_warps;                  // 4, 8 or 12 (1-3 per TMEM lane quarter)
   const int epi_first = kA16 ? 2 : 6;          // first epilogue warp
   float* sscale = reinterpret_cast<float*>(epi + EW * epi_out_bufs(EW) * epi_buf);
   uint4* sbook = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sscale) +
@@ -1079,8 +1079,10 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
   auto kernel = a16 ? aq_gemm_kernel<true> : aq_gemm_kernel<false>;
   const cudaError_t se = ensure_dynamic_smem(kernel, bytes, a16 ? configured_a16 : configured_i8);
   if (se != cudaSuccess) return se;
-  // the decoder warps (10..15) exist only on the fused path
-  if (p.epi_warps != 4 && !(p.epi_warps == 8 && !p.fused && p.BN >= 64))
+  // the decoder warps (10..15) exist only on the fused path; 12 epilogue warps only in the
+  // shared-memory A form (2 + 12 warps within the kernel's thread bound)
+  if (p.epi_warps != 4 && !(p.epi_warps == 8 && !p.fused && p.BN >= 64) &&
+      !(p.epi_warps == 12 && a16 && p.BN >= 64))
     return cudaErrorInvalidConfiguration;
   // fp16 A form: producer, MMA and epilogue warps
   const int threads = a16 ? 32 * (2 + p.epi_warps) : (p.fused ? kThreads : 32 * (6 + p.epi_warps));
