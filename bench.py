@@ -56,16 +56,14 @@ HEADLINE = "AQ linear qkv projection T=4096 K=960 N=2880 W2A8 (2x8 codebooks, g=
 METRIC = "AQ layer dense-equivalent TFLOP/s (2*T*N*K / step time)"
 NSETS = 8
 
-# DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from
-# `ncu --set full` capture of one launch (dram__bytes_read.sum + dram__bytes_write.sum;
-# summary in profiles/aq_gemm_kernel_a16_qkv_T4096_K960_N2880.md); reported only while the
-# kernel sources are the ones it was measured on (re-captured with the fp16-code epilogue
-# branch: dram__bytes_read.sum + dram__bytes_write.sum of one launch; the key was refreshed
-# after header changes for other kernels that left the GEMM's code byte-identical apart from
-# line information, checked by comparing the hashes of the GEMM kernels' code sections).
+# DRAM traffic of one launch of the tensor-core GEMM on the headline workload, from an ncu
+# capture of one launch (dram__bytes_read.sum + dram__bytes_write.sum; summary in
+# profiles/aq_gemm_kernel_a16_qkv_T4096_K960_N2880.md); reported only while the kernel sources
+# hash to the ones it was captured on (the key is refreshed either by a new capture or, after
+# changes elsewhere in these files, once the GEMM kernels' code sections hash the same).
 KERNEL_SOURCES = ["paper_2506_05960_gb300/csrc/aq_gemm.cu", "paper_2506_05960_gb300/csrc/aq_ptx.cuh",
                   "paper_2506_05960_gb300/csrc/aq_quant.cuh", "paper_2506_05960_gb300/csrc/aq_internal.h"]
-TRAFFIC = {"bytes": 13476096, "sources_sha": "f3be9d829af10fec"}
+TRAFFIC = {"bytes": 13476352, "sources_sha": "96bf5ad692151233"}
 
 
 def sources_sha() -> str:
