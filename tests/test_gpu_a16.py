@@ -203,3 +203,41 @@ def test_f16_quantizer_writes_codes_as_fp16():
     xq = O.quant_act(x16, s_x)
     assert np.array_equal(codes, xq.astype(np.float16))
     assert_close(y.cpu().numpy().astype(np.float64), O.layer_f64(dict(inp, xq=xq, s_x=s_x)), "f16")
+
+
+@pytest.mark.parametrize("BN", [64, 128, 192, 256])
+def test_a16_short_k_and_code_outputs(BN):
+    """Tiles of at most 8 K blocks, and the next layer's codes as output, run the shared-memory
+    A form with three epilogue warps per TMEM lane quarter (with N tile 64 one of the three has
+    no chunk).  fp16 output against the oracle; the int8 codes and the fp16 codes equal the
+    activation rule applied to the fp16 output, bit for bit."""
+    import torch
+    import paper_2506_05960_gb300 as aq
+    T, K, N = 700, 384, 976          # ragged row tile; a ragged N tile for every BN
+    inp, packed = _layer(T, K, N, seed=BN + 11)
+    s_out = 0.05
+    F16C, I8 = aq.AQ_DTYPE_F16_CODES, aq.AQ_DTYPE_I8
+    xh = dev(inp["xq"].astype(np.float16))
+    outs = {}
+    aq.aq_set_plan_override(BN, 1, 0)
+    try:
+        pl = aq.aq_linear_a16_plan(T, K, N, 8, 2, 8, AUTO)
+        assert pl["BN"] == BN and pl["a16"] == 1 and pl["splits"] == 1
+        y = _run_a16(aq, inp, packed, False)
+        for od in (I8, F16C):
+            wsb = aq.aq_linear_ex_workspace_size(F16C, T, K, N, 8, 2, 8, AUTO)
+            ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device="cuda")
+            yo = (torch.full((T, N), 99, dtype=torch.int8, device="cuda") if od == I8
+                  else poison((T, N), torch.float16))
+            aq.aq_linear_ex(xh, F16C, inp["s_x"], packed, dev(inp["codebooks"]),
+                            dev(inp["scale"]), dev(inp["bias"]), yo, od, s_out, T, K, N, 8, 2, 8,
+                            ws, wsb, AUTO)
+            torch.cuda.synchronize()
+            assert aq.aq_device_error() == 0
+            outs[od] = yo.cpu().numpy()
+    finally:
+        aq.aq_set_plan_override()
+    assert_close(y.astype(np.float64), O.layer_f64(inp), (BN, T, K, N))
+    q = O.quant_act(y, s_out)
+    assert np.array_equal(outs[I8], q)
+    assert np.array_equal(outs[F16C], q.astype(np.float16))
