@@ -78,6 +78,7 @@ def _conv(aq, inp, act_dtype, out_dtype, path=AUTO, s_out=0.05):
     (300, 1024, 1152, 4, 8, DENSE, (128, 3, 0)),  # K split through the workspace + reduce
     (2, 960, 2880, 2, 8, AUTO, None),             # few tokens
     (8, 960, 2880, 2, 8, LUT, None),              # lookup-table path (reduce kernel)
+    (2, 2048, 1040, 2, 8, LUT, None),             # rotated tables (chunk reduction)
     (3, 8640, 960, 1, 16, AUTO, None),            # few tokens, 2^16 codebook (gather kernel)
 ])
 def test_code_outputs_agree(T, K, N, M, B, path, override):

@@ -64,7 +64,11 @@ def _linear_pair(inp, path, s_out=None):
     (300, 1024, 1152, 4, 8, DENSE),    # ragged M tile
     (200, 208, 208, 2, 8, FUSED),      # ragged K block and N tile
     (128, 8640, 960, 1, 16, AUTO),     # 2^16 book, fused with split K (reduce epilogue)
-    (5, 960, 2880, 2, 8, AUTO),        # lookup-table path (reduce epilogue)
+    (5, 960, 2880, 2, 8, AUTO),        # fused path, one ragged row tile
+    (1, 4096, 4112, 2, 8, LUT),        # rotated tables, 32 chunks (chunk reduction epilogue)
+    (3, 2048, 1040, 4, 8, LUT),        # four floats per entry, a chunk is part of a record
+    (4, 1024, 528, 1, 8, LUT),
+    (6, 960, 2880, 2, 8, LUT),         # the general table kernel (split reduction epilogue)
 ])
 def test_linear_q8_equals_chain(T, K, N, M, B, path):
     inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=B, cb_std=0.05 / M ** 0.5),
