@@ -106,10 +106,10 @@ AQ_API int aq_abi_version(void);
 /* Text of the last error on the calling host thread ("" if none). */
 AQ_API const char* aq_last_error_string(void);
 
-/* Reads and clears the device error word of the current device (kernels set it
- * when a bounded wait gives up).  Synchronises the device.  *code_out = 0 if no
- * kernel reported an error, else an OR of AQ_DEVERR_* bits.  Returns AQ_OK or
- * AQ_ERR_CUDA. */
+/* Reads and clears the device error words of the current device (kernels set them
+ * when a bounded wait gives up, or when a kernel finds its launch inconsistent and
+ * skips its work).  Synchronises the device.  *code_out = 0 if no kernel reported an
+ * error, else an OR of AQ_DEVERR_* bits.  Returns AQ_OK or AQ_ERR_CUDA. */
 AQ_API int aq_device_error(int* code_out);
 #define AQ_DEVERR_TIMEOUT_FULL   1   /* a consumer waited too long for a loaded stage      */
 #define AQ_DEVERR_TIMEOUT_EMPTY  2   /* the loader waited too long for a free stage        */
@@ -117,6 +117,9 @@ AQ_API int aq_device_error(int* code_out);
 #define AQ_DEVERR_TIMEOUT_ACCUM  8   /* the MMA or epilogue waited too long for an
                                         accumulator buffer                                  */
 #define AQ_DEVERR_TIMEOUT_DRAIN 16   /* after a time-out, in-flight copies did not drain   */
+#define AQ_DEVERR_SMEM_LAYOUT   32   /* the rotated-table kernel found its shared memory at
+                                        another window address than its launch assumed, and
+                                        skipped its work (the call's output is undefined)   */
 
 /* Failure-path testing: later tensor-core launches of this host thread give up a
  * pipeline wait after ns nanoseconds (checked every 256 polls) instead of about two

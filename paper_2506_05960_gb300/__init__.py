@@ -17,6 +17,7 @@ from ._binding import (  # noqa: F401
     aq_linear_plan, aq_linear_workspace_size, aq_pack, aq_set_plan_override,
     aq_set_wait_limit_ns, aq_linear_input_grad, aq_linear_input_grad_workspace_size, AQ_DEVERR_TIMEOUT_FULL,
     AQ_DEVERR_TIMEOUT_EMPTY, AQ_DEVERR_TIMEOUT_CONV, AQ_DEVERR_TIMEOUT_ACCUM, AQ_DEVERR_TIMEOUT_DRAIN,
+    AQ_DEVERR_SMEM_LAYOUT,
     aq_packed_size, aq_profile_enable, aq_profile_read, aq_quant_act, library_path,
     load_library, PROFILE_KINDS,
 )

@@ -247,7 +247,7 @@ def _plan(fn, name, *args) -> dict:
 
 
 AQ_DEVERR_TIMEOUT_FULL, AQ_DEVERR_TIMEOUT_EMPTY, AQ_DEVERR_TIMEOUT_CONV = 1, 2, 4
-AQ_DEVERR_TIMEOUT_ACCUM, AQ_DEVERR_TIMEOUT_DRAIN = 8, 16
+AQ_DEVERR_TIMEOUT_ACCUM, AQ_DEVERR_TIMEOUT_DRAIN, AQ_DEVERR_SMEM_LAYOUT = 8, 16, 32
 
 
 def aq_set_wait_limit_ns(ns=-1) -> None:

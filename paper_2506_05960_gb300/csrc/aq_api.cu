@@ -890,6 +890,10 @@ int aq_device_error(int* code_out) {
   unsigned v = 0;
   e = aq::read_clear_gemm_error(&v);
   if (e != cudaSuccess) return cuda_status(e, "reading device error word");
+  unsigned vl = 0;
+  e = aq::read_clear_lut_error(&vl);
+  if (e != cudaSuccess) return cuda_status(e, "reading device error word");
+  v |= vl;
   *code_out = static_cast<int>(v);
   return ok();
 }

@@ -195,5 +195,6 @@ cudaError_t launch_skinny(SkinnyParams p, cudaStream_t st);
 
 // Device error words of each translation unit (read and cleared, synchronising).
 cudaError_t read_clear_gemm_error(unsigned* out);
+cudaError_t read_clear_lut_error(unsigned* out);
 
 }  // namespace aq

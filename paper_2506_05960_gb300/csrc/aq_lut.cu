@@ -212,6 +212,8 @@ constexpr int kLutrThreads = 1024;
 constexpr int kLutrLaneRing = 96;                // bytes of code ring per lane
 constexpr uint32_t kLutrTableAddr = 0x20000u;    // shared-window address of the tables
 
+__device__ unsigned g_lut_err = 0;               // AQ_DEVERR_* bits of the table kernels
+
 template <int MM, int TP>
 struct LutrShape {
   static constexpr int NT = 32 / TP;             // tables (code bytes of a row) per chunk
@@ -250,7 +252,10 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   uint8_t* smem = reinterpret_cast<uint8_t*>(lut_smem4);
   const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
   // the host sized the allocation for this base; any other layout would misplace the tables
-  if (sbase + p.lutr_table_off != kLutrTableAddr || p.lutr_table_off < S::kFront) return;
+  if (sbase + p.lutr_table_off != kLutrTableAddr || p.lutr_table_off < S::kFront) {
+    if (threadIdx.x == 0) atomicOr(&g_lut_err, kDevErrSmemLayout);
+    return;
+  }
   uint4* sbook = reinterpret_cast<uint4*>(smem + S::kBookOff);                  // [MM][256]
   float* xs = reinterpret_cast<float*>(smem + S::kXsOff);                       // [TP][GC*8]
   float* L = reinterpret_cast<float*>(smem + p.lutr_table_off);                 // [256][64]
@@ -481,6 +486,16 @@ static uint32_t lutr_front(int TP, int M) {
 
 size_t lut_smem_bytes(int J, int M, int Tp, int T) {
   return static_cast<size_t>(J) * M * 256 * Tp * 4 + static_cast<size_t>(T) * J * 8 * 4;
+}
+
+cudaError_t read_clear_lut_error(unsigned* out) {
+  unsigned v = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_lut_err, sizeof(v));
+  if (e != cudaSuccess) return e;
+  const unsigned zero = 0;
+  e = cudaMemcpyToSymbol(g_lut_err, &zero, sizeof(zero));
+  *out = v;
+  return e;
 }
 
 cudaError_t launch_lut(const LutParams& p, cudaStream_t st) {

@@ -16,6 +16,7 @@ enum : unsigned {
   kDevErrTimeoutConv  = 4u,   // MMA waited too long for converted operands
   kDevErrTimeoutAccum = 8u,   // epilogue waited too long for the accumulator
   kDevErrTimeoutDrain = 16u,  // abort path could not drain in-flight copies
+  kDevErrSmemLayout   = 32u,  // a kernel's shared memory is not where its launch placed it
 };
 
 // About two seconds of spinning (checked against %globaltimer, in ns).
