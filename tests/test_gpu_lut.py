@@ -104,3 +104,16 @@ def test_lut_vector_tables(T, K, N, M):
                              inp["scale"], inp["bias"])
     assert_close(run_linear(inp, path=LUT), y_lut, "table order")
     assert aq.aq_linear_workspace_size(T, K, N, 8, M, 8, LUT) > 0
+
+
+@pytest.mark.parametrize("T,K,N,M", [(1, 16, 8, 2), (2, 64, 8, 1), (4, 16, 8, 4), (3, 32, 24, 2)])
+def test_lut_smallest_layers(T, K, N, M):
+    """The smallest layers the table path takes: one partial packed record, one partial row
+    block, a single CTA; against the oracle in both output types."""
+    inp = make_linear(LinearSpec(T=T, K=K, N=N, M=M, B=8, cb_std=0.05 / M ** 0.5),
+                      seed=900 + T + K + N + M)
+    assert_close(run_linear(inp, path=LUT), O.layer_f64(inp), (T, K, N, M))
+    W = O.decode_f64(inp["codes"], inp["codebooks"])
+    y32 = run_linear(inp, path=LUT, out_f32=True, with_bias=False)
+    assert_close(y32, O.linear_f64(inp["xq"], inp["s_x"], W, inp["scale"], None), (T, K, N, M))
+
