@@ -17,6 +17,15 @@
 #include "aq_internal.h"
 #include "aq_ptx.cuh"
 
+// The kernels' error bits are the ones aq_device_error() documents.
+static_assert(aq::kDevErrTimeoutFull == AQ_DEVERR_TIMEOUT_FULL &&
+              aq::kDevErrTimeoutEmpty == AQ_DEVERR_TIMEOUT_EMPTY &&
+              aq::kDevErrTimeoutConv == AQ_DEVERR_TIMEOUT_CONV &&
+              aq::kDevErrTimeoutAccum == AQ_DEVERR_TIMEOUT_ACCUM &&
+              aq::kDevErrTimeoutDrain == AQ_DEVERR_TIMEOUT_DRAIN &&
+              aq::kDevErrSmemLayout == AQ_DEVERR_SMEM_LAYOUT,
+              "device error bits differ from aq.h");
+
 // Scratch of aq_linear_noalloc: the decoded weights of one call.  Lives for the
 // life of the process on every device that loads this module.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[AQ_NOALLOC_SCRATCH_BYTES];

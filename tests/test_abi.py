@@ -306,3 +306,35 @@ def test_auto_path_rules(lib):
         wider = aq.aq_linear_a16_plan(T, K, N)
         want = wider["splits"] == 1 and wider["BN"] > p8["BN"]
         assert p16["a16"] == (1 if want else 0), (T, K, N, p16, p8, wider)
+
+
+def _header_constants():
+    """{name: int} of every AQ_* #define and enumerator with an integer value in include/*.h."""
+    out = {}
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            for m in re.finditer(r"^#define\s+(AQ_\w+)\s+(-?\d+)\b", text, flags=re.M):
+                out[m.group(1)] = int(m.group(2))
+            for m in re.finditer(r"^\s*(AQ_(?:DTYPE|PATH)_\w+)\s*=\s*(-?\d+)", text, flags=re.M):
+                out[m.group(1)] = int(m.group(2))
+    return out
+
+
+def test_binding_constants_match_header():
+    """Status codes, dtype and path values, device error bits and the profile-kind count
+    of the binding are the header's."""
+    import paper_2506_05960_gb300 as aq
+    from paper_2506_05960_gb300 import _binding
+    c = _header_constants()
+    dtypes = {k for k in c if k.startswith("AQ_DTYPE_")}
+    paths = {k for k in c if k.startswith("AQ_PATH_")}
+    deverrs = {k for k in c if k.startswith("AQ_DEVERR_")}
+    errs = {k for k in c if k.startswith("AQ_ERR_")}
+    assert len(dtypes) == 4 and len(paths) == 6 and len(deverrs) == 6 and len(errs) == 7
+    for k in dtypes | paths | deverrs:
+        assert getattr(aq, k) == c[k], k
+    assert {v: k for k, v in _binding._ERRORS.items()} == {k: c[k] for k in errs}
+    assert c["AQ_OK"] == 0 and len(aq.PROFILE_KINDS) == c["AQ_PROFILE_KINDS"]
+    bits = sorted(c[k] for k in deverrs)
+    assert bits == [1 << i for i in range(len(bits))]   # distinct single bits
