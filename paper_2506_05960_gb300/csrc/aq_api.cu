@@ -366,6 +366,22 @@ struct LutPlan {
 // lutr_kernel: each CTA takes at least this many 32-row blocks of (chunk, row block) units, so
 // that building a chunk's 64 KB of tables is paid for by enough lookups.
 constexpr int kLutrMinRowBlocksPerCta = 64;
+// The time of one chunk's table build, in 32-row blocks of lookups (measured: a build takes
+// about as long as streaming 60-90 row blocks of one CTA).
+constexpr int kLutrBuildRowBlocks = 64;
+
+// The busiest CTA of an even split of `units` (chunk-major, nrb per chunk) over `ctas`, in row
+// blocks of lookups plus one table build per chunk the CTA touches.
+int64_t lutr_cost(int64_t units, int64_t nrb, int ctas) {
+  int64_t worst = 0;
+  for (int b = 0; b < ctas; ++b) {
+    const int64_t u0 = units * b / ctas, u1 = units * (b + 1) / ctas;
+    if (u1 <= u0) continue;
+    const int64_t c = (u1 - 1) / nrb - u0 / nrb + 1;
+    worst = std::max(worst, u1 - u0 + c * kLutrBuildRowBlocks);
+  }
+  return worst;
+}
 
 LutPlan plan_lut(int T, int K, int N, int M) {
   LutPlan lp{};
@@ -380,9 +396,17 @@ LutPlan plan_lut(int T, int K, int N, int M) {
     const int nt = 32 / lp.Tp;
     lp.J = nt / M;
     lp.chunks = (KB * 8 * M + nt - 1) / nt;
-    const int64_t units = static_cast<int64_t>(lp.chunks) * ((N + 31) / 32);
+    const int64_t nrb = (N + 31) / 32;
+    const int64_t units = static_cast<int64_t>(lp.chunks) * nrb;
     lp.ctas = static_cast<int>(std::max<int64_t>(
         1, std::min<int64_t>(kPlanSMs, units / kLutrMinRowBlocksPerCta)));
+    // fewer CTAs, a whole multiple of the chunks, when no CTA then builds two chunks' tables and
+    // that costs less than the extra lookups per CTA
+    if (lp.chunks <= lp.ctas) {
+      const int aligned = lp.ctas / lp.chunks * lp.chunks;
+      if (aligned < lp.ctas && lutr_cost(units, nrb, aligned) < lutr_cost(units, nrb, lp.ctas))
+        lp.ctas = aligned;
+    }
     lp.rows_per_cta = 0;
     lp.ws_bytes = align_up(static_cast<size_t>(lp.chunks) * T * N * 4, 1024);
     return lp;

@@ -1010,23 +1010,39 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const GemmParams p, 
 // (independent loads in flight), then warp 0 adds the eight warps' sums in order and applies
 // the epilogue.  The order is fixed, so results are reproducible.
 __global__ void __launch_bounds__(256) lut_reduce_kernel(const GemmParams p, int splits) {
-  __shared__ float4 part[8][32];
+  // 16 output quads x 16 split groups per block: group j sums splits j, j + 16, ... with up to
+  // four loads in flight, then group 0 adds the 16 group sums in order
+  __shared__ float4 part[16][16];
   grid_dependency_wait();
   allow_dependents();
-  const int qi = threadIdx.x & 31;
-  const int j = threadIdx.x >> 5;
+  const int qi = threadIdx.x & 15;
+  const int j = threadIdx.x >> 4;
   const int64_t nq = static_cast<int64_t>(p.T) * (p.N / 4);
-  for (int64_t q0 = static_cast<int64_t>(blockIdx.x) * 32; q0 < nq;
-       q0 += static_cast<int64_t>(gridDim.x) * 32) {
+  for (int64_t q0 = static_cast<int64_t>(blockIdx.x) * 16; q0 < nq;
+       q0 += static_cast<int64_t>(gridDim.x) * 16) {
     const int64_t q = q0 + qi;
     const int64_t t = q / (p.N / 4);
     const int n = static_cast<int>(q - t * (p.N / 4)) * 4;
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     if (q < nq) {
-#pragma unroll 4
-      for (int s = j; s < splits; s += 8) {
-        const float4 v = *reinterpret_cast<const float4*>(
-            p.partial + (static_cast<int64_t>(s) * p.T + t) * p.N + n);
+      const float* base = p.partial + t * p.N + n;
+      const int64_t stride = static_cast<int64_t>(p.T) * p.N;
+      int s = j;
+      for (; s + 48 < splits; s += 64) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          v[u] = *reinterpret_cast<const float4*>(base + (s + 16 * u) * stride);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc.x += v[u].x;
+          acc.y += v[u].y;
+          acc.z += v[u].z;
+          acc.w += v[u].w;
+        }
+      }
+      for (; s < splits; s += 16) {
+        const float4 v = *reinterpret_cast<const float4*>(base + s * stride);
         acc.x += v.x;
         acc.y += v.y;
         acc.z += v.z;
@@ -1038,7 +1054,7 @@ __global__ void __launch_bounds__(256) lut_reduce_kernel(const GemmParams p, int
     if (j == 0 && q < nq) {
       float4 sum = part[0][qi];
 #pragma unroll
-      for (int w = 1; w < 8; ++w) {
+      for (int w = 1; w < 16; ++w) {
         const float4 v = part[w][qi];
         sum.x += v.x;
         sum.y += v.y;
@@ -1053,7 +1069,7 @@ __global__ void __launch_bounds__(256) lut_reduce_kernel(const GemmParams p, int
 
 cudaError_t launch_lut_reduce(const GemmParams& p, int splits, cudaStream_t st) {
   const int64_t nq = static_cast<int64_t>(p.T) * (p.N / 4);
-  int64_t blocks = (nq + 31) / 32;
+  int64_t blocks = (nq + 15) / 16;
   if (blocks > 152 * 8) blocks = 152 * 8;
   if (blocks < 1) blocks = 1;
   return launch_pdl(lut_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, p,

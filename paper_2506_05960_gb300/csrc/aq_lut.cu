@@ -201,9 +201,13 @@ __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
 //    offset).
 // Each lane sums its row's entries in its own rotated order (fixed per lane: deterministic).
 // Work: (chunk, 32-row block) units in chunk-major order, one contiguous equal range per CTA
-// (one CTA per SM): a CTA builds the tables of each chunk its range reaches (one or two) from
-// codebooks staged once in shared memory, and writes fp32 partial sums [chunk][T][N]; the
-// reduction sums the chunks and applies the epilogue.
+// (one CTA per SM; the host may take a whole multiple of the chunks instead, so that no CTA
+// builds two chunks' tables): a CTA builds the tables of each chunk its range reaches from
+// codebooks staged once in shared memory (widened to fp32 there when they fit), and writes fp32
+// partial sums [chunk][T][N]; the reduction sums the chunks and applies the epilogue.
+// Start-up: before the grid-dependency wait, one thread asks L2 to prefetch the codebooks and
+// the codes of every warp's first kStages row blocks; after it, one cp.async group brings the
+// codebooks and the activations of the first two chunks, ahead of the code stream's groups.
 // Code streaming: every lane copies its own row's NT code bytes with cp.async into a private
 // ring of kLutrLaneRing bytes (kStages row blocks ahead, across chunk boundaries) and reads them
 // back after waiting for its own copies: each lane touches only what it copied, so no barrier
@@ -227,8 +231,13 @@ struct LutrShape {
   static constexpr uint32_t kRingBytes = static_cast<uint32_t>(kLutrThreads) * kLutrLaneRing;
   static constexpr uint32_t kStageBytes = static_cast<uint32_t>(kLutrThreads) * NT;
   static constexpr uint32_t kBookOff = kRingBytes;
-  static constexpr uint32_t kXsOff = kBookOff + MM * 256 * 16;
-  static constexpr uint32_t kFront = kXsOff + (TP * GC * 8 * 4 + 15) / 16 * 16;
+  // the codebooks widened to fp32 once per CTA (when they fit before the tables)
+  static constexpr bool kBookF32 = MM <= 2;
+  static constexpr uint32_t kBookFOff = kBookOff + MM * 256 * 16;
+  static constexpr uint32_t kXsOff = kBookFOff + (kBookF32 ? MM * 256 * 32 : 0);
+  static constexpr int kXq = TP * GC * 8;        // activation bytes of one chunk
+  static constexpr uint32_t kXq8Off = kXsOff + (kXq * 4 + 15) / 16 * 16;
+  static constexpr uint32_t kFront = kXq8Off + 2 * ((kXq + 15) / 16 * 16);
   static constexpr uint32_t kTableBytes = 256 * 64 * 4;
 };
 
@@ -259,8 +268,6 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   uint4* sbook = reinterpret_cast<uint4*>(smem + S::kBookOff);                  // [MM][256]
   float* xs = reinterpret_cast<float*>(smem + S::kXsOff);                       // [TP][GC*8]
   float* L = reinterpret_cast<float*>(smem + p.lutr_table_off);                 // [256][64]
-  grid_dependency_wait();
-  allow_dependents();
   const int N = p.N, T = p.T;
   const int KB = (p.K + 63) / 64;
   const int64_t stream_bytes = static_cast<int64_t>(KB) * R;   // code bytes of a row
@@ -268,15 +275,36 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   const int64_t U = static_cast<int64_t>(p.chunks) * nrb;
   const int64_t u0 = U * blockIdx.x / gridDim.x;
   const int64_t u1 = U * (blockIdx.x + 1) / gridDim.x;
-  if (u0 >= u1) return;
-  for (int i = threadIdx.x; i < MM * 256; i += blockDim.x)
-    sbook[i] = reinterpret_cast<const uint4*>(p.books)[i];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nwarps = blockDim.x >> 5;
   const int c_first = static_cast<int>(u0 / nrb);
   const int rb_first = static_cast<int>(u0 % nrb);
   const int c_last = static_cast<int>((u1 - 1) / nrb);
   const int rb_last_end = static_cast<int>((u1 - 1) % nrb) + 1;
+  if (u0 < u1 && threadIdx.x == 0) {
+    // the weights do not come from the previous kernel: the codebooks and the first kStages
+    // row blocks of every warp (contiguous rows of the first chunk) start moving into L2 while
+    // it still runs (a prefetch only warms the cache; every read of the data comes after the
+    // wait below)
+    bulk_prefetch_l2(p.books, MM * 256 * 16);
+    const int64_t total16 = (static_cast<int64_t>(KB) * N * R) & ~static_cast<int64_t>(15);
+    const int rb_stop = c_first == c_last ? rb_last_end : nrb;
+    const int rb_end = rb_first + nwarps * D < rb_stop ? rb_first + nwarps * D : rb_stop;
+    const int64_t r0 = static_cast<int64_t>(rb_first) * 32;
+    const int64_t r1 = static_cast<int64_t>(rb_end) * 32 < N ? static_cast<int64_t>(rb_end) * 32 : N;
+    const int64_t b0 = static_cast<int64_t>(c_first) * NT;
+    const int64_t b1 = b0 + NT < stream_bytes ? b0 + NT : stream_bytes;
+    for (int64_t pl = b0 / R; pl * R < b1; ++pl) {
+      // these rows' whole records of the plane, widened to 16-byte bounds inside the buffer
+      const int64_t a0 = ((pl * N + r0) * R) & ~static_cast<int64_t>(15);
+      int64_t a1 = ((pl * N + r1) * R + 15) & ~static_cast<int64_t>(15);
+      if (a1 > total16) a1 = total16;
+      if (a1 > a0) bulk_prefetch_l2(p.packed + a0, static_cast<uint32_t>(a1 - a0));
+    }
+  }
+  grid_dependency_wait();
+  allow_dependents();
+  if (u0 >= u1) return;
   const int li = lane & (NT - 1);
   // entry address = kLutrTableAddr | code << 8 | lane_off (bytes 2, 0 of lane_reg; byte 1 from
   // the code)
@@ -325,19 +353,54 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
     wr += S::kStageBytes;
     if (wr == S::kRingBytes) wr = 0;
   };
+  // the codebooks and the first chunk's activations: one copy group ahead of the code stream
+  {
+    const uint32_t sb = sbase + S::kBookOff;
+    for (int i = threadIdx.x; i < MM * 256; i += blockDim.x)
+      cp_async_zfill(sb + i * 16, reinterpret_cast<const uint4*>(p.books) + i, true, 16);
+    constexpr int kPieces = S::kXq / 16;           // per chunk; the first two chunks
+    if (threadIdx.x < 2 * kPieces) {
+      const int h = threadIdx.x / kPieces;
+      const int i = threadIdx.x - h * kPieces;
+      const int tt = i / (GC * 8 / 16);
+      const int k = (c_first + h) * GC * 8 + (i % (GC * 8 / 16)) * 16;
+      const bool ok = tt < T && k < p.K;         // K % 16 == 0: a piece is all in or all out
+      cp_async_zfill(sbase + S::kXq8Off + threadIdx.x * 16,
+                     ok ? p.xq + static_cast<int64_t>(tt) * p.K + k : p.xq, ok, 16);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
 #pragma unroll 1
   for (int d = 0; d < D; ++d) produce();
   uint32_t rd = 0;                               // read offset of the oldest stage
+  asm volatile("cp.async.wait_group %0;" ::"n"(D) : "memory");
+  __syncthreads();
+  float4* sbookf = reinterpret_cast<float4*>(smem + S::kBookFOff);          // [MM][256][2]
+  if constexpr (S::kBookF32) {
+    for (int i = threadIdx.x; i < MM * 256; i += blockDim.x) {
+      const uint4 raw = sbook[i];
+      const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+      const float2 f0 = __half22float2(h2[0]), f1 = __half22float2(h2[1]);
+      const float2 f2 = __half22float2(h2[2]), f3 = __half22float2(h2[3]);
+      sbookf[2 * i] = make_float4(f0.x, f0.y, f1.x, f1.y);
+      sbookf[2 * i + 1] = make_float4(f2.x, f2.y, f3.x, f3.y);
+    }
+  }
 
   for (int c = c_first; c <= c_last; ++c) {
     const int g0 = c * GC;                       // first group of the chunk
     // ---- the chunk's tables (after every warp is done with the previous chunk's)
     __syncthreads();
-    for (int i = threadIdx.x; i < TP * GC * 8; i += blockDim.x) {
-      const int tt = i / (GC * 8);
-      const int k = g0 * 8 + (i - tt * GC * 8);
-      xs[i] = (tt < T && k < p.K) ? static_cast<float>(p.xq[static_cast<int64_t>(tt) * p.K + k])
-                                  : 0.0f;
+    if (c <= c_first + 1) {
+      const int8_t* xq8 = reinterpret_cast<const int8_t*>(smem + S::kXq8Off) + (c - c_first) * S::kXq;
+      for (int i = threadIdx.x; i < TP * GC * 8; i += blockDim.x) xs[i] = static_cast<float>(xq8[i]);
+    } else {
+      for (int i = threadIdx.x; i < TP * GC * 8; i += blockDim.x) {
+        const int tt = i / (GC * 8);
+        const int k = g0 * 8 + (i - tt * GC * 8);
+        xs[i] = (tt < T && k < p.K) ? static_cast<float>(p.xq[static_cast<int64_t>(tt) * p.K + k])
+                                    : 0.0f;
+      }
     }
     __syncthreads();
     {
@@ -350,21 +413,29 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
 #pragma unroll
         for (int e = 0; e < 8; ++e) xr[tt][e] = xs[tt * GC * 8 + j * 8 + e];
       const uint4* book = sbook + (t % MM) * 256;
-      for (int e = threadIdx.x / NT; e < 256; e += blockDim.x / NT) {
+#pragma unroll 2
+      for (int e = threadIdx.x / NT; e < 256; e += kLutrThreads / NT) {
         float o[TP];
 #pragma unroll
         for (int tt = 0; tt < TP; ++tt) o[tt] = 0.0f;
         if (live) {
           // L[e] = sum_u x[g0 + j][u] * C^(m)[e][u], ascending u (the other table kernels'
           // arithmetic)
-          const uint4 raw = book[e];
-          const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
           float cw[8];
+          if constexpr (S::kBookF32) {
+            const float4 a = sbookf[((t % MM) * 256 + e) * 2];
+            const float4 b = sbookf[((t % MM) * 256 + e) * 2 + 1];
+            cw[0] = a.x; cw[1] = a.y; cw[2] = a.z; cw[3] = a.w;
+            cw[4] = b.x; cw[5] = b.y; cw[6] = b.z; cw[7] = b.w;
+          } else {
+            const uint4 raw = book[e];
+            const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 f = __half22float2(h2[i]);
-            cw[2 * i] = f.x;
-            cw[2 * i + 1] = f.y;
+            for (int i = 0; i < 4; ++i) {
+              const float2 f = __half22float2(h2[i]);
+              cw[2 * i] = f.x;
+              cw[2 * i + 1] = f.y;
+            }
           }
 #pragma unroll
           for (int tt = 0; tt < TP; ++tt) {
