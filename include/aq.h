@@ -262,7 +262,10 @@ AQ_API int aq_set_plan_override(int BN, int splits, int cluster);
  * info[6] = 1 when the tensor cores read fp16 activations from shared memory
  * (aq_linear_f16 and aq_linear_a16 on the dense paths; 0: int8 activations
  * converted into tensor memory), info[7] = 64-wide K blocks per pipeline stage;
- * 0 for the other paths.  Writes min(n_info, 8) entries (zero past 8).  No
+ * for AQ_PATH_LUT info[2] = chunks of the code stream (fp32 partial sums per
+ * output) and info[5] = CTAs of the rotated-table kernel (0 when another table
+ * kernel runs; the launch takes at most the device's SM count); 0 for the other
+ * paths and fields.  Writes min(n_info, 8) entries (zero past 8).  No
  * device access.  aq_linear_f16_plan / aq_linear_a16_plan: the plans of those
  * entry points.                                                                */
 AQ_API int aq_linear_plan(int T, int K, int N, int g, int M, int B, int path, int* info,

@@ -1077,7 +1077,15 @@ int linear_plan_impl(int T, int K, int N, int g, int M, int B, int path, bool a1
   if (K % 16 != 0 || N % 8 != 0) return set_error(AQ_ERR_SHAPE, "need K %% 16 == 0 and N %% 8 == 0");
   const int rp = a16_only ? resolve_a16_path(path) : resolve_linear_path(path, T, B, N, K, M);
   if (rp < 0) return path_error(rp, path);
-  if (rp == AQ_PATH_FEW_TOKENS || rp == AQ_PATH_LUT) return fill_plan_info(rp, nullptr, info, n_info);
+  if (rp == AQ_PATH_LUT) {
+    // the table path: [2] chunks (partial sums per output), [5] CTAs of the table kernel
+    const LutPlan lp = plan_lut(std::max(T, 1), K, N, M);
+    const int r2 = fill_plan_info(rp, nullptr, info, n_info);
+    if (r2 == AQ_OK && n_info > 2) info[2] = lp.chunks;
+    if (r2 == AQ_OK && n_info > 5) info[5] = lp.vec == 2 ? lp.ctas : 0;
+    return r2;
+  }
+  if (rp == AQ_PATH_FEW_TOKENS) return fill_plan_info(rp, nullptr, info, n_info);
   const Route rt = route_layer(rp, T, N, K, (T + aq::kBM - 1) / aq::kBM, false, M, B,
                               a16_only ? kActF16Codes : (a16 ? kActF16 : kActInt8));
   return fill_plan_info(rp, &rt.pl, info, n_info);

@@ -338,3 +338,64 @@ def test_binding_constants_match_header():
     assert c["AQ_OK"] == 0 and len(aq.PROFILE_KINDS) == c["AQ_PROFILE_KINDS"]
     bits = sorted(c[k] for k in deverrs)
     assert bits == [1 << i for i in range(len(bits))]   # distinct single bits
+
+
+def _lutr_plan(T, K, N, M, sms=152, min_blocks=64, build_blocks=64):
+    """The rotated-table kernel's chunks and CTA count: NT = 32 / TP code bytes per chunk;
+    one CTA per SM with at least `min_blocks` (chunk, 32-row block) units each, or a whole
+    multiple of the chunks when no CTA then builds two chunks' tables and the busiest CTA's
+    row blocks plus `build_blocks` per table build come out lower."""
+    tp = 1 if T == 1 else (2 if T == 2 else 4)
+    nt = 32 // tp
+    chunks = (((K + 63) // 64) * 8 * M + nt - 1) // nt
+    nrb = (N + 31) // 32
+    units = chunks * nrb
+
+    def cost(ctas):
+        worst = 0
+        for b in range(ctas):
+            u0, u1 = units * b // ctas, units * (b + 1) // ctas
+            if u1 > u0:
+                worst = max(worst, u1 - u0 + ((u1 - 1) // nrb - u0 // nrb + 1) * build_blocks)
+        return worst
+
+    ctas = max(1, min(sms, units // min_blocks))
+    if chunks <= ctas:
+        aligned = ctas // chunks * chunks
+        if aligned < ctas and cost(aligned) < cost(ctas):
+            ctas = aligned
+    return chunks, ctas
+
+
+@pytest.mark.parametrize("T,K,N,M,chunks,ctas", [
+    (1, 8192, 16384, 2, 64, 128),    # 152 CTAs would cross chunk boundaries: 2 per chunk
+    (1, 8192, 65536, 2, 64, 152),    # long ranges: the second build is cheap against them
+    (1, 8192, 16384, 1, 32, 128),
+    (2, 8192, 16384, 2, 128, 152),   # more chunks than SMs
+    (1, 2048, 8192, 2, 16, 64),      # at least 64 row blocks per CTA
+    (4, 1024, 528, 1, 16, 4),        # 272 units: 4 CTAs of 68
+])
+def test_table_plan_chunks_and_ctas(lib, T, K, N, M, chunks, ctas):
+    """The table path's plan query reports the rotated-table kernel's chunks and CTA count,
+    and both follow the planning rule (restated here)."""
+    import paper_2506_05960_gb300 as aq
+    p = aq.aq_linear_plan(T, K, N, 8, M, 8, aq.AQ_PATH_LUT)
+    assert p["path"] == aq.AQ_PATH_LUT
+    assert (p["splits"], p["work_items"]) == (chunks, ctas) == _lutr_plan(T, K, N, M)
+    # no CTA of an aligned plan spans two chunks
+    if ctas % chunks == 0:
+        nrb = (N + 31) // 32
+        units = chunks * nrb
+        for b in range(ctas):
+            u0, u1 = units * b // ctas, units * (b + 1) // ctas
+            assert u1 <= u0 or (u1 - 1) // nrb == u0 // nrb
+
+
+def test_table_plan_matches_rule_on_many_shapes(lib):
+    import paper_2506_05960_gb300 as aq
+    for T in (1, 2, 3, 4):
+        for M in (1, 2, 4):
+            for K in (512, 960, 2048, 4096, 8192):
+                for N in (64, 1000, 2880, 16384):
+                    p = aq.aq_linear_plan(T, K, N, 8, M, 8, aq.AQ_PATH_LUT)
+                    assert (p["splits"], p["work_items"]) == _lutr_plan(T, K, N, M), (T, K, N, M)
