@@ -195,7 +195,8 @@ __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
 //    (l' + s) mod NT, l' = l mod NT, read from slot l' + s < 2 NT (the copy spares the wrap).
 //    The lanes of one shared-memory phase (32 / TP lanes, distinct l') read TP-word slots
 //    (l' + s) * TP mod 32 that are pairwise distinct: one conflict-free wavefront per phase;
-//  * the row's NT code bytes are rotated by l' bytes once (selects and funnel shifts), so step
+//  * the row's NT code bytes are rotated by l' bytes once (the half-chunk step by the order in
+//    which the ring's pieces are read, the rest by selects and funnel shifts), so step
 //    s takes byte s of the rotated words, and one byte permute assembles the entry's whole
 //    shared address: kLutrTableAddr | code << 8 | l' * TP * 4 (plus s * TP * 4 as the load's
 //    offset).
@@ -331,6 +332,13 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   };
   prod_settle();
   const uint32_t ring_lane = sbase + static_cast<uint32_t>(threadIdx.x * P);
+  // two or more pieces per row and chunk: a lane whose rotation includes half the chunk reads
+  // the second half's pieces first
+  constexpr bool kSwap = NP >= 2;
+  const bool swap = kSwap && ((li >> 2) & (NW / 2)) != 0;
+  const uint32_t half = static_cast<uint32_t>((NP / 2) * kLutrThreads * P);
+  const uint32_t ring_lo = ring_lane + (swap ? half : 0u);
+  const uint32_t ring_hi = ring_lane + (swap ? 0u : half);
   uint32_t wr = 0;                               // write offset of the next stage
   auto produce = [&]() {
     if (pc <= c_last) {
@@ -468,7 +476,11 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
       uint32_t r[NW];
 #pragma unroll
       for (int q = 0; q < NP; ++q) {
-        const uint32_t a = ring_lane + rd + static_cast<uint32_t>(q * kLutrThreads * P);
+        // pieces of the second half come from ring_hi: the top rotation step is the choice of
+        // which half is read first
+        const uint32_t a = (q < NP / 2 || !kSwap ? ring_lo : ring_hi) + rd +
+                           static_cast<uint32_t>((kSwap ? q % (NP / 2 > 0 ? NP / 2 : 1) : q) *
+                                                 kLutrThreads * P);
         if constexpr (P == 16) {
           asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
                        : "=r"(r[4 * q]), "=r"(r[4 * q + 1]), "=r"(r[4 * q + 2]), "=r"(r[4 * q + 3])
@@ -481,7 +493,7 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
       // rotate the row's code bytes left by li: byte s of r is stream byte (s + li) mod NT
       const int qw = li >> 2;
 #pragma unroll
-      for (int d = 1; d < NW; d <<= 1) {
+      for (int d = 1; d < (kSwap ? NW / 2 : NW); d <<= 1) {
         uint32_t tmp[NW];
 #pragma unroll
         for (int k = 0; k < NW; ++k) tmp[k] = (qw & d) ? r[(k + d) % NW] : r[k];
@@ -501,32 +513,24 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
       produce();
       rd += S::kStageBytes;
       if (rd == S::kRingBytes) rd = 0;
+      // two running sums (even and odd steps), each started by its first entry
       float acc0[TP], acc1[TP];
-#pragma unroll
-      for (int tt = 0; tt < TP; ++tt) acc0[tt] = acc1[tt] = 0.0f;
 #pragma unroll
       for (int s = 0; s < NT; ++s) {
         const uint32_t addr = __byte_perm(r[s >> 2], lane_reg, 0x7604u | ((s & 3) << 4)) +
                               static_cast<uint32_t>(s * TP * 4);
         float* acc = (s & 1) ? acc1 : acc0;
+        float v[TP];
         if constexpr (TP == 1) {
-          float v;
-          asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
-          acc[0] += v;
+          asm("ld.shared.f32 %0, [%1];" : "=f"(v[0]) : "r"(addr));
         } else if constexpr (TP == 2) {
-          float v0, v1;
-          asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v0), "=f"(v1) : "r"(addr));
-          acc[0] += v0;
-          acc[1] += v1;
+          asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v[0]), "=f"(v[1]) : "r"(addr));
         } else {
-          float v0, v1, v2, v3;
           asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
-              : "=f"(v0), "=f"(v1), "=f"(v2), "=f"(v3) : "r"(addr));
-          acc[0] += v0;
-          acc[1] += v1;
-          acc[2] += v2;
-          acc[3] += v3;
+              : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]) : "r"(addr));
         }
+#pragma unroll
+        for (int tt = 0; tt < TP; ++tt) acc[tt] = s < 2 ? v[tt] : acc[tt] + v[tt];
       }
       if (rb * 32 + lane < N) {
 #pragma unroll
