@@ -370,17 +370,43 @@ constexpr int kLutrMinRowBlocksPerCta = 64;
 // about as long as streaming 60-90 row blocks of one CTA).
 constexpr int kLutrBuildRowBlocks = 64;
 
-// The busiest CTA of an even split of `units` (chunk-major, nrb per chunk) over `ctas`, in row
-// blocks of lookups plus one table build per chunk the CTA touches.
-int64_t lutr_cost(int64_t units, int64_t nrb, int ctas) {
-  int64_t worst = 0;
+// Contiguous ranges of the chunk-major (chunk, 32-row block) units for `ctas` CTAs such that
+// no CTA's cost -- its row blocks plus kLutrBuildRowBlocks per chunk whose tables it builds --
+// exceeds `tau`: each CTA in turn takes as many units as that allows.  Fills bounds[0..ctas]
+// (later CTAs may get empty ranges) and returns whether every unit was placed.
+bool lutr_fill(int64_t units, int64_t nrb, int ctas, int64_t tau, int64_t* bounds) {
+  int64_t u = 0;
+  bounds[0] = 0;
   for (int b = 0; b < ctas; ++b) {
-    const int64_t u0 = units * b / ctas, u1 = units * (b + 1) / ctas;
-    if (u1 <= u0) continue;
-    const int64_t c = (u1 - 1) / nrb - u0 / nrb + 1;
-    worst = std::max(worst, u1 - u0 + c * kLutrBuildRowBlocks);
+    int64_t r = u < units ? tau - kLutrBuildRowBlocks : 0;   // the first chunk's build
+    while (r > 0 && u < units) {
+      const int64_t e = std::min(units, (u / nrb + 1) * nrb);  // end of the current chunk
+      if (u + r <= e) {
+        u += r;
+        r = 0;
+      } else {
+        r -= e - u;
+        u = e;
+        r -= kLutrBuildRowBlocks;                            // entering the next chunk
+      }
+    }
+    bounds[b + 1] = u;
   }
-  return worst;
+  return u >= units;
+}
+
+// The smallest such cost for `ctas` CTAs (bisection over tau), with its ranges in bounds.
+int64_t lutr_partition(int64_t units, int64_t nrb, int ctas, int64_t* bounds) {
+  int64_t lo = kLutrBuildRowBlocks, hi = units + kLutrBuildRowBlocks * (units / nrb + 2);
+  while (lo + 1 < hi) {
+    const int64_t mid = lo + (hi - lo) / 2;
+    if (lutr_fill(units, nrb, ctas, mid, bounds))
+      hi = mid;
+    else
+      lo = mid;
+  }
+  lutr_fill(units, nrb, ctas, hi, bounds);
+  return hi;
 }
 
 LutPlan plan_lut(int T, int K, int N, int M) {
@@ -401,10 +427,12 @@ LutPlan plan_lut(int T, int K, int N, int M) {
     lp.ctas = static_cast<int>(std::max<int64_t>(
         1, std::min<int64_t>(kPlanSMs, units / kLutrMinRowBlocksPerCta)));
     // fewer CTAs, a whole multiple of the chunks, when no CTA then builds two chunks' tables and
-    // that costs less than the extra lookups per CTA
+    // the busiest CTA's cost comes out lower
     if (lp.chunks <= lp.ctas) {
       const int aligned = lp.ctas / lp.chunks * lp.chunks;
-      if (aligned < lp.ctas && lutr_cost(units, nrb, aligned) < lutr_cost(units, nrb, lp.ctas))
+      int64_t b[kPlanSMs + 1];
+      if (aligned < lp.ctas &&
+          lutr_partition(units, nrb, aligned, b) < lutr_partition(units, nrb, lp.ctas, b))
         lp.ctas = aligned;
     }
     lp.rows_per_cta = 0;
@@ -1286,7 +1314,10 @@ int linear_impl(const int8_t* xq, float s_x, const void* codes_packed, const voi
     lpar.G = K / 8;
     lpar.chunks = lp.chunks;
     lpar.rows_per_cta = lp.rows_per_cta;
-    lpar.ctas = std::min(lp.ctas, sm_count());
+    lpar.ctas = std::min(std::min(lp.ctas, sm_count()), aq::kLutrMaxCtas);
+    if (lp.vec == 2)
+      lutr_partition(static_cast<int64_t>(lp.chunks) * ((N + 31) / 32), (N + 31) / 32, lpar.ctas,
+                     lpar.unit_bounds);
     cudaError_t e;
     {
       ProfScope ps(kProfLutGather, st);

@@ -75,6 +75,8 @@ struct GemmParams {
 };
 
 // Parameters of the lookup-table kernel (linear layer, 8-bit codes, T <= 16).
+constexpr int kLutrMaxCtas = 160;  // grid limit of the rotated-table kernel (one CTA per SM)
+
 struct LutParams {
   const int8_t* xq;             // [T][K]
   const uint8_t* packed;        // packed codes [K/64][N][8][M]
@@ -89,10 +91,12 @@ struct LutParams {
   int J;                        // groups per chunk (vec: whole K blocks; else divides 8)
   int G;                        // K / 8
   int chunks, rows_per_cta;
-  int ctas;                     // lutr_kernel: grid size (CTAs share the (chunk, row block)
-                                // units in equal contiguous ranges)
+  int ctas;                     // lutr_kernel: grid size (at most kLutrMaxCtas)
   unsigned lutr_table_off;      // lutr_kernel: dynamic shared-memory offset of the tables (set
                                 // by launch_lut so that they start at a 64 KB boundary)
+  // lutr_kernel: CTA b takes the (chunk, 32-row block) units [unit_bounds[b], unit_bounds[b+1])
+  // of the chunk-major order (contiguous ranges, balanced by the host for lookups plus builds)
+  int64_t unit_bounds[kLutrMaxCtas + 1];
 };
 
 // Parameters of the few-token kernel (linear layer, T <= 16, one pass, no workspace).

@@ -201,9 +201,9 @@ __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
 //    shared address: kLutrTableAddr | code << 8 | l' * TP * 4 (plus s * TP * 4 as the load's
 //    offset).
 // Each lane sums its row's entries in its own rotated order (fixed per lane: deterministic).
-// Work: (chunk, 32-row block) units in chunk-major order, one contiguous equal range per CTA
-// (one CTA per SM; the host may take a whole multiple of the chunks instead, so that no CTA
-// builds two chunks' tables): a CTA builds the tables of each chunk its range reaches from
+// Work: (chunk, 32-row block) units in chunk-major order, one contiguous range per CTA (one CTA
+// per SM), the ranges set by the host so that the busiest CTA's lookups plus table builds are as
+// few as it can make them: a CTA builds the tables of each chunk its range reaches from
 // codebooks staged once in shared memory (widened to fp32 there when they fit), and writes fp32
 // partial sums [chunk][T][N]; the reduction sums the chunks and applies the epilogue.
 // Start-up: before the grid-dependency wait, one thread asks L2 to prefetch the codebooks and
@@ -273,9 +273,8 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   const int KB = (p.K + 63) / 64;
   const int64_t stream_bytes = static_cast<int64_t>(KB) * R;   // code bytes of a row
   const int nrb = (N + 31) / 32;
-  const int64_t U = static_cast<int64_t>(p.chunks) * nrb;
-  const int64_t u0 = U * blockIdx.x / gridDim.x;
-  const int64_t u1 = U * (blockIdx.x + 1) / gridDim.x;
+  const int64_t u0 = p.unit_bounds[blockIdx.x];
+  const int64_t u1 = p.unit_bounds[blockIdx.x + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nwarps = blockDim.x >> 5;
   const int c_first = static_cast<int>(u0 / nrb);

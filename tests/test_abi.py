@@ -340,40 +340,74 @@ def test_binding_constants_match_header():
     assert bits == [1 << i for i in range(len(bits))]   # distinct single bits
 
 
-def _lutr_plan(T, K, N, M, sms=152, min_blocks=64, build_blocks=64):
+def _lutr_fill(units, nrb, ctas, tau, build):
+    """Greedy ranges: each CTA in turn takes as many chunk-major units as keep its row blocks
+    plus `build` per chunk whose tables it builds within tau.  (placed all?, bounds)"""
+    u, bounds = 0, [0]
+    for _ in range(ctas):
+        r = tau - build if u < units else 0
+        while r > 0 and u < units:
+            e = min(units, (u // nrb + 1) * nrb)
+            if u + r <= e:
+                u, r = u + r, 0
+            else:
+                r -= e - u + build
+                u = e
+        bounds.append(u)
+    return u >= units, bounds
+
+
+def _lutr_partition(units, nrb, ctas, build=64):
+    lo, hi = build, units + build * (units // nrb + 2)
+    while lo + 1 < hi:
+        mid = (lo + hi) // 2
+        if _lutr_fill(units, nrb, ctas, mid, build)[0]:
+            hi = mid
+        else:
+            lo = mid
+    return hi, _lutr_fill(units, nrb, ctas, hi, build)[1]
+
+
+def _lutr_plan(T, K, N, M, sms=152, min_blocks=64):
     """The rotated-table kernel's chunks and CTA count: NT = 32 / TP code bytes per chunk;
     one CTA per SM with at least `min_blocks` (chunk, 32-row block) units each, or a whole
-    multiple of the chunks when no CTA then builds two chunks' tables and the busiest CTA's
-    row blocks plus `build_blocks` per table build come out lower."""
+    multiple of the chunks when the balanced ranges' busiest CTA comes out cheaper."""
     tp = 1 if T == 1 else (2 if T == 2 else 4)
     nt = 32 // tp
     chunks = (((K + 63) // 64) * 8 * M + nt - 1) // nt
     nrb = (N + 31) // 32
     units = chunks * nrb
-
-    def cost(ctas):
-        worst = 0
-        for b in range(ctas):
-            u0, u1 = units * b // ctas, units * (b + 1) // ctas
-            if u1 > u0:
-                worst = max(worst, u1 - u0 + ((u1 - 1) // nrb - u0 // nrb + 1) * build_blocks)
-        return worst
-
     ctas = max(1, min(sms, units // min_blocks))
     if chunks <= ctas:
         aligned = ctas // chunks * chunks
-        if aligned < ctas and cost(aligned) < cost(ctas):
+        if aligned < ctas and _lutr_partition(units, nrb, aligned)[0] < _lutr_partition(units, nrb, ctas)[0]:
             ctas = aligned
     return chunks, ctas
 
 
+def test_table_ranges_cover_every_unit_once():
+    """The balanced ranges are contiguous, ordered and cover all units; no CTA exceeds the
+    bisected cost, and one unit less of budget cannot place them all."""
+    for chunks, nrb, ctas in [(64, 512, 152), (64, 2048, 152), (32, 512, 128), (16, 17, 4),
+                              (3, 1, 2), (1, 5000, 152)]:
+        units = chunks * nrb
+        tau, b = _lutr_partition(units, nrb, ctas)
+        assert b[0] == 0 and b[-1] == units and len(b) == ctas + 1
+        assert all(b[i] <= b[i + 1] for i in range(ctas))
+        for i in range(ctas):
+            if b[i + 1] > b[i]:
+                touched = (b[i + 1] - 1) // nrb - b[i] // nrb + 1
+                assert b[i + 1] - b[i] + 64 * touched <= tau
+        assert not _lutr_fill(units, nrb, ctas, tau - 1, 64)[0]
+
+
 @pytest.mark.parametrize("T,K,N,M,chunks,ctas", [
-    (1, 8192, 16384, 2, 64, 128),    # 152 CTAs would cross chunk boundaries: 2 per chunk
-    (1, 8192, 65536, 2, 64, 152),    # long ranges: the second build is cheap against them
-    (1, 8192, 16384, 1, 32, 128),
+    (1, 8192, 16384, 2, 64, 152),
+    (1, 8192, 65536, 2, 64, 152),
+    (1, 4096, 8192, 2, 32, 128),     # aligned: every CTA inside one chunk is cheaper
     (2, 8192, 16384, 2, 128, 152),   # more chunks than SMs
     (1, 2048, 8192, 2, 16, 64),      # at least 64 row blocks per CTA
-    (4, 1024, 528, 1, 16, 4),        # 272 units: 4 CTAs of 68
+    (4, 1024, 528, 1, 16, 4),        # 272 units: 4 CTAs
 ])
 def test_table_plan_chunks_and_ctas(lib, T, K, N, M, chunks, ctas):
     """The table path's plan query reports the rotated-table kernel's chunks and CTA count,
@@ -382,13 +416,6 @@ def test_table_plan_chunks_and_ctas(lib, T, K, N, M, chunks, ctas):
     p = aq.aq_linear_plan(T, K, N, 8, M, 8, aq.AQ_PATH_LUT)
     assert p["path"] == aq.AQ_PATH_LUT
     assert (p["splits"], p["work_items"]) == (chunks, ctas) == _lutr_plan(T, K, N, M)
-    # no CTA of an aligned plan spans two chunks
-    if ctas % chunks == 0:
-        nrb = (N + 31) // 32
-        units = chunks * nrb
-        for b in range(ctas):
-            u0, u1 = units * b // ctas, units * (b + 1) // ctas
-            assert u1 <= u0 or (u1 - 1) // nrb == u0 // nrb
 
 
 def test_table_plan_matches_rule_on_many_shapes(lib):
