@@ -414,8 +414,8 @@ LutPlan plan_lut(int T, int K, int N, int M) {
   const bool mm = M == 1 || M == 2 || M == 4;
   if (T <= 4 && mm) {
     // lutr_kernel: TP = 1, 2 or 4 floats per entry; a chunk is 32 / TP code bytes of every row
-    // (32 / (TP * M) groups); one CTA of 1024 threads per SM at most, each with an equal
-    // contiguous range of (chunk, 32-row block) units
+    // (32 / (TP * M) groups); one CTA of 1024 threads per SM at most, each with a contiguous
+    // range of (chunk, 32-row block) units (lutr_partition, at launch)
     lp.vec = 2;
     lp.Tp = T == 1 ? 1 : (T == 2 ? 2 : 4);
     const int KB = (K + 63) / 64;
