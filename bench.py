@@ -1195,12 +1195,13 @@ def main():
                                   "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
                     del gs, Ls
         # few tokens on a layer large enough to amortise the launches: how fast each path
-        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes); AUTO takes the
-        # table path up to four tokens here
-        for Ts, pth in ((1, aq.AQ_PATH_FEW_TOKENS), (1, aq.AQ_PATH_AUTO),
-                        (2, aq.AQ_PATH_FEW_TOKENS), (2, aq.AQ_PATH_AUTO),
-                        (4, aq.AQ_PATH_FEW_TOKENS), (4, aq.AQ_PATH_FUSED), (4, aq.AQ_PATH_AUTO)):
-            inp_s = _mlin(LinearSpec(T=Ts, K=8192, N=16384, M=2, B=8), seed=90 + Ts)
+        # streams the codes (K=8192, N=16384, 2x8: 33.6 MB of codes; N=65536: 134 MB, more
+        # than L2); AUTO takes the table path up to four tokens here
+        for Ts, Ns, pth in ((1, 16384, aq.AQ_PATH_FEW_TOKENS), (1, 16384, aq.AQ_PATH_AUTO),
+                            (2, 16384, aq.AQ_PATH_FEW_TOKENS), (2, 16384, aq.AQ_PATH_AUTO),
+                            (4, 16384, aq.AQ_PATH_FEW_TOKENS), (4, 16384, aq.AQ_PATH_FUSED),
+                            (4, 16384, aq.AQ_PATH_AUTO), (1, 65536, aq.AQ_PATH_AUTO)):
+            inp_s = _mlin(LinearSpec(T=Ts, K=8192, N=Ns, M=2, B=8), seed=90 + Ts)
             Ls = [Dev(aq, torch, inp_s, dev, path=pth) for _ in range(4)]
             with torch.cuda.stream(stream):
                 for L in Ls:
@@ -1208,10 +1209,10 @@ def main():
             stream.synchronize()
             gs = capture(torch, stream, lambda: [L.layer(stream) for L in Ls])
             ms = replay_ms(torch, stream, gs, 10) / len(Ls)
-            wbytes = alg_bytes(Ts, 8192, 16384, 2, 8)
+            wbytes = alg_bytes(Ts, 8192, Ns, 2, 8)
             pname = {aq.AQ_PATH_FEW_TOKENS: "FEW", aq.AQ_PATH_AUTO: "AUTO (table)",
                      aq.AQ_PATH_FUSED: "FUSED"}[pth]
-            sweep[f"K=8192 N=16384 2x8 T={Ts} {pname} (layer only, 4 rotating buffer sets)"] = {
+            sweep[f"K=8192 N={Ns} 2x8 T={Ts} {pname} (layer only, 4 rotating buffer sets)"] = {
                 "us_per_step": ms * 1e3, "hbm_gbs_algorithmic": wbytes / (ms * 1e-3) / 1e9,
                 "hbm_roofline_frac": wbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"]}
             del gs, Ls
