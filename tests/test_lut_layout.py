@@ -8,6 +8,7 @@ import pytest
 TABLE_ADDR = 0x20000          # shared-window address of the tables (a multiple of 64 KB)
 BANKS = 32
 
+
 def prmt(a, b, sel):
     """PTX prmt.b32 default mode: result byte i = byte (nibble i of sel) & 7 of {a, b}."""
     src = a | (b << 32)
@@ -16,6 +17,7 @@ def prmt(a, b, sel):
         k = (sel >> (4 * i)) & 7
         out |= ((src >> (8 * k)) & 0xFF) << (8 * i)
     return out
+
 
 @pytest.mark.parametrize("TP", [1, 2, 4])
 def test_phase_lanes_hit_distinct_banks_for_any_codes(TP):
@@ -31,6 +33,7 @@ def test_phase_lanes_hit_distinct_banks_for_any_codes(TP):
                 banks += [(word + w) % BANKS for w in range(TP)]
             assert sorted(banks) == list(range(BANKS))
             assert all(lp + s < 2 * NT for lp in range(NT))     # inside the duplicated slots
+
 
 @pytest.mark.parametrize("TP", [1, 2, 4])
 def test_byte_permute_assembles_the_entry_address(TP):
@@ -48,6 +51,7 @@ def test_byte_permute_assembles_the_entry_address(TP):
                     addr = prmt(word, lane_reg, 0x7604 | (c << 4)) + s * TP * 4
                     assert addr == TABLE_ADDR + code * 256 + (lp + s) * TP * 4
                     assert lp * TP * 4 + s * TP * 4 < 256
+
 
 def _kernel_rotation(stream_bytes, li, NT, P):
     """The kernel's rotation of a row's NT code bytes by li: the ring holds NP = NT/P pieces;
@@ -73,6 +77,7 @@ def _kernel_rotation(stream_bytes, li, NT, P):
     if sh:
         r = [((r[k] >> sh) | (r[(k + 1) % NW] << (32 - sh))) & 0xFFFFFFFF for k in range(NW)]
     return b"".join(w.to_bytes(4, "little") for w in r)
+
 
 @pytest.mark.parametrize("TP,M", [(1, 1), (1, 2), (1, 4), (2, 1), (2, 2), (2, 4), (4, 1),
                                   (4, 2), (4, 4)])
