@@ -282,16 +282,17 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   const int c_last = static_cast<int>((u1 - 1) / nrb);
   const int rb_last_end = static_cast<int>((u1 - 1) % nrb) + 1;
   if (u0 < u1 && threadIdx.x == 0) {
-    // the weights do not come from the previous kernel: the codebooks and the first kStages
-    // row blocks of every warp (contiguous rows of the first chunk) start moving into L2 while
-    // it still runs (a prefetch only warms the cache; every read of the data comes after the
-    // wait below)
+    // the codebooks and the first kStages row blocks of every warp (contiguous rows of the
+    // first chunk) start moving into L2 while the previous kernel still runs: a prefetch only
+    // warms the cache and every read of the data comes after the wait below, so this holds
+    // even if that kernel wrote them
     bulk_prefetch_l2(p.books, MM * 256 * 16);
     const int64_t total16 = (static_cast<int64_t>(KB) * N * R) & ~static_cast<int64_t>(15);
     const int rb_stop = c_first == c_last ? rb_last_end : nrb;
     const int rb_end = rb_first + nwarps * D < rb_stop ? rb_first + nwarps * D : rb_stop;
     const int64_t r0 = static_cast<int64_t>(rb_first) * 32;
-    const int64_t r1 = static_cast<int64_t>(rb_end) * 32 < N ? static_cast<int64_t>(rb_end) * 32 : N;
+    const int64_t r_end = static_cast<int64_t>(rb_end) * 32;
+    const int64_t r1 = r_end < N ? r_end : N;
     const int64_t b0 = static_cast<int64_t>(c_first) * NT;
     const int64_t b1 = b0 + NT < stream_bytes ? b0 + NT : stream_bytes;
     for (int64_t pl = b0 / R; pl * R < b1; ++pl) {
