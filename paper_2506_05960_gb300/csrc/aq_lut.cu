@@ -195,8 +195,8 @@ __global__ void __launch_bounds__(256) lutv_kernel(const LutParams p) {
 //    (l' + s) mod NT, l' = l mod NT, read from slot l' + s < 2 NT (the copy spares the wrap).
 //    The lanes of one shared-memory phase (32 / TP lanes, distinct l') read TP-word slots
 //    (l' + s) * TP mod 32 that are pairwise distinct: one conflict-free wavefront per phase;
-//  * the row's NT code bytes are rotated by l' bytes once (the half-chunk step by the order in
-//    which the ring's pieces are read, the rest by selects and funnel shifts), so step
+//  * the row's NT code bytes are rotated by l' bytes once (whole 8-byte steps by the order in
+//    which the ring's 8-byte slots are read, then one word select and a funnel shift), so step
 //    s takes byte s of the rotated words, and one byte permute assembles the entry's whole
 //    shared address: kLutrTableAddr | code << 8 | l' * TP * 4 (plus s * TP * 4 as the load's
 //    offset).
@@ -334,11 +334,16 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   const uint32_t ring_lane = sbase + static_cast<uint32_t>(threadIdx.x * P);
   // two or more pieces per row and chunk: a lane whose rotation includes half the chunk reads
   // the second half's pieces first
-  constexpr bool kSwap = NP >= 2;
-  const bool swap = kSwap && ((li >> 2) & (NW / 2)) != 0;
-  const uint32_t half = static_cast<uint32_t>((NP / 2) * kLutrThreads * P);
-  const uint32_t ring_lo = ring_lane + (swap ? half : 0u);
-  const uint32_t ring_hi = ring_lane + (swap ? 0u : half);
+  // the row's chunk as NS 8-byte slots: slot i of the registers is read from ring slot
+  // (i + li / 8) mod NS, which is the rotation by whole 8-byte slots
+  constexpr int NS = NT / 8;
+  uint32_t slot_addr[NS];
+#pragma unroll
+  for (int i = 0; i < NS; ++i) {
+    const int j = (i + (li >> 3)) & (NS - 1);
+    slot_addr[i] =
+        ring_lane + static_cast<uint32_t>((j * 8 / P) * kLutrThreads * P + (j * 8) % P);
+  }
   uint32_t wr = 0;                               // write offset of the next stage
   auto produce = [&]() {
     if (pc <= c_last) {
@@ -475,28 +480,15 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
       asm volatile("cp.async.wait_group %0;" ::"n"(D - 1) : "memory");
       uint32_t r[NW];
 #pragma unroll
-      for (int q = 0; q < NP; ++q) {
-        // pieces of the second half come from ring_hi: the top rotation step is the choice of
-        // which half is read first
-        const uint32_t a = (q < NP / 2 || !kSwap ? ring_lo : ring_hi) + rd +
-                           static_cast<uint32_t>((kSwap ? q % (NP / 2 > 0 ? NP / 2 : 1) : q) *
-                                                 kLutrThreads * P);
-        if constexpr (P == 16) {
-          asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                       : "=r"(r[4 * q]), "=r"(r[4 * q + 1]), "=r"(r[4 * q + 2]), "=r"(r[4 * q + 3])
-                       : "r"(a) : "memory");
-        } else {
-          asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];"
-                       : "=r"(r[2 * q]), "=r"(r[2 * q + 1]) : "r"(a) : "memory");
-        }
-      }
-      // rotate the row's code bytes left by li: byte s of r is stream byte (s + li) mod NT
-      const int qw = li >> 2;
-#pragma unroll
-      for (int d = 1; d < (kSwap ? NW / 2 : NW); d <<= 1) {
+      for (int i = 0; i < NS; ++i)
+        asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];"
+                     : "=r"(r[2 * i]), "=r"(r[2 * i + 1]) : "r"(slot_addr[i] + rd) : "memory");
+      // rotate the row's code bytes left by li: byte s of r is stream byte (s + li) mod NT (the
+      // slots above rotated by whole 8 bytes; one word step and a funnel shift remain)
+      if ((li >> 2) & 1) {
         uint32_t tmp[NW];
 #pragma unroll
-        for (int k = 0; k < NW; ++k) tmp[k] = (qw & d) ? r[(k + d) % NW] : r[k];
+        for (int k = 0; k < NW; ++k) tmp[k] = r[(k + 1) % NW];
 #pragma unroll
         for (int k = 0; k < NW; ++k) r[k] = tmp[k];
       }

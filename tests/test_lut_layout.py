@@ -1,7 +1,7 @@
 """Layout rules of the rotated-table kernel (App. A.1 table order; aq_lut.cu), checked on the
 CPU: conflict-free shared-memory banks for every code pattern, the byte-permute address
-assembly, and the code-byte rotation (half-chunk step by the ring read order, the rest by
-selects and funnel shifts).  Pure integer arithmetic; no device."""
+assembly, and the code-byte rotation (whole 8-byte steps by the order of the ring's slot
+reads, then one word select and a funnel shift).  Pure integer arithmetic; no device."""
 
 import pytest
 
@@ -54,29 +54,41 @@ def test_byte_permute_assembles_the_entry_address(TP):
 
 
 def _kernel_rotation(stream_bytes, li, NT, P):
-    """The kernel's rotation of a row's NT code bytes by li: the ring holds NP = NT/P pieces;
-    a lane whose word rotation qw = li >> 2 has the half-chunk bit reads the second half's
-    pieces first; the remaining select stages rotate by the lower bits of qw, then a funnel
-    shift by 8 * (li & 3) bits."""
-    NW, NP = NT // 4, NT // P
-    words = [int.from_bytes(bytes(stream_bytes[4 * k:4 * k + 4]), "little") for k in range(NW)]
-    swap = NP >= 2 and ((li >> 2) & (NW // 2)) != 0
-    wpp = P // 4                                           # words per piece
-    order = list(range(NP))
-    if swap:
-        order = order[NP // 2:] + order[:NP // 2]
-    r = [words[q * wpp + w] for q in order for w in range(wpp)]
-    qw = li >> 2
-    top = NW // 2 if NP >= 2 else NW
-    d = 1
-    while d < top:
-        if qw & d:
-            r = [r[(k + d) % NW] for k in range(NW)]
-        d <<= 1
+    """The kernel's rotation of a row's NT code bytes by li: the ring holds the row's bytes in
+    pieces of P bytes; register slot i (8 bytes) is read from ring slot (i + li // 8) mod NS,
+    NS = NT / 8 (whole 8-byte steps), then the words are rotated by one when bit 2 of li is
+    set, then a funnel shift by 8 * (li & 3) bits."""
+    NW, NS = NT // 4, NT // 8
+    ring = list(stream_bytes)                              # piece q holds bytes q*P .. q*P+P-1
+    regs = []
+    for i in range(NS):
+        j = (i + (li >> 3)) & (NS - 1)
+        piece, off = (j * 8) // P, (j * 8) % P
+        regs += ring[piece * P + off:piece * P + off + 8]
+    r = [int.from_bytes(bytes(regs[4 * k:4 * k + 4]), "little") for k in range(NW)]
+    if (li >> 2) & 1:
+        r = [r[(k + 1) % NW] for k in range(NW)]
     sh = 8 * (li & 3)
     if sh:
         r = [((r[k] >> sh) | (r[(k + 1) % NW] << (32 - sh))) & 0xFFFFFFFF for k in range(NW)]
     return b"".join(w.to_bytes(4, "little") for w in r)
+
+
+def test_slot_reads_are_conflict_free():
+    """Each 8-byte slot read of a warp (ring layout [piece][thread][P bytes]) touches every bank
+    pair at most twice: two wavefronts, the least 32 lanes x 8 bytes can take."""
+    for NT, P in ((32, 16), (32, 8), (16, 16), (16, 8), (8, 8)):
+        NS = NT // 8
+        for i in range(NS):
+            banks = {}
+            for lane in range(32):
+                li = lane % NT
+                j = (i + (li >> 3)) & (NS - 1)
+                addr = (j * 8 // P) * 1024 * P + lane * P + (j * 8) % P
+                for w in range(2):
+                    b = (addr // 4 + w) % BANKS
+                    banks[b] = banks.get(b, 0) + 1
+            assert max(banks.values()) <= 2, (NT, P, i)
 
 
 @pytest.mark.parametrize("TP,M", [(1, 1), (1, 2), (1, 4), (2, 1), (2, 2), (2, 4), (4, 1),
