@@ -332,8 +332,6 @@ __global__ void __launch_bounds__(kLutrThreads, 1) lutr_kernel(const LutParams p
   };
   prod_settle();
   const uint32_t ring_lane = sbase + static_cast<uint32_t>(threadIdx.x * P);
-  // two or more pieces per row and chunk: a lane whose rotation includes half the chunk reads
-  // the second half's pieces first
   // the row's chunk as NS 8-byte slots: slot i of the registers is read from ring slot
   // (i + li / 8) mod NS, which is the rotation by whole 8-byte slots
   constexpr int NS = NT / 8;
