@@ -395,9 +395,31 @@ bool lutr_fill(int64_t units, int64_t nrb, int ctas, int64_t tau, int64_t* bound
   return u >= units;
 }
 
-// The smallest such cost for `ctas` CTAs (bisection over tau), with its ranges in bounds.
+// The smallest such cost for `ctas` CTAs (1 <= ctas <= kLutrMaxCtas), with its ranges in
+// bounds: bisection between a cost no split meets (each CTA's share of the units plus one
+// build, less one) and one the even split meets (its busiest CTA), so a handful of fills.
+// The last few results are kept per host thread, so repeated calls of a layer skip the search.
 int64_t lutr_partition(int64_t units, int64_t nrb, int ctas, int64_t* bounds) {
-  int64_t lo = kLutrBuildRowBlocks, hi = units + kLutrBuildRowBlocks * (units / nrb + 2);
+  struct Entry {
+    int64_t units = -1, nrb = 0, tau = 0;
+    int ctas = 0;
+    int64_t b[aq::kLutrMaxCtas + 1];
+  };
+  thread_local Entry cache[8];
+  thread_local int next = 0;
+  for (const Entry& e : cache) {
+    if (e.units == units && e.nrb == nrb && e.ctas == ctas) {
+      std::memcpy(bounds, e.b, sizeof(int64_t) * (ctas + 1));
+      return e.tau;
+    }
+  }
+  int64_t hi = 0;
+  for (int b = 0; b < ctas; ++b) {
+    const int64_t u0 = units * b / ctas, u1 = units * (b + 1) / ctas;
+    if (u1 > u0)
+      hi = std::max(hi, u1 - u0 + kLutrBuildRowBlocks * ((u1 - 1) / nrb - u0 / nrb + 1));
+  }
+  int64_t lo = (units + ctas - 1) / ctas + kLutrBuildRowBlocks - 1;
   while (lo + 1 < hi) {
     const int64_t mid = lo + (hi - lo) / 2;
     if (lutr_fill(units, nrb, ctas, mid, bounds))
@@ -406,6 +428,13 @@ int64_t lutr_partition(int64_t units, int64_t nrb, int ctas, int64_t* bounds) {
       lo = mid;
   }
   lutr_fill(units, nrb, ctas, hi, bounds);
+  Entry& e = cache[next];
+  next = (next + 1) % 8;
+  e.units = units;
+  e.nrb = nrb;
+  e.ctas = ctas;
+  e.tau = hi;
+  std::memcpy(e.b, bounds, sizeof(int64_t) * (ctas + 1));
   return hi;
 }
 
